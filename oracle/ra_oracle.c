@@ -1,0 +1,236 @@
+/*
+ * ra_oracle.c -- the CPU oracle for Random Attention's decode hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the slow, plain, single-threaded
+ * statement of what the GPU library computes.  Only the tests, the smoke
+ * check and the benchmark's CPU-baseline leg may load it; the product path
+ * never does.  It shares no code, header, table or helper with the CUDA
+ * library: everything below is written out from the paper (and, for the
+ * counter-based generator, from its published definition).
+ *
+ * What it states:
+ *   - Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers:
+ *     as easy as 1, 2, 3", SC'11): the per-candidate random score.
+ *   - Random Attention's selection (paper section 3): every evictable
+ *     candidate gets an i.i.d. uniform score, the K best are kept
+ *     (Eq. 1, section 2 "Periodic eviction with budget K and buffer r").
+ *     Scores are 32-bit Philox words; "best" = smallest (key, ordinal),
+ *     which draws a uniform K-subset exactly as a real-valued
+ *     Uniform(0,1) top-K does.
+ *   - The periodic trigger and the chronological compaction
+ *     (section 2 and Appendix F "Engine details": every r steps, once the
+ *     cache exceeds the budget plus the buffer; keep-sets sorted
+ *     chronologically before the gather).
+ *   - Decode attention o = sum_i softmax_i(q.k_i / sqrt(d)) v_i in fp64
+ *     (section 2 "Notation"), grouped-query: a KV head's keep-set serves
+ *     every query head of its group (Appendix F).
+ *
+ * Parity status: every function here is pinned by the "not gpu" tests
+ * (Philox against an independent Philox implementation, selection by brute
+ * force and by the paper's closed-form survival law, attention by closed
+ * forms and an independent library softmax).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ------------------------------------------------------------------------- */
+/* Philox4x32-10 (SC'11, section 3.3 of that paper).                          */
+/* Round: two 32x32->64 multiplies by fixed multipliers, the high halves     */
+/* xored with the other two words and the round key; the key is bumped by    */
+/* two Weyl constants between rounds.                                        */
+/* ------------------------------------------------------------------------- */
+#define PHILOX_M4x32_0 0xD2511F53u
+#define PHILOX_M4x32_1 0xCD9E8D57u
+#define PHILOX_W32_0 0x9E3779B9u /* golden ratio */
+#define PHILOX_W32_1 0xBB67AE85u /* sqrt(3) - 1 */
+
+void ora_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4])
+{
+    uint32_t x0 = ctr[0], x1 = ctr[1], x2 = ctr[2], x3 = ctr[3];
+    uint32_t k0 = key[0], k1 = key[1];
+    for (int round = 0; round < 10; ++round) {
+        if (round > 0) {
+            k0 += PHILOX_W32_0;
+            k1 += PHILOX_W32_1;
+        }
+        uint64_t p0 = (uint64_t)PHILOX_M4x32_0 * (uint64_t)x0;
+        uint64_t p1 = (uint64_t)PHILOX_M4x32_1 * (uint64_t)x2;
+        uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
+        uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
+        uint32_t y0 = hi1 ^ x1 ^ k0;
+        uint32_t y1 = lo1;
+        uint32_t y2 = hi0 ^ x3 ^ k1;
+        uint32_t y3 = lo0;
+        x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+    }
+    out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+/*
+ * The random score of one candidate (section 3: s_i ~ Uniform(0,1), drawn
+ * independently per KV head at every eviction).  The paper does not fix a
+ * generator; this library's mapping is
+ *     counter = (j, step, layer, head_id),  key = (seed_lo, seed_hi),
+ *     score   = word 0 of Philox4x32-10,
+ * with j the candidate's ordinal in slot order, step = number of generated
+ * tokens appended when the eviction fires, and head_id = seq * kv_heads + h.
+ */
+uint32_t ora_random_key(uint64_t seed, uint32_t layer, uint32_t head_id, uint32_t step, uint32_t j)
+{
+    uint32_t ctr[4] = {j, step, layer, head_id};
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t out[4];
+    ora_philox4x32_10(ctr, key, out);
+    return out[0];
+}
+
+/* ------------------------------------------------------------------------- */
+/* Selection: Eq. 1, S_t = top-K over the candidates of s_i.                 */
+/* ------------------------------------------------------------------------- */
+typedef struct {
+    uint32_t key;
+    int32_t ordinal;
+} ora_cand;
+
+static int ora_cmp_cand(const void* a, const void* b)
+{
+    const ora_cand* x = (const ora_cand*)a;
+    const ora_cand* y = (const ora_cand*)b;
+    if (x->key != y->key) return x->key < y->key ? -1 : 1;
+    return x->ordinal < y->ordinal ? -1 : (x->ordinal > y->ordinal ? 1 : 0);
+}
+
+static int ora_cmp_i32(const void* a, const void* b)
+{
+    int32_t x = *(const int32_t*)a, y = *(const int32_t*)b;
+    return x < y ? -1 : (x > y ? 1 : 0);
+}
+
+/*
+ * Keep the K candidates with the smallest (key, ordinal), returned in
+ * ascending ordinal order ("keep-sets are sorted chronologically before
+ * compaction", Appendix F).  The plain definition: sort all, take K.
+ * Returns 0, or -1 on bad arguments / allocation failure.
+ */
+int ora_select_keep(const uint32_t* keys, int n, int K, int32_t* keep_out)
+{
+    if (n < 0 || K < 0 || K > n) return -1;
+    if (K == 0) return 0;
+    ora_cand* c = (ora_cand*)malloc(sizeof(ora_cand) * (size_t)n);
+    if (!c) return -1;
+    for (int j = 0; j < n; ++j) {
+        c[j].key = keys[j];
+        c[j].ordinal = j;
+    }
+    qsort(c, (size_t)n, sizeof(ora_cand), ora_cmp_cand);
+    for (int i = 0; i < K; ++i) keep_out[i] = c[i].ordinal;
+    free(c);
+    qsort(keep_out, (size_t)K, sizeof(int32_t), ora_cmp_i32);
+    return 0;
+}
+
+/*
+ * The periodic trigger (section 2: "the buffer fills every r steps and
+ * triggers an eviction"; Appendix F: "every r=64 decode steps, once the
+ * cache exceeds K+r").  `c` counts the cached generated tokens, `g` the
+ * generated tokens appended so far; the check runs after the step's append.
+ * Fires iff g is a multiple of r and the candidates (everything but the
+ * newest r) outnumber the budget.
+ */
+int ora_should_evict(int g, int c, int K, int r)
+{
+    return (r > 0) && (g > 0) && (g % r == 0) && (c - r > K);
+}
+
+/*
+ * One eviction round for one (sequence, layer, KV head).
+ *   gen[0..*c)  positions of the cached generated tokens, in slot order
+ *               (ascending position); the prompt is not in this list -- it is
+ *               never a candidate (section 3, "Protect the question").
+ * If the trigger fires: candidates are gen[0 .. c-r) (everything outside the
+ * recent buffer), each gets its Philox score, the K smallest survive, and
+ * gen becomes kept-candidates ++ the r buffer positions, in order.
+ * evicted_out (may be NULL) receives the m evicted ordinals, ascending.
+ * Returns m (0 when the trigger does not fire), or -1 on error.
+ */
+int ora_evict_head(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int layer,
+                   int head_id, int32_t* evicted_out)
+{
+    int cc = *c;
+    if (!ora_should_evict(g, cc, K, r)) return 0;
+    int n = cc - r;
+    uint32_t* keys = (uint32_t*)malloc(sizeof(uint32_t) * (size_t)n);
+    int32_t* keep = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
+    int32_t* next = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K + r));
+    if (!keys || !keep || !next) {
+        free(keys); free(keep); free(next);
+        return -1;
+    }
+    for (int j = 0; j < n; ++j)
+        keys[j] = ora_random_key(seed, (uint32_t)layer, (uint32_t)head_id, (uint32_t)g, (uint32_t)j);
+    if (ora_select_keep(keys, n, K, keep) != 0) {
+        free(keys); free(keep); free(next);
+        return -1;
+    }
+    int m = 0, ki = 0;
+    for (int j = 0; j < n; ++j) {
+        if (ki < K && keep[ki] == j) {
+            next[ki] = gen[j];
+            ++ki;
+        } else {
+            if (evicted_out) evicted_out[m] = j;
+            ++m;
+        }
+    }
+    for (int i = 0; i < r; ++i) next[K + i] = gen[n + i];
+    memcpy(gen, next, sizeof(int32_t) * (size_t)(K + r));
+    *c = K + r;
+    free(keys); free(keep); free(next);
+    return m;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Decode attention (section 2, "Notation"), fp64.                           */
+/* ------------------------------------------------------------------------- */
+static double ora_bf16_to_double(uint16_t b)
+{
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/*
+ * o_g = sum_i softmax_i(scale * q_g . k_i) v_i for each query head g of one
+ * GQA group: q [G][d], k and v [n][d] (bf16 bit patterns), out [G][d].
+ * scale <= 0 means 1/sqrt(d).  n == 0 leaves out at zero.
+ */
+void ora_attend(const uint16_t* q, const uint16_t* k, const uint16_t* v, int n, int G, int d,
+                double scale, double* out)
+{
+    if (scale <= 0.0) scale = 1.0 / sqrt((double)d);
+    double* s = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    for (int g = 0; g < G; ++g) {
+        double* o = out + (size_t)g * d;
+        for (int c = 0; c < d; ++c) o[c] = 0.0;
+        if (n == 0 || !s) continue;
+        double mx = -INFINITY;
+        for (int i = 0; i < n; ++i) {
+            double dot = 0.0;
+            for (int c = 0; c < d; ++c)
+                dot += ora_bf16_to_double(q[(size_t)g * d + c]) * ora_bf16_to_double(k[(size_t)i * d + c]);
+            s[i] = scale * dot;
+            if (s[i] > mx) mx = s[i];
+        }
+        double den = 0.0;
+        for (int i = 0; i < n; ++i) {
+            double w = exp(s[i] - mx);
+            den += w;
+            for (int c = 0; c < d; ++c) o[c] += w * ora_bf16_to_double(v[(size_t)i * d + c]);
+        }
+        for (int c = 0; c < d; ++c) o[c] /= den;
+    }
+    free(s);
+}
