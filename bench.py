@@ -1,0 +1,483 @@
+#!/usr/bin/env python3
+"""Decode-throughput benchmark of the Random Attention hot path on GB300.
+
+A step is one decode step of the whole layer stack through the C ABI
+(``ra_decode_step``): for every layer, append the new token's K/V, run the
+periodic random eviction (fires every r steps per sequence), and GQA decode
+attention over the compacted caches.  Caches start at steady state
+(K + r cached generated tokens per head right after an eviction, plus the
+prompt), filled on the device by the seeded generator.
+
+Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle
+(the slow, plain reference of what the path computes) on a bounded sample of
+the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "decode tokens/sec (all layers, 1 GB300) and % of HBM peak GB/s per kernel"
+UNIT = "tokens/s"
+D = 128
+
+
+def _workloads():
+    """The five synthetic workloads (shapes of the paper's models; values from synth)."""
+    w = {
+        1: dict(name="qwen3-4b-shape 1 layer batch 1", L=1, H=32, KVH=8, B=1, lp=[128], K=256, r=64, gen=[1024],
+                key_scale=False, dseed=1, eseed=0),
+        2: dict(name="qwen3-4b-shape", L=36, H=32, KVH=8, B=16, lp=[512] * 16, K=2048, r=64, gen=[32768] * 16,
+                key_scale=True, dseed=2, eseed=2),
+        3: dict(name="qwen3-14b-shape", L=40, H=40, KVH=8, B=64, lp=[2048] * 64, K=4096, r=64, gen=[32768] * 64,
+                key_scale=False, dseed=3, eseed=3),
+        4: dict(name="qwen3-32b-shape", L=64, H=64, KVH=8, B=32, lp=[1024] * 32, K=8192, r=64, gen=[32768] * 32,
+                key_scale=False, dseed=4, eseed=4),
+    }
+    lp5 = synth.uniform_ints(5, 48, 256, 4096).tolist()
+    gen5 = synth.uniform_ints(55, 48, 8192, 32768).tolist()
+    w[5] = dict(name="phi-4-reasoning-shape ragged", L=40, H=40, KVH=10, B=48, lp=lp5, K=4096, r=64, gen=gen5,
+                key_scale=False, dseed=5, eseed=5)
+    return w
+
+
+WORKLOADS = _workloads()
+DEFAULT_CONFIG = 2
+
+
+def steady_state(w, rank=0):
+    """Per-sequence (g0, c0): right after an eviction (c0 = K + r) for lock-step configs; with a
+    per-sequence phase in [0, r) for the ragged one.  Positions are the newest c0 generated ones."""
+    K, r, B = w["K"], w["r"], w["B"]
+    if w["B"] == 1 and w["L"] == 1:  # the small config starts empty (full run from step 0)
+        return [0] * B, [0] * B
+    ragged = len(set(w["lp"])) > 1
+    g0, c0 = [], []
+    for b in range(B):
+        if ragged:
+            phase = int(synth.uniform_ints(1000 + b, 1, 0, r - 1)[0])
+            lo_epochs = -(-(K + 2 * r) // r)
+            hi_epochs = max((w["gen"][b] - 2048) // r, lo_epochs)
+            ep = int(synth.uniform_ints(2000 + b, 1, lo_epochs, hi_epochs)[0])
+        else:  # an eviction step at least K + 2r (the first one possible), mid-generation
+            phase, ep = 0, max(8192, -(-(K + 2 * r) // r) * r) // r
+        ge = ep * r
+        g0.append(ge + phase)
+        c0.append(K + r + phase)
+    return g0, c0
+
+
+def describe(w):
+    lp = w["lp"]
+    lp_s = str(lp[0]) if len(set(lp)) == 1 else f"U[256,4096] (mean {np.mean(lp):.0f})"
+    return (f"{w['name']}: {w['L']} layers, {w['H']}q/{w['KVH']}kv heads, d=128, batch {w['B']}, prompt {lp_s}, "
+            f"K={w['K']}, r={w['r']}")
+
+
+class Workload:
+    """Device-side setup of one workload through the public API."""
+
+    def __init__(self, cfg, rank=0, ring=4):
+        import torch
+
+        import paper_2609_03430_gb300 as ra
+        import synth.gpu as sg
+
+        self.torch, self.ra, self.sg = torch, ra, sg
+        self.w = w = WORKLOADS[cfg]
+        self.cfg = cfg
+        self.L, self.H, self.KVH, self.B, self.K, self.r = w["L"], w["H"], w["KVH"], w["B"], w["K"], w["r"]
+        self.G = self.H // self.KVH
+        self.lp = w["lp"]
+        self.dseed = w["dseed"] + 1000003 * rank
+        self.eseed = w["eseed"] + (rank << 32)
+        self.dev = torch.device("cuda", torch.cuda.current_device())
+        self.stream = torch.cuda.current_stream()
+        self.cache = ra.RandomAttentionCache(self.L, self.H, self.KVH, D, self.lp, self.K, self.r, self.eseed)
+        self.ctx = self.cache.ctx
+        self.key_scale = None
+        if w["key_scale"]:
+            self.key_scale = torch.from_numpy(synth.key_channel_scale(self.dseed, self.L, self.KVH, D)).to(self.dev)
+        self.g0, self.c0 = steady_state(w, rank)
+        self._fill()
+        self.ring = ring
+        self._make_inputs(ring)
+
+    def _scale(self, l):
+        return None if self.key_scale is None else self.key_scale[l].contiguous()
+
+    def _fill(self):
+        torch = self.torch
+        B, KVH = self.B, self.KVH
+        maxlp = max(max(self.lp), 1)
+        ppos = torch.full((B, KVH, maxlp), -1, dtype=torch.int32)
+        for b in range(B):
+            ppos[b, :, : self.lp[b]] = torch.arange(self.lp[b], dtype=torch.int32)
+        ppos = ppos.to(self.dev)
+        maxc = max(max(self.c0), 1)
+        gpos = torch.full((B, KVH, maxc), -1, dtype=torch.int32)
+        for b in range(B):
+            c, g = self.c0[b], self.g0[b]
+            gpos[b, :, :c] = torch.arange(self.lp[b] + g - c, self.lp[b] + g, dtype=torch.int32)
+        gpos = gpos.to(self.dev)
+        kp = torch.empty((B, KVH, maxlp, D), dtype=torch.int16, device=self.dev)
+        vp = torch.empty_like(kp)
+        kg = torch.empty((B, KVH, maxc, D), dtype=torch.int16, device=self.dev)
+        vg = torch.empty_like(kg)
+        for l in range(self.L):
+            self.sg.fill_rows(kp, ppos, self.dseed, 0, l, 0, self._scale(l))
+            self.sg.fill_rows(vp, ppos, self.dseed, 1, l, 0)
+            self.ra.ra_prefill(self.ctx, l, kp.data_ptr(), vp.data_ptr(), maxlp)
+            if max(self.c0) > 0:
+                self.sg.fill_rows(kg, gpos, self.dseed, 0, l, 0, self._scale(l))
+                self.sg.fill_rows(vg, gpos, self.dseed, 1, l, 0)
+                self.ra.ra_restore(self.ctx, l, self.g0, self.c0, gpos.data_ptr(), kg.data_ptr(), vg.data_ptr(), maxc)
+        torch.cuda.synchronize()
+        del kp, vp, kg, vg
+
+    def _make_inputs(self, ring):
+        """Device-resident inputs of `ring` distinct steps (cycled): q [L][B][H][d], k/v [L][B][KVH][d]."""
+        torch = self.torch
+        L, B, H, KVH = self.L, self.B, self.H, self.KVH
+        self.q = torch.empty((ring, L, B, H, D), dtype=torch.int16, device=self.dev)
+        self.kn = torch.empty((ring, L, B, KVH, D), dtype=torch.int16, device=self.dev)
+        self.vn = torch.empty_like(self.kn)
+        self.out = torch.empty((L, B, H, D), dtype=torch.int16, device=self.dev)
+        for t in range(ring):
+            qpos = torch.full((B, H, 1), t, dtype=torch.int32, device=self.dev)
+            npos = torch.tensor([[self.lp[b] + self.g0[b] + t] * KVH for b in range(B)], dtype=torch.int32,
+                                device=self.dev).reshape(B, KVH, 1)
+            for l in range(L):
+                self.sg.fill_rows(self.q[t, l].view(B, H, 1, D), qpos, self.dseed, 2, l, 0)
+                self.sg.fill_rows(self.kn[t, l].view(B, KVH, 1, D), npos, self.dseed, 0, l, 0, self._scale(l))
+                self.sg.fill_rows(self.vn[t, l].view(B, KVH, 1, D), npos, self.dseed, 1, l, 0)
+        torch.cuda.synchronize()
+
+    def step(self, t):
+        i = t % self.ring
+        self.ra.ra_decode_step(self.ctx, self.q[i].data_ptr(), self.kn[i].data_ptr(), self.vn[i].data_ptr(),
+                               self.out.data_ptr(), 0.0, self.stream)
+
+    def bytes_per_step(self):
+        """Algorithmic cache bytes read by attention in one step (all layers), at the current state."""
+        tot = 0
+        for b in range(self.B):
+            _, c, _ = self.ra.ra_get_counters(self.ctx, b, 0)
+            tot += self.KVH * (self.lp[b] + c) * 2 * D * 2
+        return tot * self.L
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons (started before, stopped after)."""
+
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        rows = []
+        for ts, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            rows.append((ts, parts))
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["clock samples unavailable"]}
+        inside = [p for ts, p in rows if t0 <= ts <= t1 + 0.15] or [p for ts, p in rows]
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(p[2]) for p in inside if num(p[2]) is not None]
+        mx = [num(p[3]) for p in inside if num(p[3]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for p in inside for i in range(4) if p[6 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(inside)}
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def reduce_over_ranks(ms, units, world):
+    """max of per-rank times, sum of per-rank units (barrier implied by the collectives)."""
+    if world == 1:
+        return ms, units
+    import torch
+    import torch.distributed as dist
+
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    u = torch.tensor([units], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+# --------------------------------------------------------------------------- CPU oracle timing
+def oracle_sample(w, budget_s=12.0, rank=0):
+    """Time the oracle (single-threaded C, fp64) on a bounded slice of the workload: attention for
+    every KV head of one (sequence, layer) at its steady-state length plus one eviction round per
+    head; extrapolated to tokens/s of the full layer stack.  Inputs are generated before timing."""
+    import oracle
+
+    oracle.build()
+    g0, c0 = steady_state(w, rank)
+    b = 0
+    lp, K, r, KVH, G = w["lp"][b], w["K"], w["r"], w["KVH"], w["H"] // w["KVH"]
+    c = max(c0[b], 1) + r // 2  # mean steady-state length between evictions
+    g = max(g0[b], c)
+    pos = np.concatenate([np.arange(lp), lp + g - c + np.arange(c)])
+    heads = []
+    for h in range(KVH):
+        heads.append((synth.q_rows(w["dseed"], 0, b, np.arange(h * G, (h + 1) * G), 0, D),
+                      synth.kv_rows(w["dseed"], 0, 0, b, h, pos, D), synth.kv_rows(w["dseed"], 1, 0, b, h, pos, D)))
+    gen = (lp + np.arange(K + 2 * r)).astype(np.int32)
+    t_attn, n_attn, t_ev, n_ev = 0.0, 0, 0.0, 0
+    t_start = time.perf_counter()
+    while time.perf_counter() - t_start < budget_s or n_attn == 0:
+        for (q, kk, vv) in heads:
+            t0 = time.perf_counter()
+            oracle.attend(q, kk, vv)
+            t_attn += time.perf_counter() - t0
+            n_attn += 1
+        for h in range(KVH):
+            t0 = time.perf_counter()
+            oracle.evict_head(gen, 8192, K, r, w["eseed"], 0, h)
+            t_ev += time.perf_counter() - t0
+            n_ev += 1
+    per_head_step = t_attn / n_attn + (t_ev / n_ev) / r  # eviction every r steps
+    per_token = per_head_step * KVH * w["L"]
+    return {"value": 1.0 / per_token, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": (f"seq 0 of {describe(w)}: {n_attn} KV-head attention passes at length {lp + c} "
+                       f"(fp64, G={G}) and {n_ev} eviction rounds of {K + r} candidates, "
+                       f"{time.perf_counter() - t_start:.1f} s single-threaded; extrapolated x{KVH} heads x "
+                       f"{w['L']} layers per token, eviction amortised over r={r} steps"),
+            "nproc": os.cpu_count()}
+
+
+def run_reference(args, w):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    per_step = []
+    total = args.cpu_seconds if args.cpu_seconds_set else 60.0
+    budget = max(0.05, min(10.0, total / max(1, args.steps + args.warmup)))
+    res = None
+    for i in range(args.warmup + args.steps):
+        res = oracle_sample(w, budget_s=budget)
+        if i >= args.warmup:
+            per_step.append(1.0 / res["value"])
+    ms = 1000.0 * statistics.mean(per_step)
+    value = 1.0 / statistics.mean(per_step)
+    cpu = dict(res)
+    cpu["value"] = value
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(w, args), "cpu_baseline": cpu,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_dict(w, args):
+    return {"workload": describe(w), "config_index": args.config, "batch": w["B"], "layers": w["L"],
+            "q_heads": w["H"], "kv_heads": w["KVH"], "head_dim": D, "K": w["K"], "r": w["r"],
+            "prompt_mean": float(np.mean(w["lp"])), "start": "steady state (K + r cached generated per head)",
+            "l2": "inputs larger than L2 (every step streams the whole cache)", "parallelism": f"replicas x{args.gpus}"}
+
+
+# --------------------------------------------------------------------------- GPU run
+def run_ours(args, w):
+    import torch
+
+    import paper_2609_03430_gb300 as ra
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    wl = Workload(args.config, rank=rank)
+    stream = wl.stream
+    ctx = wl.ctx
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for t in range(args.warmup):
+        wl.step(t)
+    ra.ra_check_device(ctx)
+    attn_bytes_before = wl.bytes_per_step()
+    ra.ra_profile_reset(ctx)
+    ra.ra_profile_enable(ctx, True)
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    wall0 = time.time()
+    e0.record(stream)
+    for t in range(args.warmup, args.warmup + args.steps):
+        wl.step(t)
+    e1.record(stream)
+    barrier()
+    wall1 = time.time()
+    clocks.stop()
+    ms_total = e0.elapsed_time(e1)
+    ra.ra_profile_enable(ctx, False)
+    kern = {}
+    launches = 0
+    for kind, name in enumerate(ra.KERNEL_NAMES):
+        kms, n, by = ra.ra_profile_read(ctx, kind)
+        launches += n
+        if n:
+            kern[name] = {"launches": n, "ms_total": kms, "us_per_launch": 1000.0 * kms / n,
+                          "bytes_per_launch": by / n,
+                          "algorithmic_GBps": (by / (kms * 1e-3) / 1e9) if kms > 0 else None}
+    ra.ra_check_device(ctx)
+
+    ms_step, units = reduce_over_ranks(ms_total / args.steps, float(wl.B), world)
+    value = units / (ms_step * 1e-3)
+
+    # e2e: the same steps with host buffers -- H2D of the step's inputs from pinned memory,
+    # ra_decode_step, D2H of the outputs, all inside the timed region.
+    e2e = None
+    if not args.no_e2e:
+        hq = torch.empty(wl.q[0].shape, dtype=torch.int16).pin_memory()
+        hk = torch.empty(wl.kn[0].shape, dtype=torch.int16).pin_memory()
+        hv = torch.empty(wl.vn[0].shape, dtype=torch.int16).pin_memory()
+        ho = torch.empty(wl.out.shape, dtype=torch.int16).pin_memory()
+        hq.copy_(wl.q[0].cpu()); hk.copy_(wl.kn[0].cpu()); hv.copy_(wl.vn[0].cpu())
+        dq, dk, dv = torch.empty_like(wl.q[0]), torch.empty_like(wl.kn[0]), torch.empty_like(wl.vn[0])
+        barrier()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for t in range(args.steps):
+            dq.copy_(hq, non_blocking=True)
+            dk.copy_(hk, non_blocking=True)
+            dv.copy_(hv, non_blocking=True)
+            ra.ra_decode_step(ctx, dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), wl.out.data_ptr(), 0.0, stream)
+            ho.copy_(wl.out, non_blocking=True)
+        f1.record(stream)
+        barrier()
+        e2e_ms, e2e_units = reduce_over_ranks(f0.elapsed_time(f1) / args.steps, float(wl.B), world)
+        e2e = {"value": e2e_units / (e2e_ms * 1e-3), "unit": UNIT,
+               "h2d_bytes_per_step": int(hq.numel() * 2 + hk.numel() * 2 + hv.numel() * 2),
+               "d2h_bytes_per_step": int(ho.numel() * 2), "ms_per_step": e2e_ms}
+
+    peaks, peak_src = measured_peaks()
+    a = kern.get("attn")
+    roof = None
+    if a:
+        by_launch = a["bytes_per_launch"]
+        achieved = a["algorithmic_GBps"]
+        roof = {"kernel": "attn_kernel (split-K decode attention)", "bound": "hbm", "achieved": achieved,
+                "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+                else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
+                "algorithmic_bytes_per_launch": by_launch, "us_per_launch": a["us_per_launch"],
+                "traffic": args.traffic}
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_dict(w, args),
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "clocks": clocks.summary(wall0, wall1), "kernels": kern,
+                "attn_cache_bytes_per_step": attn_bytes_before}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+    wl.cache.close()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--config", type=int, default=DEFAULT_CONFIG, choices=sorted(WORKLOADS))
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="ncu dram bytes per attention launch (from a committed profile), if current")
+    args = ap.parse_args(argv)
+    args.cpu_seconds_set = any(a.startswith("--cpu-seconds") for a in (argv if argv is not None else sys.argv[1:]))
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    w = WORKLOADS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_ours(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

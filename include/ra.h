@@ -1,0 +1,195 @@
+/*
+ * ra.h -- C ABI of the GB300 (sm_103a) Random Attention decode library.
+ *
+ * Random Attention (arXiv 2609.03430) evicts KV-cache entries during decoding
+ * with no score: the prompt is always kept, the newest r tokens form a buffer
+ * that is never a candidate, and among the older generated tokens every KV head
+ * independently keeps a budget of K drawn uniformly at random (section 3,
+ * applied through Eq. 1 of section 2).  This library owns the per-(sequence,
+ * layer, KV head) caches and runs the decode hot path on the GPU:
+ *
+ *   ra_append_kv    write the step's new post-RoPE K/V          (Appendix F)
+ *   ra_evict        periodic random eviction + compaction       (sections 2-3)
+ *   ra_decode_attn  GQA decode attention over the caches        (section 2)
+ *
+ * Conventions (every entry point):
+ *   - Return RA_OK (0) or a negative RA_ERR_* code; ra_last_error() gives text.
+ *     Argument and state errors are detected on the host before any launch
+ *     and leave the state unchanged.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All calls are
+ *     asynchronous on it and never synchronise, except the debug getters
+ *     (ra_get_*) and ra_check_device, which synchronise that stream.  Issue all
+ *     calls of one context on one stream (or order them yourself).
+ *   - Device pointers are caller-owned and must stay valid until the stream
+ *     work that uses them has finished.  bf16 tensors are passed as uint16_t
+ *     bit patterns.  Every device pointer must be 16-byte aligned.
+ *   - The library never allocates device memory: the caller sizes one arena
+ *     with ra_device_bytes() (e.g. a torch uint8 CUDA tensor) and binds it.
+ *   - head_dim must be 128; G = q_heads / kv_heads must be an integer in
+ *     [1, 8]; query head qh reads KV head qh / G (consecutive grouping; the
+ *     paper's GQA models share a KV head's keep-set across its query group,
+ *     Appendix F).
+ *
+ * Budget convention: K counts the retained *generated* tokens of a head.  The
+ * paper's budget holds the prompt too (prompt entries score +inf, section 3),
+ * so K_paper = prompt_len + K.
+ *
+ * Random draw (the paper fixes none; this is the library's mapping): the score
+ * of candidate j (its ordinal in slot order among the c - r candidates) is
+ * word 0 of Philox4x32-10 (Salmon et al., SC'11) with
+ *     counter = (j, g, layer, seq * kv_heads + kv_head),  key = (seed lo, seed hi),
+ * where g is the number of generated tokens appended when the eviction fires.
+ * The K smallest (score, j) survive.
+ */
+#ifndef RA_H_
+#define RA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RA_OK 0
+#define RA_ERR_INVALID_ARG (-1)    /* bad argument (range, alignment, NULL) */
+#define RA_ERR_STATE (-2)          /* call not valid in the current state (e.g. no arena bound) */
+#define RA_ERR_CAPACITY (-3)       /* append would exceed prompt_len + K + 2r slots (evict not called) */
+#define RA_ERR_CUDA (-4)           /* a CUDA runtime call or launch failed */
+#define RA_ERR_DEVICE_TIMEOUT (-5) /* a kernel gave up a bounded wait and flagged it (ra_check_device) */
+#define RA_ERR_UNSUPPORTED (-6)    /* shape outside what the kernels implement */
+
+#define RA_MAX_BATCH 512
+
+typedef struct ra_ctx ra_ctx;
+
+/* Per-kernel timing classes for ra_profile_read. */
+enum ra_kernel_kind {
+    RA_KERNEL_APPEND = 0,
+    RA_KERNEL_SELECT = 1,
+    RA_KERNEL_COMPACT = 2,
+    RA_KERNEL_ATTN = 3,
+    RA_KERNEL_COMBINE = 4,
+    RA_KERNEL_KINDS = 5
+};
+
+/*
+ * Create a batch-1 context: `layers` layers of `q_heads` query / `kv_heads` KV
+ * heads of size head_dim, a prompt of prompt_len tokens, budget K >= 0 and
+ * buffer r >= 1 (the paper uses r = 64, Appendix F), eviction seed `seed`.
+ * Host-only; bind an arena before any other call.
+ */
+int ra_create(ra_ctx** out, int layers, int q_heads, int kv_heads, int head_dim, int prompt_len, int K, int r,
+              uint64_t seed);
+
+/*
+ * Same for `batch` sequences with their own prompt lengths
+ * (prompt_lens: host array [batch], each >= 0).  batch <= RA_MAX_BATCH.
+ */
+int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int head_dim, int batch,
+                      const int32_t* prompt_lens, int K, int r, uint64_t seed);
+
+/* Bytes of device memory the context needs (caches, tables, scratch). */
+size_t ra_device_bytes(const ra_ctx* ctx);
+
+/*
+ * Bind `bytes` >= ra_device_bytes() of caller-owned device memory (256-byte
+ * aligned) on the current device and initialise the tables on `stream`.
+ * All caches start empty (g = c = 0 for every sequence and layer).
+ */
+int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream);
+
+/*
+ * Fill layer `layer`'s prompt caches: k, v device [batch][kv_heads][row_stride][head_dim],
+ * of which rows [0, prompt_len(seq)) are used; row_stride >= max prompt_len.
+ */
+int ra_prefill(ra_ctx* ctx, int layer, const uint16_t* k, const uint16_t* v, int row_stride, void* stream);
+
+/*
+ * Restore the generated part of layer `layer` (warm start / checkpoint load):
+ * for every sequence b, g_host[b] tokens have been generated and c_host[b]
+ * (<= K + 2r, <= g_host[b]) of them are cached, at positions
+ * pos[b][h][0..c) (device int32 [batch][kv_heads][row_stride], strictly
+ * increasing, in [prompt_len(b), prompt_len(b) + g)) with rows k, v
+ * (device [batch][kv_heads][row_stride][head_dim]).
+ */
+int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_host, const int32_t* pos,
+               const uint16_t* k, const uint16_t* v, int row_stride, void* stream);
+
+/* Mark sequence `seq` active (1) or finished (0); finished ones are skipped by every call. */
+int ra_set_active(ra_ctx* ctx, int seq, int active);
+
+/*
+ * Append the step's new token of every active sequence to layer `layer`:
+ * k_new, v_new device [batch][kv_heads][head_dim] (post-RoPE keys, Appendix F).
+ * The token's position is prompt_len + g; g and c advance by one.
+ * RA_ERR_CAPACITY if a cache already holds K + 2r generated tokens.
+ */
+int ra_append_kv(ra_ctx* ctx, int layer, const uint16_t* k_new, const uint16_t* v_new, void* stream);
+
+/*
+ * Random Attention eviction of layer `layer` (sections 2-3, Appendix F).  Runs
+ * after the step's append.  For every active sequence whose trigger fires --
+ * g is a multiple of r and the candidates (all cached generated tokens but the
+ * newest r) exceed K -- each KV head keeps the K candidates with the smallest
+ * Philox scores (see above), in their original order, followed by the r buffer
+ * tokens; K/V rows and positions are compacted order-preserving.  A no-op for
+ * sequences whose trigger does not fire.  *n_fired (may be NULL) receives the
+ * number of sequences that evicted.
+ */
+int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream);
+
+/*
+ * GQA decode attention of layer `layer` (section 2, "Notation"):
+ * out[b][qh] = sum_i softmax_i(scale * q[b][qh] . k_i) v_i over the prompt and
+ * the cached generated tokens of KV head qh / G.  q, out: device
+ * [batch][q_heads][head_dim] bf16; fp32 accumulation, bf16 round-to-nearest
+ * output.  scale <= 0 means 1/sqrt(head_dim).  Rows of inactive sequences are
+ * not written.
+ */
+int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, float scale, void* stream);
+
+/*
+ * One decode step of the whole layer stack: for l = 0..layers-1,
+ * append(l) -> evict(l) -> decode_attn(l), with q_all [layers][batch][q_heads][d],
+ * k_all / v_all [layers][batch][kv_heads][d], out_all [layers][batch][q_heads][d].
+ */
+int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, const uint16_t* v_all,
+                   uint16_t* out_all, float scale, void* stream);
+
+/* Host-mirrored counters of (seq, layer): generated tokens g, cached generated c, evictions so far. */
+int ra_get_counters(const ra_ctx* ctx, int seq, int layer, int32_t* g, int32_t* c, int32_t* n_evictions);
+
+/* Debug: copy the c cached generated positions of (layer, seq, kv_head) to host (synchronises). */
+int ra_get_positions(ra_ctx* ctx, int layer, int seq, int kv_head, int32_t* host_pos, int capacity, int* n,
+                     void* stream);
+
+/* Debug: copy all rows (prompt, then cached generated) of (layer, seq, kv_head) to host (synchronises). */
+int ra_get_kv(ra_ctx* ctx, int layer, int seq, int kv_head, uint16_t* host_k, uint16_t* host_v, int capacity_rows,
+              int* n_rows, void* stream);
+
+/* Synchronise `stream` and report RA_ERR_DEVICE_TIMEOUT if any kernel flagged a bounded-wait timeout. */
+int ra_check_device(ra_ctx* ctx, void* stream);
+
+/*
+ * Per-kernel accounting.  Launch counts and algorithmic bytes (the bytes each
+ * kernel must move by definition: cache rows read, rows moved, q/out rows) are
+ * always counted; CUDA-event timing of every launch is recorded only while
+ * enabled (ra_profile_enable).  ra_profile_read synchronises on the recorded
+ * events and returns the totals of one ra_kernel_kind since the last reset.
+ */
+int ra_profile_enable(ra_ctx* ctx, int on);
+int ra_profile_read(ra_ctx* ctx, int kind, double* total_ms, int64_t* launches, double* algorithmic_bytes);
+int ra_profile_reset(ra_ctx* ctx);
+
+/* Static message for the last error of ctx (or of the calling thread if ctx is NULL). */
+const char* ra_last_error(const ra_ctx* ctx);
+
+/* Release the context (host memory only; the arena stays the caller's). */
+void ra_destroy(ra_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RA_H_ */

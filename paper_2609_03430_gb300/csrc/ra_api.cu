@@ -1,0 +1,727 @@
+// ra_api.cu -- host side of the C ABI declared in include/ra.h.
+//
+// Owns the host mirror of every per-(layer, sequence) counter, so that trigger
+// decisions (section 2: every r steps once the candidates exceed K), capacity
+// checks and the attention work split are made on the host without reading
+// device memory; the kernels keep identical counters on the device.  No call
+// allocates device memory or synchronises, except the debug getters.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <vector>
+
+#include "ra.h"
+#include "ra_internal.h"
+
+using namespace ra;
+
+namespace {
+
+thread_local std::string g_tls_error = "no error";
+
+constexpr int kMaxSMs = 256;       // partial-buffer sizing bound (the GB300 has 152)
+constexpr int kMaxAttnWarps = 8;   // warps per attention CTA, upper bound
+constexpr int kMinSlotsPerWarp = 64;
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct ProfRec {
+    int kind;
+    cudaEvent_t start, stop;
+    double bytes;
+};
+
+}  // namespace
+
+struct ra_ctx {
+    // shape
+    int L, H, KVH, G, D, B, K, r, Cmax;
+    uint64_t seed;
+    std::vector<int32_t> lp;       // prompt lengths
+    std::vector<int32_t> poff;     // KVH * prefix sum of prompt lengths
+    long long prompt_rows_per_layer = 0;
+    long long total_rows = 0;
+    long long gen_rows = 0;
+    int regions = 0;
+    // arena layout (byte offsets)
+    size_t off_k, off_v, off_pos, off_region, off_spare, off_cnt, off_lp, off_poff, off_plan, off_partial, off_err,
+        bytes;
+    // binding
+    bool bound = false;
+    int device = -1;
+    int sms = 0;
+    uint8_t* arena = nullptr;
+    DevLayout lay{};
+    CUtensorMap tmap_k{}, tmap_v{};
+    // host mirror
+    std::vector<int32_t> g, c, nev;  // [L][B]
+    std::vector<uint8_t> active;     // [B]
+    // profiling
+    bool prof = false;
+    std::vector<ProfRec> pending;
+    std::vector<cudaEvent_t> pool;
+    double prof_ms[RA_KERNEL_KINDS] = {0};
+    int64_t prof_n[RA_KERNEL_KINDS] = {0};
+    double prof_bytes[RA_KERNEL_KINDS] = {0};
+    int64_t launch_n[RA_KERNEL_KINDS] = {0};      // always counted
+    double launch_bytes[RA_KERNEL_KINDS] = {0};
+    std::string err = "no error";
+};
+
+namespace {
+
+int fail(ra_ctx* ctx, int code, const char* fmt, ...) __attribute__((format(printf, 3, 4)));
+int fail(ra_ctx* ctx, int code, const char* fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (ctx) ctx->err = buf;
+    g_tls_error = buf;
+    return code;
+}
+
+int cuda_fail(ra_ctx* ctx, cudaError_t e, const char* what)
+{
+    return fail(ctx, RA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int check_bound(ra_ctx* ctx)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (!ctx->bound) return fail(ctx, RA_ERR_STATE, "no device arena bound (call ra_bind first)");
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev != ctx->device)
+        return fail(ctx, RA_ERR_STATE, "current device %d is not the bound device %d", dev, ctx->device);
+    return RA_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_layer(ra_ctx* ctx, int layer)
+{
+    if (layer < 0 || layer >= ctx->L) return fail(ctx, RA_ERR_INVALID_ARG, "layer %d out of [0, %d)", layer, ctx->L);
+    return RA_OK;
+}
+
+// --- profiling
+cudaEvent_t take_event(ra_ctx* ctx)
+{
+    if (!ctx->pool.empty()) {
+        cudaEvent_t e = ctx->pool.back();
+        ctx->pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+struct ProfScope {
+    ra_ctx* ctx;
+    int kind;
+    double bytes;
+    cudaStream_t s;
+    cudaEvent_t start = nullptr;
+    ProfScope(ra_ctx* c, int k, double b, cudaStream_t st) : ctx(c), kind(k), bytes(b), s(st)
+    {
+        if (ctx->prof) {
+            start = take_event(ctx);
+            cudaEventRecord(start, s);
+        }
+    }
+    void done()
+    {
+        ctx->launch_n[kind] += 1;
+        ctx->launch_bytes[kind] += bytes;
+        if (ctx->prof && start) {
+            cudaEvent_t stop = take_event(ctx);
+            cudaEventRecord(stop, s);
+            ctx->pending.push_back({kind, start, stop, bytes});
+            start = nullptr;
+        }
+    }
+};
+
+int collect_profile(ra_ctx* ctx)
+{
+    for (auto& pr : ctx->pending) {
+        cudaError_t e = cudaEventSynchronize(pr.stop);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "profile event sync");
+        float ms = 0.f;
+        cudaEventElapsedTime(&ms, pr.start, pr.stop);
+        ctx->prof_ms[pr.kind] += ms;
+        ctx->prof_n[pr.kind] += 1;
+        ctx->prof_bytes[pr.kind] += pr.bytes;
+        ctx->pool.push_back(pr.start);
+        ctx->pool.push_back(pr.stop);
+    }
+    ctx->pending.clear();
+    return RA_OK;
+}
+
+// --- tensor maps over the K and V pools
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+int make_tmap(ra_ctx* ctx, CUtensorMap* map, void* base, int box_rows)
+{
+    static EncodeTiledFn encode = nullptr;
+    if (!encode) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess || !fn || q != cudaDriverEntryPointSuccess)
+            return fail(ctx, RA_ERR_CUDA, "cuTensorMapEncodeTiled entry point not available");
+        encode = reinterpret_cast<EncodeTiledFn>(fn);
+    }
+    const cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)ctx->total_rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)kRowBytes};
+    const cuuint32_t box[2] = {(cuuint32_t)kHeadDim, (cuuint32_t)box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(ctx, RA_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return RA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ra_last_error(const ra_ctx* ctx) { return ctx ? ctx->err.c_str() : g_tls_error.c_str(); }
+
+int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int head_dim, int batch,
+                      const int32_t* prompt_lens, int K, int r, uint64_t seed)
+{
+    if (!out) return fail(nullptr, RA_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (layers < 1) return fail(nullptr, RA_ERR_INVALID_ARG, "layers must be >= 1");
+    if (kv_heads < 1 || kv_heads > 32) return fail(nullptr, RA_ERR_INVALID_ARG, "kv_heads must be in [1, 32]");
+    if (q_heads < kv_heads || q_heads % kv_heads != 0)
+        return fail(nullptr, RA_ERR_INVALID_ARG, "q_heads must be a positive multiple of kv_heads");
+    if (q_heads / kv_heads > kMaxG) return fail(nullptr, RA_ERR_UNSUPPORTED, "q_heads / kv_heads must be <= 8");
+    if (head_dim != kHeadDim) return fail(nullptr, RA_ERR_UNSUPPORTED, "head_dim must be 128");
+    if (batch < 1 || batch > RA_MAX_BATCH) return fail(nullptr, RA_ERR_INVALID_ARG, "batch must be in [1, %d]", RA_MAX_BATCH);
+    if (!prompt_lens) return fail(nullptr, RA_ERR_INVALID_ARG, "prompt_lens is NULL");
+    if (K < 0 || r < 1) return fail(nullptr, RA_ERR_INVALID_ARG, "need K >= 0 and r >= 1");
+    if ((long long)K + r > kMaxCandidates) return fail(nullptr, RA_ERR_UNSUPPORTED, "K + r must be <= %d", kMaxCandidates);
+
+    ra_ctx* ctx = new ra_ctx();
+    ctx->L = layers;
+    ctx->H = q_heads;
+    ctx->KVH = kv_heads;
+    ctx->G = q_heads / kv_heads;
+    ctx->D = head_dim;
+    ctx->B = batch;
+    ctx->K = K;
+    ctx->r = r;
+    ctx->Cmax = K + 2 * r;
+    ctx->seed = seed;
+    ctx->lp.assign(prompt_lens, prompt_lens + batch);
+    ctx->poff.resize(batch);
+    long long acc = 0;
+    for (int b = 0; b < batch; ++b) {
+        if (prompt_lens[b] < 0) {
+            delete ctx;
+            return fail(nullptr, RA_ERR_INVALID_ARG, "prompt_lens[%d] < 0", b);
+        }
+        ctx->poff[b] = (int32_t)(acc * kv_heads);
+        acc += prompt_lens[b];
+    }
+    ctx->prompt_rows_per_layer = acc * kv_heads;
+    ctx->regions = (layers + 1) * batch * kv_heads;
+    ctx->gen_rows = (long long)ctx->regions * ctx->Cmax;
+    ctx->total_rows = ctx->prompt_rows_per_layer * layers + ctx->gen_rows;
+    // every slot position and every row index must fit the int32 coordinates the kernels use
+    if (ctx->total_rows >= (1LL << 31) || ctx->prompt_rows_per_layer >= (1LL << 31)) {
+        delete ctx;
+        return fail(nullptr, RA_ERR_UNSUPPORTED, "cache too large for 32-bit row coordinates");
+    }
+    size_t o = 0;
+    auto take = [&](size_t n) {
+        size_t at = o;
+        o = align_up(o + n, kAlign);
+        return at;
+    };
+    const size_t pool_bytes = (size_t)ctx->total_rows * kRowBytes;
+    ctx->off_k = take(pool_bytes);
+    ctx->off_v = take(pool_bytes);
+    ctx->off_pos = take((size_t)ctx->regions * ctx->Cmax * 4);
+    ctx->off_region = take((size_t)layers * batch * kv_heads * 4);
+    ctx->off_spare = take((size_t)batch * kv_heads * 4);
+    ctx->off_cnt = take((size_t)layers * batch * sizeof(DevCounters));
+    ctx->off_lp = take((size_t)batch * 4);
+    ctx->off_poff = take((size_t)batch * 4);
+    ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
+    ctx->off_partial = take((size_t)(kMaxSMs * kMaxAttnWarps + batch * kv_heads) * partial_stride(ctx->G) * 4);
+    ctx->off_err = take(256);
+    ctx->bytes = o;
+    ctx->g.assign((size_t)layers * batch, 0);
+    ctx->c.assign((size_t)layers * batch, 0);
+    ctx->nev.assign((size_t)layers * batch, 0);
+    ctx->active.assign(batch, 1);
+    *out = ctx;
+    return RA_OK;
+}
+
+int ra_create(ra_ctx** out, int layers, int q_heads, int kv_heads, int head_dim, int prompt_len, int K, int r,
+              uint64_t seed)
+{
+    const int32_t lp = prompt_len;
+    if (prompt_len < 0) return fail(nullptr, RA_ERR_INVALID_ARG, "prompt_len < 0");
+    return ra_create_batched(out, layers, q_heads, kv_heads, head_dim, 1, &lp, K, r, seed);
+}
+
+size_t ra_device_bytes(const ra_ctx* ctx) { return ctx ? ctx->bytes : 0; }
+
+int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (!device_arena || (reinterpret_cast<uintptr_t>(device_arena) & (kAlign - 1)))
+        return fail(ctx, RA_ERR_INVALID_ARG, "arena must be a non-NULL 256-byte aligned device pointer");
+    if (bytes < ctx->bytes) return fail(ctx, RA_ERR_INVALID_ARG, "arena has %zu bytes, need %zu", bytes, ctx->bytes);
+    cudaError_t e;
+    cudaPointerAttributes attr{};
+    if ((e = cudaPointerGetAttributes(&attr, device_arena)) != cudaSuccess) return cuda_fail(ctx, e, "arena attributes");
+    if (attr.type != cudaMemoryTypeDevice) return fail(ctx, RA_ERR_INVALID_ARG, "arena is not device memory");
+    int dev = -1;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return cuda_fail(ctx, e, "cudaGetDevice");
+    if (attr.device != dev) return fail(ctx, RA_ERR_INVALID_ARG, "arena lives on device %d, current is %d", attr.device, dev);
+    int sms = 0;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return cuda_fail(ctx, e, "SM count");
+    if (sms > kMaxSMs) return fail(ctx, RA_ERR_UNSUPPORTED, "more than %d SMs", kMaxSMs);
+    cudaStream_t s = (cudaStream_t)stream;
+
+    uint8_t* a = (uint8_t*)device_arena;
+    DevLayout& Ly = ctx->lay;
+    Ly.kpool = (uint16_t*)(a + ctx->off_k);
+    Ly.vpool = (uint16_t*)(a + ctx->off_v);
+    Ly.pos = (int32_t*)(a + ctx->off_pos);
+    Ly.region = (int32_t*)(a + ctx->off_region);
+    Ly.spare = (int32_t*)(a + ctx->off_spare);
+    Ly.counters = (DevCounters*)(a + ctx->off_cnt);
+    Ly.seq_lp = (int32_t*)(a + ctx->off_lp);
+    Ly.seq_poff = (int32_t*)(a + ctx->off_poff);
+    Ly.plan = (int32_t*)(a + ctx->off_plan);
+    Ly.partial = (float*)(a + ctx->off_partial);
+    Ly.err = (int32_t*)(a + ctx->off_err);
+    Ly.prompt_rows_per_layer = ctx->prompt_rows_per_layer;
+    Ly.gen_row0 = ctx->prompt_rows_per_layer * ctx->L;
+    Ly.L = ctx->L;
+    Ly.B = ctx->B;
+    Ly.KVH = ctx->KVH;
+    Ly.H = ctx->H;
+    Ly.G = ctx->G;
+    Ly.Cmax = ctx->Cmax;
+    Ly.K = ctx->K;
+    Ly.r = ctx->r;
+    Ly.seed = ctx->seed;
+
+    // Tables: regions of (layer, seq, head) in order, one spare per (seq, head).
+    const int BH = ctx->B * ctx->KVH;
+    std::vector<int32_t> region((size_t)ctx->L * BH), spare(BH);
+    for (size_t i = 0; i < region.size(); ++i) region[i] = (int32_t)i;
+    for (int i = 0; i < BH; ++i) spare[i] = ctx->L * BH + i;
+    std::vector<DevCounters> cnt((size_t)ctx->L * ctx->B, DevCounters{0, 0, 0, 0});
+    int32_t zero = 0;
+    // Pageable host sources: cudaMemcpyAsync returns once the data is staged, so the vectors may die here.
+    if ((e = cudaMemcpyAsync(Ly.region, region.data(), region.size() * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(Ly.spare, spare.data(), spare.size() * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(Ly.counters, cnt.data(), cnt.size() * sizeof(DevCounters), cudaMemcpyHostToDevice, s)) !=
+            cudaSuccess ||
+        (e = cudaMemcpyAsync(Ly.seq_lp, ctx->lp.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(Ly.seq_poff, ctx->poff.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(ctx, e, "table initialisation");
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(ctx, e, "table initialisation sync");
+
+    const int tile = attn_tile_rows(ctx->G);
+    int rc;
+    if ((rc = make_tmap(ctx, &ctx->tmap_k, Ly.kpool, tile)) != RA_OK) return rc;
+    if ((rc = make_tmap(ctx, &ctx->tmap_v, Ly.vpool, tile)) != RA_OK) return rc;
+    if ((e = attn_prepare(ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
+
+    ctx->arena = a;
+    ctx->device = dev;
+    ctx->sms = sms;
+    ctx->bound = true;
+    std::fill(ctx->g.begin(), ctx->g.end(), 0);
+    std::fill(ctx->c.begin(), ctx->c.end(), 0);
+    std::fill(ctx->nev.begin(), ctx->nev.end(), 0);
+    return RA_OK;
+}
+
+int ra_prefill(ra_ctx* ctx, int layer, const uint16_t* k, const uint16_t* v, int row_stride, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!k || !v || !aligned16(k) || !aligned16(v)) return fail(ctx, RA_ERR_INVALID_ARG, "k/v must be 16-byte aligned");
+    int maxlp = 0;
+    for (int b = 0; b < ctx->B; ++b) maxlp = std::max(maxlp, (int)ctx->lp[b]);
+    if (row_stride < maxlp) return fail(ctx, RA_ERR_INVALID_ARG, "row_stride %d < max prompt length %d", row_stride, maxlp);
+    if (maxlp == 0) return RA_OK;
+    CopyRowsParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    p.k = k;
+    p.v = v;
+    p.row_stride = row_stride;
+    for (int b = 0; b < ctx->B; ++b) p.n_rows[b] = ctx->lp[b];
+    cudaError_t e = launch_prefill(p, (cudaStream_t)stream);
+    return e == cudaSuccess ? RA_OK : cuda_fail(ctx, e, "prefill launch");
+}
+
+int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_host, const int32_t* pos,
+               const uint16_t* k, const uint16_t* v, int row_stride, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!g_host || !c_host || !pos || !k || !v) return fail(ctx, RA_ERR_INVALID_ARG, "NULL argument");
+    if (!aligned16(k) || !aligned16(v)) return fail(ctx, RA_ERR_INVALID_ARG, "k/v must be 16-byte aligned");
+    int maxc = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (c_host[b] < 0 || c_host[b] > ctx->Cmax || c_host[b] > g_host[b])
+            return fail(ctx, RA_ERR_INVALID_ARG, "seq %d: need 0 <= c <= min(g, K + 2r)", b);
+        maxc = std::max(maxc, (int)c_host[b]);
+    }
+    if (row_stride < maxc) return fail(ctx, RA_ERR_INVALID_ARG, "row_stride %d < max c %d", row_stride, maxc);
+    cudaStream_t s = (cudaStream_t)stream;
+    CopyRowsParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    p.k = k;
+    p.v = v;
+    p.pos = pos;
+    p.row_stride = row_stride;
+    std::vector<DevCounters> cnt(ctx->B);
+    for (int b = 0; b < ctx->B; ++b) {
+        p.n_rows[b] = c_host[b];
+        cnt[b] = DevCounters{c_host[b], g_host[b], ctx->nev[(size_t)layer * ctx->B + b], 0};
+    }
+    cudaError_t e;
+    if (maxc > 0 && (e = launch_restore(p, s)) != cudaSuccess) return cuda_fail(ctx, e, "restore launch");
+    if ((e = cudaMemcpyAsync(ctx->lay.counters + (size_t)layer * ctx->B, cnt.data(), cnt.size() * sizeof(DevCounters),
+                             cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(ctx, e, "restore counters");
+    for (int b = 0; b < ctx->B; ++b) {
+        ctx->g[(size_t)layer * ctx->B + b] = g_host[b];
+        ctx->c[(size_t)layer * ctx->B + b] = c_host[b];
+    }
+    return RA_OK;
+}
+
+int ra_set_active(ra_ctx* ctx, int seq, int active)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (seq < 0 || seq >= ctx->B) return fail(ctx, RA_ERR_INVALID_ARG, "seq %d out of range", seq);
+    ctx->active[seq] = active ? 1 : 0;
+    return RA_OK;
+}
+
+static void fill_active(const ra_ctx* ctx, uint32_t* mask)
+{
+    for (int i = 0; i < RA_MAX_BATCH / 32; ++i) mask[i] = 0;
+    for (int b = 0; b < ctx->B; ++b)
+        if (ctx->active[b]) mask[b >> 5] |= 1u << (b & 31);
+}
+
+int ra_append_kv(ra_ctx* ctx, int layer, const uint16_t* k_new, const uint16_t* v_new, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new))
+        return fail(ctx, RA_ERR_INVALID_ARG, "k_new/v_new must be non-NULL and 16-byte aligned");
+    int n_active = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (!ctx->active[b]) continue;
+        ++n_active;
+        if (ctx->c[(size_t)layer * ctx->B + b] >= ctx->Cmax)
+            return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d already caches K + 2r = %d generated tokens", layer, b,
+                        ctx->Cmax);
+    }
+    if (n_active == 0) return RA_OK;
+    AppendParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    p.k_new = k_new;
+    p.v_new = v_new;
+    fill_active(ctx, p.active);
+    cudaStream_t s = (cudaStream_t)stream;
+    ProfScope ps(ctx, RA_KERNEL_APPEND, 2.0 * n_active * ctx->KVH * kRowBytes * 2, s);
+    cudaError_t e = launch_append(p, ctx->B, s);
+    ps.done();
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");
+    for (int b = 0; b < ctx->B; ++b) {
+        if (!ctx->active[b]) continue;
+        ctx->c[(size_t)layer * ctx->B + b] += 1;
+        ctx->g[(size_t)layer * ctx->B + b] += 1;
+    }
+    return RA_OK;
+}
+
+int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
+{
+    int rc;
+    if (n_fired) *n_fired = 0;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    EvictParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    int n = 0;
+    double moved = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (!ctx->active[b]) continue;
+        const int g = ctx->g[(size_t)layer * ctx->B + b], c = ctx->c[(size_t)layer * ctx->B + b];
+        // section 2 / Appendix F trigger: every r steps, once the candidates exceed the budget
+        if (g > 0 && g % ctx->r == 0 && c - ctx->r > ctx->K) {
+            p.trig[n++] = (int16_t)b;
+            moved += (double)(ctx->K + ctx->r) * ctx->KVH;
+        }
+    }
+    if (n == 0) return RA_OK;
+    p.n_trig = n;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e;
+    {
+        ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
+        e = launch_select(p, s);
+        ps.done();
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
+    {
+        ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
+        e = launch_compact(p, s);
+        ps.done();
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
+    for (int i = 0; i < n; ++i) {
+        const int b = p.trig[i];
+        ctx->c[(size_t)layer * ctx->B + b] = ctx->K + ctx->r;
+        ctx->nev[(size_t)layer * ctx->B + b] += 1;
+    }
+    if (n_fired) *n_fired = n;
+    return RA_OK;
+}
+
+int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, float scale, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!q || !out || !aligned16(q) || !aligned16(out))
+        return fail(ctx, RA_ERR_INVALID_ARG, "q/out must be non-NULL and 16-byte aligned");
+    AttnParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    p.q = q;
+    p.out = out;
+    fill_active(ctx, p.active);
+    long long acc = 0;
+    int n_active = 0;
+    p.seq_base[0] = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (ctx->active[b]) {
+            acc += (long long)ctx->KVH * (ctx->lp[b] + ctx->c[(size_t)layer * ctx->B + b]);
+            ++n_active;
+        }
+        p.seq_base[b + 1] = (int32_t)acc;
+    }
+    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 slots");
+    if (n_active == 0) return RA_OK;
+    const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)kHeadDim);
+    p.qk_scale_log2 = sc * 1.4426950408889634f;
+    p.total = (int)acc;
+    const int wpc = attn_warps_per_cta(ctx->G);
+    const long long nwarps_max = (long long)ctx->sms * wpc;
+    long long W = (acc + nwarps_max - 1) / nwarps_max;
+    if (W < kMinSlotsPerWarp) W = kMinSlotsPerWarp;
+    p.W = (int)W;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e;
+    if (acc > 0) {
+        const long long warps = (acc + W - 1) / W;
+        const int ctas = (int)((warps + wpc - 1) / wpc);
+        ProfScope ps(ctx, RA_KERNEL_ATTN, (double)acc * 2 * kRowBytes + (double)n_active * ctx->H * kRowBytes, s);
+        e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+        ps.done();
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
+    }
+    {
+        ProfScope ps(ctx, RA_KERNEL_COMBINE, (double)n_active * ctx->H * kRowBytes, s);
+        e = launch_combine(p, s);
+        ps.done();
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "combine launch");
+    return RA_OK;
+}
+
+int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, const uint16_t* v_all, uint16_t* out_all,
+                   float scale, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if (!q_all || !k_all || !v_all || !out_all) return fail(ctx, RA_ERR_INVALID_ARG, "NULL argument");
+    // validate every layer's capacity first so that a failing step changes nothing
+    for (int l = 0; l < ctx->L; ++l)
+        for (int b = 0; b < ctx->B; ++b)
+            if (ctx->active[b] && ctx->c[(size_t)l * ctx->B + b] >= ctx->Cmax)
+                return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d is full (evict not called)", l, b);
+    const size_t qs = (size_t)ctx->B * ctx->H * kHeadDim, ks = (size_t)ctx->B * ctx->KVH * kHeadDim;
+    for (int l = 0; l < ctx->L; ++l) {
+        if ((rc = ra_append_kv(ctx, l, k_all + l * ks, v_all + l * ks, stream)) != RA_OK) return rc;
+        if ((rc = ra_evict(ctx, l, nullptr, stream)) != RA_OK) return rc;
+        if ((rc = ra_decode_attn(ctx, l, q_all + l * qs, out_all + l * qs, scale, stream)) != RA_OK) return rc;
+    }
+    return RA_OK;
+}
+
+int ra_get_counters(const ra_ctx* ctx, int seq, int layer, int32_t* g, int32_t* c, int32_t* n_evictions)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (seq < 0 || seq >= ctx->B || layer < 0 || layer >= ctx->L)
+        return fail(const_cast<ra_ctx*>(ctx), RA_ERR_INVALID_ARG, "seq/layer out of range");
+    const size_t i = (size_t)layer * ctx->B + seq;
+    if (g) *g = ctx->g[i];
+    if (c) *c = ctx->c[i];
+    if (n_evictions) *n_evictions = ctx->nev[i];
+    return RA_OK;
+}
+
+static int read_region(ra_ctx* ctx, int layer, int seq, int kv_head, int32_t* reg, cudaStream_t s)
+{
+    cudaError_t e;
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(ctx, e, "stream sync");
+    if ((e = cudaMemcpy(reg, ctx->lay.region + ((size_t)layer * ctx->B + seq) * ctx->KVH + kv_head, 4,
+                        cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_fail(ctx, e, "region read");
+    return RA_OK;
+}
+
+int ra_get_positions(ra_ctx* ctx, int layer, int seq, int kv_head, int32_t* host_pos, int capacity, int* n,
+                     void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (seq < 0 || seq >= ctx->B || kv_head < 0 || kv_head >= ctx->KVH || !n)
+        return fail(ctx, RA_ERR_INVALID_ARG, "seq/kv_head out of range or n NULL");
+    const int c = ctx->c[(size_t)layer * ctx->B + seq];
+    *n = c;
+    if (capacity < c || (c > 0 && !host_pos)) return fail(ctx, RA_ERR_INVALID_ARG, "capacity %d < %d", capacity, c);
+    int32_t reg;
+    if ((rc = read_region(ctx, layer, seq, kv_head, &reg, (cudaStream_t)stream)) != RA_OK) return rc;
+    cudaError_t e;
+    if (c > 0 && (e = cudaMemcpy(host_pos, ctx->lay.pos + (size_t)reg * ctx->Cmax, (size_t)c * 4,
+                                 cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_fail(ctx, e, "positions read");
+    return RA_OK;
+}
+
+int ra_get_kv(ra_ctx* ctx, int layer, int seq, int kv_head, uint16_t* host_k, uint16_t* host_v, int capacity_rows,
+              int* n_rows, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (seq < 0 || seq >= ctx->B || kv_head < 0 || kv_head >= ctx->KVH || !n_rows)
+        return fail(ctx, RA_ERR_INVALID_ARG, "seq/kv_head out of range or n_rows NULL");
+    const int lp = ctx->lp[seq], c = ctx->c[(size_t)layer * ctx->B + seq];
+    *n_rows = lp + c;
+    if (capacity_rows < lp + c || !host_k || !host_v)
+        return fail(ctx, RA_ERR_INVALID_ARG, "capacity %d < %d rows", capacity_rows, lp + c);
+    int32_t reg;
+    if ((rc = read_region(ctx, layer, seq, kv_head, &reg, (cudaStream_t)stream)) != RA_OK) return rc;
+    const long long prow = (long long)layer * ctx->prompt_rows_per_layer + ctx->poff[seq] + (long long)kv_head * lp;
+    const long long grow = ctx->lay.gen_row0 + (long long)reg * ctx->Cmax;
+    cudaError_t e;
+    for (int w = 0; w < 2; ++w) {
+        const uint16_t* pool = w ? ctx->lay.vpool : ctx->lay.kpool;
+        uint16_t* dst = w ? host_v : host_k;
+        if (lp > 0 && (e = cudaMemcpy(dst, pool + prow * kHeadDim, (size_t)lp * kRowBytes, cudaMemcpyDeviceToHost)) !=
+                          cudaSuccess)
+            return cuda_fail(ctx, e, "prompt rows read");
+        if (c > 0 && (e = cudaMemcpy(dst + (size_t)lp * kHeadDim, pool + grow * kHeadDim, (size_t)c * kRowBytes,
+                                     cudaMemcpyDeviceToHost)) != cudaSuccess)
+            return cuda_fail(ctx, e, "generated rows read");
+    }
+    return RA_OK;
+}
+
+int ra_check_device(ra_ctx* ctx, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    cudaError_t e;
+    if ((e = cudaStreamSynchronize((cudaStream_t)stream)) != cudaSuccess) return cuda_fail(ctx, e, "stream sync");
+    int32_t w = 0;
+    if ((e = cudaMemcpy(&w, ctx->lay.err, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(ctx, e, "err read");
+    if (w == kDeviceErrTimeout) return fail(ctx, RA_ERR_DEVICE_TIMEOUT, "a kernel gave up a bounded wait");
+    if (w == kDeviceErrPlan) return fail(ctx, RA_ERR_STATE, "device eviction plan inconsistent with host counters");
+    if (w != 0) return fail(ctx, RA_ERR_STATE, "device error word %d", w);
+    return RA_OK;
+}
+
+int ra_profile_enable(ra_ctx* ctx, int on)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    ctx->prof = on != 0;
+    return RA_OK;
+}
+
+int ra_profile_reset(ra_ctx* ctx)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    int rc = collect_profile(ctx);
+    for (int k = 0; k < RA_KERNEL_KINDS; ++k) {
+        ctx->prof_ms[k] = 0;
+        ctx->prof_n[k] = 0;
+        ctx->prof_bytes[k] = 0;
+        ctx->launch_n[k] = 0;
+        ctx->launch_bytes[k] = 0;
+    }
+    return rc;
+}
+
+int ra_profile_read(ra_ctx* ctx, int kind, double* total_ms, int64_t* launches, double* algorithmic_bytes)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (kind < 0 || kind >= RA_KERNEL_KINDS) return fail(ctx, RA_ERR_INVALID_ARG, "bad kernel kind %d", kind);
+    int rc = collect_profile(ctx);
+    if (rc != RA_OK) return rc;
+    if (total_ms) *total_ms = ctx->prof_ms[kind];
+    if (launches) *launches = ctx->launch_n[kind];
+    if (algorithmic_bytes) *algorithmic_bytes = ctx->launch_bytes[kind];
+    return RA_OK;
+}
+
+void ra_destroy(ra_ctx* ctx)
+{
+    if (!ctx) return;
+    for (auto& pr : ctx->pending) {
+        cudaEventSynchronize(pr.stop);
+        cudaEventDestroy(pr.start);
+        cudaEventDestroy(pr.stop);
+    }
+    for (auto e : ctx->pool) cudaEventDestroy(e);
+    delete ctx;
+}
+
+}  // extern "C"

@@ -1,0 +1,359 @@
+// ra_evict.cu -- cache writes and Random Attention eviction on sm_103a.
+//
+//   append_kernel   one warp per (seq, KV head): the step's post-RoPE K/V row
+//                   and its position go to slot c of the head's region
+//                   (Appendix F: keys stored post-RoPE, cumulative counter).
+//   select_kernel   one CTA per triggered (seq, KV head): Philox4x32-10 score
+//                   per candidate (section 3's i.i.d. uniform draw), radix
+//                   select of the K smallest (score, ordinal) -- Eq. 1 -- and a
+//                   ballot-compacted, ascending list of the evicted ordinals.
+//   compact_kernel  many CTAs per triggered head: order-preserving move of the
+//                   survivors (kept candidates, then the r-token buffer) into
+//                   the head's spare region with coalesced 16-byte copies
+//                   ("keep-sets sorted chronologically ... compacted with a
+//                   gather", Appendix F).  Out of place, so CTAs never wait on
+//                   each other; the old region becomes the spare.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ra_internal.h"
+#include "ra_ptx.cuh"
+
+namespace ra {
+namespace {
+
+// Philox4x32-10, Salmon et al. (SC'11): ten rounds of two 32x32->64-bit
+// multiplies; the high halves are xored with the other two counter words and
+// the round key; the key advances by the two Weyl constants between rounds.
+// Returns word 0 of the output block.
+__device__ __forceinline__ uint32_t philox4x32_10_w0(uint32_t x0, uint32_t x1, uint32_t x2, uint32_t x3,
+                                                     uint32_t k0, uint32_t k1)
+{
+#pragma unroll
+    for (int round = 0; round < 10; ++round) {
+        const uint32_t p_hi = __umulhi(0xD2511F53u, x0), p_lo = 0xD2511F53u * x0;
+        const uint32_t q_hi = __umulhi(0xCD9E8D57u, x2), q_lo = 0xCD9E8D57u * x2;
+        const uint32_t n0 = q_hi ^ x1 ^ k0;
+        const uint32_t n2 = p_hi ^ x3 ^ k1;
+        x0 = n0;
+        x1 = q_lo;
+        x2 = n2;
+        x3 = p_lo;
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    return x0;
+}
+
+__device__ __forceinline__ bool bit_on(const uint32_t* mask, int b) { return (mask[b >> 5] >> (b & 31)) & 1u; }
+
+// ----------------------------------------------------------------------------- append
+__global__ void __launch_bounds__(1024) append_kernel(const __grid_constant__ AppendParams p)
+{
+    const int b = blockIdx.x;
+    if (!bit_on(p.active, b)) return;
+    const DevLayout& L = p.lay;
+    const int h = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    DevCounters* cnt = L.counters + (size_t)p.layer * L.B + b;
+    const int c = cnt->c, g = cnt->g;
+    const int reg = L.region[((size_t)p.layer * L.B + b) * L.KVH + h];
+    const long long row = L.gen_row0 + (long long)reg * L.Cmax + c;
+    const size_t src = ((size_t)b * L.KVH + h) * kHeadDim;
+    if (lane < 16) {
+        const uint4 v = reinterpret_cast<const uint4*>(p.k_new + src)[lane];
+        reinterpret_cast<uint4*>(L.kpool + row * kHeadDim)[lane] = v;
+    } else {
+        const uint4 v = reinterpret_cast<const uint4*>(p.v_new + src)[lane - 16];
+        reinterpret_cast<uint4*>(L.vpool + row * kHeadDim)[lane - 16] = v;
+    }
+    if (lane == 0) L.pos[(size_t)reg * L.Cmax + c] = L.seq_lp[b] + g;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        cnt->c = c + 1;
+        cnt->g = g + 1;
+    }
+}
+
+// ----------------------------------------------------------------------------- select
+constexpr int kSelThreads = 256;
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ EvictParams p)
+{
+    extern __shared__ uint32_t sm[];
+    __shared__ uint32_t hist[256];
+    __shared__ uint32_t s_bin, s_before, s_total;
+    const DevLayout& L = p.lay;
+    const int b = p.trig[blockIdx.x], h = blockIdx.y;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const DevCounters cnt = L.counters[(size_t)p.layer * L.B + b];
+    const int c = cnt.c, g = cnt.g, K = L.K, r = L.r;
+    const int N = c - r, m = N - K;
+    const int head_id = b * L.KVH + h;
+    int32_t* plan = L.plan + (size_t)head_id * (kPlanHeader + r);
+    if (m <= 0 || m > r || N > kMaxCandidates) {  // the host mirror rules this out; never move data on a bad plan
+        if (tid == 0) {
+            atomicExch(L.err, kDeviceErrPlan);
+            plan[3] = 0;
+        }
+        return;
+    }
+    const int nwords = (N + 31) >> 5;
+    uint32_t* keys = sm;                 // [N]
+    uint32_t* evbits = sm + nwords * 32; // [nwords]
+
+    const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
+    for (int j = tid; j < N; j += kSelThreads)
+        keys[j] = philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)p.layer, (uint32_t)head_id, k0, k1);
+    __syncthreads();
+
+    // Radix select of the element at rank K (0-based) of the (key, ordinal) order:
+    // 8 bits at a time from the top.  Afterwards T is its key and `rank` is its
+    // rank among the keys equal to T, i.e. the number of ties that are kept.
+    uint32_t prefix = 0, mask = 0;
+    uint32_t rank = (uint32_t)K;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        hist[tid] = 0;
+        __syncthreads();
+        for (int j = tid; j < N; j += kSelThreads) {
+            const uint32_t kk = keys[j];
+            if ((kk & mask) == prefix) atomicAdd(&hist[(kk >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (warp == 0) {
+            uint32_t loc[8], sum = 0;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                loc[q] = hist[lane * 8 + q];
+                sum += loc[q];
+            }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += t;
+            }
+            const uint32_t excl = incl - sum;
+            if (excl <= rank && rank < incl) {
+                uint32_t cum = excl;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    if (rank < cum + loc[q]) {
+                        s_bin = (uint32_t)(lane * 8 + q);
+                        s_before = cum;
+                        break;
+                    }
+                    cum += loc[q];
+                }
+            }
+        }
+        __syncthreads();
+        rank -= s_before;
+        prefix |= s_bin << shift;
+        mask |= 255u << shift;
+    }
+    const uint32_t T = prefix;
+    const uint32_t kept_ties = rank;
+
+    // Evicted: key > T, and the ties beyond the first `kept_ties` (in ordinal order).
+    for (int w = warp; w < nwords; w += kSelThreads / 32) {
+        const int j = w * 32 + lane;
+        const bool ev = (j < N) && keys[j] >= T;
+        const uint32_t bits = __ballot_sync(0xffffffffu, ev);
+        if (lane == 0) evbits[w] = bits;
+    }
+    __syncthreads();
+    if (kept_ties > 0 && warp == 0) {  // rare: give the lowest-ordinal ties back to the keep-set
+        uint32_t remaining = kept_ties;
+        for (int w = 0; w < nwords && remaining > 0; ++w) {
+            const int j = w * 32 + lane;
+            const uint32_t eq = __ballot_sync(0xffffffffu, (j < N) && keys[j] == T);
+            uint32_t clear = 0, e = eq;
+            while (e && remaining > 0) {
+                const uint32_t low = e & (~e + 1u);
+                clear |= low;
+                e ^= low;
+                --remaining;
+            }
+            if (lane == 0) evbits[w] &= ~clear;
+        }
+    }
+    __syncthreads();
+
+    // Ascending list of evicted ordinals: warp 0 walks the bitmap 32 words at a time.
+    if (warp == 0) {
+        uint32_t off = 0;
+        for (int base = 0; base < nwords; base += 32) {
+            const int w = base + lane;
+            uint32_t bits = (w < nwords) ? evbits[w] : 0u;
+            const uint32_t cntb = __popc(bits);
+            uint32_t incl = cntb;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += t;
+            }
+            uint32_t pos = off + incl - cntb;
+            while (bits) {
+                const int bit = __ffs(bits) - 1;
+                bits &= bits - 1;
+                if (pos < (uint32_t)r) plan[kPlanHeader + pos] = w * 32 + bit;
+                ++pos;
+            }
+            off += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (lane == 0) s_total = off;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        const int32_t* regp = L.region + ((size_t)p.layer * L.B + b) * L.KVH + h;
+        const int src = *regp, dst = L.spare[b * L.KVH + h];
+        const bool ok = (s_total == (uint32_t)m);
+        plan[0] = src;
+        plan[1] = dst;
+        plan[2] = c;
+        plan[3] = ok ? m : 0;
+        if (ok) {
+            L.region[((size_t)p.layer * L.B + b) * L.KVH + h] = dst;
+            L.spare[b * L.KVH + h] = src;
+        } else {
+            atomicExch(L.err, kDeviceErrPlan);
+        }
+    }
+}
+
+// ----------------------------------------------------------------------------- compact
+constexpr int kCompactThreads = 256;
+constexpr int kCompactUnroll = 4;
+constexpr int kCompactChunk = 256;  // slots per CTA
+
+__global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_constant__ EvictParams p)
+{
+    extern __shared__ int32_t s_ev[];
+    __shared__ int32_t s_hdr[4];
+    const DevLayout& L = p.lay;
+    const int t = blockIdx.y / L.KVH, h = blockIdx.y % L.KVH;
+    const int b = p.trig[t];
+    const int head_id = b * L.KVH + h;
+    const int32_t* plan = L.plan + (size_t)head_id * (kPlanHeader + L.r);
+    if (threadIdx.x < 4) s_hdr[threadIdx.x] = plan[threadIdx.x];
+    __syncthreads();
+    const int src = s_hdr[0], dst = s_hdr[1], c = s_hdr[2], m = s_hdr[3];
+    if (m <= 0) return;  // select flagged a bad plan: region table untouched, nothing moves
+    for (int i = threadIdx.x; i < m; i += kCompactThreads) s_ev[i] = plan[kPlanHeader + i];
+    __syncthreads();
+    const int s0 = blockIdx.x * kCompactChunk;
+    if (s0 >= c) return;
+    const int s1 = min(c, s0 + kCompactChunk);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint16_t* sbase = (lane < 16 ? L.kpool : L.vpool) + (L.gen_row0 + (long long)src * L.Cmax) * kHeadDim;
+    uint16_t* dbase = (lane < 16 ? L.kpool : L.vpool) + (L.gen_row0 + (long long)dst * L.Cmax) * kHeadDim;
+    const int part = lane & 15;
+    const int32_t* spos = L.pos + (size_t)src * L.Cmax;
+    int32_t* dpos = L.pos + (size_t)dst * L.Cmax;
+    for (int base = s0 + warp * kCompactUnroll; base < s1; base += (kCompactThreads / 32) * kCompactUnroll) {
+        uint4 val[kCompactUnroll];
+        int dj[kCompactUnroll];
+        int pv[kCompactUnroll];
+#pragma unroll
+        for (int u = 0; u < kCompactUnroll; ++u) {
+            const int j = base + u;
+            dj[u] = -1;
+            if (j < s1) {
+                int lo = 0, hi = m;  // rank = number of evicted ordinals < j
+                while (lo < hi) {
+                    const int mid = (lo + hi) >> 1;
+                    if (s_ev[mid] < j) lo = mid + 1; else hi = mid;
+                }
+                if (!(lo < m && s_ev[lo] == j)) {
+                    dj[u] = j - lo;
+                    val[u] = __ldg(reinterpret_cast<const uint4*>(sbase + (size_t)j * kHeadDim) + part);
+                    if (lane == 0) pv[u] = __ldg(spos + j);
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kCompactUnroll; ++u) {
+            if (dj[u] >= 0) {
+                reinterpret_cast<uint4*>(dbase + (size_t)dj[u] * kHeadDim)[part] = val[u];
+                if (lane == 0) dpos[dj[u]] = pv[u];
+            }
+        }
+    }
+    if (blockIdx.x == 0 && h == 0 && threadIdx.x == 0) {
+        DevCounters* cnt = L.counters + (size_t)p.layer * L.B + b;
+        cnt->c = c - m;
+        cnt->nev = cnt->nev + 1;
+    }
+}
+
+// ----------------------------------------------------------------------------- prefill / restore
+__global__ void __launch_bounds__(256) copy_rows_kernel(const __grid_constant__ CopyRowsParams p, int restore)
+{
+    const DevLayout& L = p.lay;
+    const int b = blockIdx.x / L.KVH, h = blockIdx.x % L.KVH;
+    const int n = p.n_rows[b];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    long long row0;
+    int32_t* dpos = nullptr;
+    if (restore) {
+        const int reg = L.region[((size_t)p.layer * L.B + b) * L.KVH + h];
+        row0 = L.gen_row0 + (long long)reg * L.Cmax;
+        dpos = L.pos + (size_t)reg * L.Cmax;
+    } else {
+        row0 = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[b] + (long long)h * L.seq_lp[b];
+    }
+    const size_t src0 = ((size_t)b * L.KVH + h) * (size_t)p.row_stride;
+    const uint16_t* sb = (lane < 16 ? p.k : p.v);
+    uint16_t* db = (lane < 16 ? L.kpool : L.vpool);
+    for (int i = warp; i < n; i += 8) {
+        const uint4 v = reinterpret_cast<const uint4*>(sb + (src0 + i) * kHeadDim)[lane & 15];
+        reinterpret_cast<uint4*>(db + (row0 + i) * kHeadDim)[lane & 15] = v;
+        if (restore && lane == 0) dpos[i] = p.pos[src0 + i];
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s)
+{
+    append_kernel<<<B, p.lay.KVH * 32, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+static size_t select_smem(int N) { return ((size_t)((N + 31) / 32) * 32 + (N + 31) / 32) * sizeof(uint32_t); }
+
+cudaError_t launch_select(const EvictParams& p, cudaStream_t s)
+{
+    const int N = p.lay.K + p.lay.r;  // candidates at a firing step never exceed K + r
+    const size_t smem = select_smem(N);
+    static size_t configured = 0;
+    if (smem > 48 * 1024 && smem > configured) {
+        cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = smem;
+    }
+    select_kernel<<<dim3(p.n_trig, p.lay.KVH), kSelThreads, smem, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_compact(const EvictParams& p, cudaStream_t s)
+{
+    const int Cmax = p.lay.Cmax;
+    const int chunks = (Cmax + kCompactChunk - 1) / kCompactChunk;
+    compact_kernel<<<dim3(chunks, p.n_trig * p.lay.KVH), kCompactThreads, p.lay.r * sizeof(int32_t), s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s)
+{
+    copy_rows_kernel<<<p.lay.B * p.lay.KVH, 256, 0, s>>>(p, 0);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s)
+{
+    copy_rows_kernel<<<p.lay.B * p.lay.KVH, 256, 0, s>>>(p, 1);
+    return cudaGetLastError();
+}
+
+}  // namespace ra

@@ -1,0 +1,103 @@
+// ra_internal.h -- launch parameters and launchers shared by the library's own
+// translation units (host API in ra_api.cu; kernels in ra_evict.cu, ra_attn.cu).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ra.h"
+
+namespace ra {
+
+constexpr int kHeadDim = 128;            // d; one K or V row is 256 bytes of bf16
+constexpr int kRowBytes = kHeadDim * 2;
+constexpr int kMaxG = 8;                 // query heads per KV head supported by the kernels
+constexpr int kPlanHeader = 8;           // int32 words before the evicted-ordinal list
+constexpr int kMaxCandidates = 32768;    // K + r bound (select keeps one u32 key per candidate in smem)
+// Split-K partial record of one (warp, KV head) piece: o[G][128], m[G], l[G] in fp32,
+// padded to a multiple of 4 floats so that every record starts 16-byte aligned.
+__host__ __device__ constexpr int partial_stride(int G) { return G * 128 + ((2 * G + 3) / 4) * 4; }
+constexpr int kDeviceErrTimeout = 1;     // values of the device error word
+constexpr int kDeviceErrPlan = 2;
+
+// Device-side per-(layer, seq) counters (mirrored on the host).
+struct DevCounters {
+    int32_t c;    // cached generated tokens
+    int32_t g;    // generated tokens appended
+    int32_t nev;  // evictions so far
+    int32_t pad;
+};
+
+// Pointers into the bound arena plus the static shape of a context.
+struct DevLayout {
+    uint16_t* kpool;       // [total_rows][128] bf16: prompt rows of every layer, then generated regions
+    uint16_t* vpool;
+    int32_t* pos;          // [regions][Cmax] positions of generated slots
+    int32_t* region;       // [L][B][KVH] region index currently holding a head's generated slots
+    int32_t* spare;        // [B][KVH] the free region that a head's next compaction writes into
+    DevCounters* counters; // [L][B]
+    int32_t* seq_lp;       // [B] prompt length
+    int32_t* seq_poff;     // [B] row offset of a sequence's prompt block inside a layer (KVH * sum lp)
+    int32_t* plan;         // [B*KVH][kPlanHeader + r] eviction plan of the current layer
+    float* partial;        // attention split partials
+    int32_t* err;          // device error word
+    long long prompt_rows_per_layer;
+    long long gen_row0;    // first row of the generated regions
+    int L, B, KVH, H, G, Cmax, K, r;
+    uint64_t seed;
+};
+
+struct AppendParams {
+    DevLayout lay;
+    int layer;
+    const uint16_t* k_new;  // [B][KVH][128]
+    const uint16_t* v_new;
+    uint32_t active[RA_MAX_BATCH / 32];
+};
+
+struct EvictParams {
+    DevLayout lay;
+    int layer;
+    int n_trig;
+    int16_t trig[RA_MAX_BATCH];  // triggered sequence ids
+};
+
+struct AttnParams {
+    DevLayout lay;
+    int layer;
+    const uint16_t* q;      // [B][H][128]
+    uint16_t* out;          // [B][H][128] (combine)
+    int W;                  // slots per warp (stream-K split)
+    int total;              // total slots of the layer
+    float qk_scale_log2;    // scale * log2(e)
+    uint32_t active[RA_MAX_BATCH / 32];
+    int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of (lp + c) over active sequences
+};
+
+struct CopyRowsParams {
+    DevLayout lay;
+    int layer;
+    const uint16_t* k;  // [B][KVH][row_stride][128]
+    const uint16_t* v;
+    const int32_t* pos; // restore only: [B][KVH][row_stride]
+    int row_stride;
+    int32_t n_rows[RA_MAX_BATCH];  // rows to copy per sequence
+};
+
+// Launchers (return cudaError_t of the launch).
+cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s);
+cudaError_t launch_select(const EvictParams& p, cudaStream_t s);
+cudaError_t launch_compact(const EvictParams& p, cudaStream_t s);
+cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s);
+cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s);
+
+// Attention: the tensor maps cover kpool / vpool as [total_rows][128] bf16.
+int attn_warps_per_cta(int G);
+int attn_tile_rows(int G);
+cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tmap_k, const CUtensorMap* tmap_v, int ctas,
+                             cudaStream_t s);
+cudaError_t launch_combine(const AttnParams& p, cudaStream_t s);
+cudaError_t attn_prepare(int G);  // one-time function attributes (dynamic smem)
+
+}  // namespace ra

@@ -1,0 +1,84 @@
+"""The C-ABI library loads, exports every symbol include/ra.h declares, and its
+host-side validation works without a GPU (no compute calls here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def ra():
+    from paper_2609_03430_gb300 import _build
+
+    _build.build()
+    import paper_2609_03430_gb300 as ra
+
+    ra.lib()
+    return ra
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "ra.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:[\w\s\*]+?)\b(ra_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_every_declared_symbol_is_exported(ra):
+    names = declared_functions()
+    assert len(names) >= 20, names
+    for n in names:
+        assert hasattr(ra.lib(), n), n
+        assert n in ra.SIGNATURES, f"binding lacks {n}"
+
+
+def test_binding_has_no_undeclared_symbols(ra):
+    assert set(ra.SIGNATURES) == set(declared_functions())
+
+
+def test_create_validation_is_host_only(ra):
+    L = ra.lib()
+    ctx = ctypes.c_void_p()
+    cases = [
+        ((0, 32, 8, 128, 10, 64, 64, 0), ra.RA_ERR_INVALID_ARG),   # layers
+        ((1, 30, 8, 128, 10, 64, 64, 0), ra.RA_ERR_INVALID_ARG),   # q_heads not a multiple
+        ((1, 72, 8, 128, 10, 64, 64, 0), ra.RA_ERR_UNSUPPORTED),   # G = 9
+        ((1, 32, 8, 64, 10, 64, 64, 0), ra.RA_ERR_UNSUPPORTED),    # head_dim
+        ((1, 32, 8, 128, -1, 64, 64, 0), ra.RA_ERR_INVALID_ARG),   # prompt
+        ((1, 32, 8, 128, 10, -1, 64, 0), ra.RA_ERR_INVALID_ARG),   # K
+        ((1, 32, 8, 128, 10, 64, 0, 0), ra.RA_ERR_INVALID_ARG),    # r
+        ((1, 32, 8, 128, 10, 40000, 64, 0), ra.RA_ERR_UNSUPPORTED),  # K + r too large for select
+    ]
+    for args, code in cases:
+        assert L.ra_create(ctypes.byref(ctx), *args) == code, args
+        assert ra.ra_last_error(None)
+    assert L.ra_create(ctypes.byref(ctx), 2, 32, 8, 128, 10, 64, 64, 0) == ra.RA_OK
+    assert ra.ra_device_bytes(ctx) > 0
+    # unbound context: every device call is a state error, detected before any CUDA call
+    assert L.ra_append_kv(ctx, 0, None, None, None) == ra.RA_ERR_STATE
+    assert L.ra_evict(ctx, 0, None, None) == ra.RA_ERR_STATE
+    assert L.ra_decode_attn(ctx, 0, None, None, ctypes.c_float(0), None) == ra.RA_ERR_STATE
+    assert L.ra_bind(ctx, None, 0, None) == ra.RA_ERR_INVALID_ARG
+    assert ra.ra_get_counters(ctx, 0, 1) == (0, 0, 0)
+    ra.ra_destroy(ctx)
+
+
+def test_device_bytes_cover_the_caches(ra):
+    # config-2 shape: 36 layers, 16 seqs, 8 KV heads, prompt 512, K 2048, r 64
+    ctx = ra.ra_create_batched(36, 32, 8, 128, [512] * 16, 2048, 64, 2)
+    rows = 36 * 16 * 8 * 512 + (36 + 1) * 16 * 8 * (2048 + 128)
+    assert ra.ra_device_bytes(ctx) >= 2 * rows * 256 + (36 + 1) * 16 * 8 * (2048 + 128) * 4
+    assert ra.ra_device_bytes(ctx) < 2 * rows * 256 * 1.01 + (64 << 20)
+    ra.ra_destroy(ctx)
+
+
+def test_no_cpu_fallback_in_product_package():
+    """The product package never imports the oracle (test infrastructure)."""
+    pkg = os.path.join(ROOT, "paper_2609_03430_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
+                src = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in src and "from oracle" not in src and "ra_oracle" not in src, f

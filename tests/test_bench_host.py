@@ -1,0 +1,85 @@
+"""Host-side logic of bench.py: workload shapes, steady-state starts, rank reduction (gloo, 2 ranks),
+and the reference (oracle) arm's JSON line."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def test_workloads_match_the_stated_configs():
+    w = bench.WORKLOADS
+    assert (w[1]["L"], w[1]["H"], w[1]["KVH"], w[1]["B"], w[1]["lp"], w[1]["K"], w[1]["r"]) == (1, 32, 8, 1, [128], 256, 64)
+    assert (w[2]["L"], w[2]["H"], w[2]["KVH"], w[2]["B"], w[2]["lp"][0], w[2]["K"]) == (36, 32, 8, 16, 512, 2048)
+    assert w[2]["key_scale"]
+    assert (w[3]["L"], w[3]["H"], w[3]["KVH"], w[3]["B"], w[3]["lp"][0], w[3]["K"]) == (40, 40, 8, 64, 2048, 4096)
+    assert (w[4]["L"], w[4]["H"], w[4]["KVH"], w[4]["B"], w[4]["lp"][0], w[4]["K"]) == (64, 64, 8, 32, 1024, 8192)
+    assert (w[5]["L"], w[5]["H"], w[5]["KVH"], w[5]["B"], w[5]["K"]) == (40, 40, 10, 48, 4096)
+    assert min(w[5]["lp"]) >= 256 and max(w[5]["lp"]) <= 4096 and len(set(w[5]["lp"])) > 10
+    assert min(w[5]["gen"]) >= 8192 and max(w[5]["gen"]) <= 32768
+    assert all(x["r"] == 64 for x in w.values())
+
+
+@pytest.mark.parametrize("cfg", [2, 3, 4, 5])
+def test_steady_state_is_a_reachable_state(cfg):
+    w = bench.WORKLOADS[cfg]
+    g0, c0 = bench.steady_state(w)
+    for g, c, gen in zip(g0, c0, w["gen"]):
+        phase = g % w["r"]
+        assert c == w["K"] + w["r"] + phase  # c right after an eviction, plus the appends since
+        assert g - phase >= w["K"] + 2 * w["r"]  # that eviction step is one the trigger can reach
+        assert g + 2048 <= gen  # the sequence stays active through a benchmark window
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    p = s.getsockname()[1]
+    s.close()
+    return p
+
+
+def _rank_main(rank, world, port, q):
+    import torch.distributed as dist
+
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    ms, units = bench.reduce_over_ranks(10.0 + rank, 16.0, world)
+    q.put((rank, ms, units))
+    dist.destroy_process_group()
+
+
+def test_reduce_over_ranks_gloo_two_ranks():
+    import torch.multiprocessing as mp
+
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    got = sorted(q.get(timeout=10) for _ in range(2))
+    # time = max over ranks, units = sum over ranks (weak scaling: every rank runs its own batch)
+    assert got == [(0, 11.0, 32.0), (1, 11.0, 32.0)]
+
+
+def test_reference_arm_prints_one_json_line():
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "1",
+                          "--steps", "1", "--warmup", "3", "--cpu-seconds", "0.4"],
+                         capture_output=True, text=True, timeout=300, check=True).stdout
+    lines = [l for l in out.splitlines() if l.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["unit"] == "tokens/s" and d["value"] > 0
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
+    assert d["metric"] == bench.METRIC
