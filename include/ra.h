@@ -157,6 +157,24 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
 int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, const uint16_t* v_all,
                    uint16_t* out_all, float scale, void* stream);
 
+/*
+ * Same computation and result as ra_decode_attn, for callers that cannot supply
+ * device scratch memory at call time -- e.g. code that runs while another
+ * framework owns all device allocation, or inside a region where cudaMalloc is
+ * not allowed.  The split-K partials go to a fixed 8 MiB device array inside
+ * this library (one per GPU that loads it, held until the process exits)
+ * instead of the bound arena; this call allocates nothing.  (The paper has no
+ * counterpart: this is an interface convenience.)
+ *   - Layers whose split needs more than 8 MiB of partials (roughly more than
+ *     (8 MiB / (G*128*4 B)) warps-plus-heads) are rejected with RA_ERR_CAPACITY.
+ *   - The first call on a device looks up the array's device address; make that
+ *     first call before any stream capture.
+ *   - Every call shares the one array: calls whose work overlaps on the GPU
+ *     (different streams, or different contexts on one device) race.  Calls
+ *     ordered on one stream are safe; no state is carried between calls.
+ */
+int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, float scale, void* stream);
+
 /* Host-mirrored counters of (seq, layer): generated tokens g, cached generated c, evictions so far. */
 int ra_get_counters(const ra_ctx* ctx, int seq, int layer, int32_t* g, int32_t* c, int32_t* n_evictions);
 

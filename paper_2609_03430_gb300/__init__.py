@@ -45,6 +45,7 @@ SIGNATURES = {
     "ra_append_kv": (_i, [_vp, _i, _vp, _vp, _vp]),
     "ra_evict": (_i, [_vp, _i, _ip, _vp]),
     "ra_decode_attn": (_i, [_vp, _i, _vp, _vp, ctypes.c_float, _vp]),
+    "ra_decode_attn_noalloc": (_i, [_vp, _i, _vp, _vp, ctypes.c_float, _vp]),
     "ra_decode_step": (_i, [_vp, _vp, _vp, _vp, _vp, ctypes.c_float, _vp]),
     "ra_get_counters": (_i, [_vp, _i, _i, _i32p, _i32p, _i32p]),
     "ra_get_positions": (_i, [_vp, _i, _i, _i, _i32p, _i, _ip, _vp]),
@@ -148,6 +149,10 @@ def ra_evict(ctx, layer, stream=None):
 
 def ra_decode_attn(ctx, layer, q_ptr, out_ptr, scale=0.0, stream=None):
     return _check(lib().ra_decode_attn(ctx, layer, q_ptr, out_ptr, float(scale), _stream_ptr(stream)), ctx)
+
+
+def ra_decode_attn_noalloc(ctx, layer, q_ptr, out_ptr, scale=0.0, stream=None):
+    return _check(lib().ra_decode_attn_noalloc(ctx, layer, q_ptr, out_ptr, float(scale), _stream_ptr(stream)), ctx)
 
 
 def ra_decode_step(ctx, q_ptr, k_ptr, v_ptr, out_ptr, scale=0.0, stream=None):

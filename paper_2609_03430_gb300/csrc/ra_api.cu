@@ -14,6 +14,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -725,3 +726,95 @@ void ra_destroy(ra_ctx* ctx)
 }
 
 }  // extern "C"
+
+// ----------------------------------------------------------------------------
+// ra_decode_attn_noalloc: decode attention whose split-K scratch lives in a
+// fixed device array of this library instead of the caller's arena.
+//
+// The array below is allocated by the CUDA module loader when the library is
+// loaded on a device and is held until the process exits.  Host code must not
+// pass the symbol itself to a kernel (on the host it names a shadow, not device
+// memory): its device address is looked up once per device with
+// cudaGetSymbolAddress while that device is current, and that address is what
+// the kernels receive.
+// ----------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = 8u << 20;  // 8 MiB per device
+constexpr int kNoAllocMaxDevices = 64;
+
+static __device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchBytes / sizeof(float)];
+
+std::mutex g_noalloc_mu;
+float* g_noalloc_ptr[kNoAllocMaxDevices] = {nullptr};
+
+int noalloc_scratch(ra_ctx* ctx, int dev, float** out)
+{
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(ctx, RA_ERR_UNSUPPORTED, "device %d out of range", dev);
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) return cuda_fail(ctx, e, "cudaGetSymbolAddress(scratch)");
+        g_noalloc_ptr[dev] = static_cast<float*>(p);
+    }
+    *out = g_noalloc_ptr[dev];
+    return RA_OK;
+}
+
+}  // namespace
+
+extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, float scale,
+                                      void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!q || !out || !aligned16(q) || !aligned16(out))
+        return fail(ctx, RA_ERR_INVALID_ARG, "q/out must be non-NULL and 16-byte aligned");
+    AttnParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    p.q = q;
+    p.out = out;
+    fill_active(ctx, p.active);
+    long long acc = 0;
+    int n_active = 0;
+    p.seq_base[0] = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (ctx->active[b]) {
+            acc += (long long)ctx->KVH * (ctx->lp[b] + ctx->c[(size_t)layer * ctx->B + b]);
+            ++n_active;
+        }
+        p.seq_base[b + 1] = (int32_t)acc;
+    }
+    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 slots");
+    if (n_active == 0) return RA_OK;
+    const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)kHeadDim);
+    p.qk_scale_log2 = sc * 1.4426950408889634f;
+    p.total = (int)acc;
+    const int wpc = attn_warps_per_cta(ctx->G);
+    const long long nwarps_max = (long long)ctx->sms * wpc;
+    long long W = (acc + nwarps_max - 1) / nwarps_max;
+    if (W < kMinSlotsPerWarp) W = kMinSlotsPerWarp;
+    p.W = (int)W;
+    const long long warps = acc > 0 ? (acc + W - 1) / W : 0;
+    // partial records written: one per (warp, head) piece, at index warp + head
+    const size_t need = (size_t)(warps + (long long)ctx->B * ctx->KVH) * partial_stride(ctx->G) * sizeof(float);
+    if (need > kNoAllocScratchBytes)
+        return fail(ctx, RA_ERR_CAPACITY, "layer needs %zu bytes of split-K scratch; the fixed array holds %zu", need,
+                    kNoAllocScratchBytes);
+    float* scratch = nullptr;
+    if ((rc = noalloc_scratch(ctx, ctx->device, &scratch)) != RA_OK) return rc;
+    p.lay.partial = scratch;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e;
+    if (acc > 0) {
+        const int ctas = (int)((warps + wpc - 1) / wpc);
+        e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
+    }
+    e = launch_combine(p, s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "combine launch");
+    return RA_OK;
+}
