@@ -467,6 +467,8 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--layers", type=int, default=None,
+                    help="override the layer count (only to shrink profiler captures; not a benchmark workload)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per attention launch (from a committed profile), if current")
     args = ap.parse_args(argv)
@@ -474,6 +476,9 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     w = WORKLOADS[args.config]
+    if args.layers is not None:
+        w = dict(w, L=args.layers, name=w["name"] + f" (truncated to {args.layers} layers for profiling)")
+        WORKLOADS[args.config] = w
     if args.impl == "reference":
         return run_reference(args, w)
     return run_ours(args, w)

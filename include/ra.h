@@ -69,8 +69,7 @@ enum ra_kernel_kind {
     RA_KERNEL_SELECT = 1,
     RA_KERNEL_COMPACT = 2,
     RA_KERNEL_ATTN = 3,
-    RA_KERNEL_COMBINE = 4,
-    RA_KERNEL_KINDS = 5
+    RA_KERNEL_KINDS = 4
 };
 
 /*
@@ -150,9 +149,23 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream);
 int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, float scale, void* stream);
 
 /*
- * One decode step of the whole layer stack: for l = 0..layers-1,
- * append(l) -> evict(l) -> decode_attn(l), with q_all [layers][batch][q_heads][d],
- * k_all / v_all [layers][batch][kv_heads][d], out_all [layers][batch][q_heads][d].
+ * One decode step of one layer, fused; same result as ra_append_kv ->
+ * ra_evict -> ra_decode_attn with the same arguments.  The eviction runs first
+ * with the step's token pending: the newest slot is never a candidate, so
+ * evicting before writing it leaves the identical cache.  One attention kernel
+ * then writes the new token's row and position, attends over prompt + cache +
+ * new token, and merges its own split pieces.  k_new, v_new: device
+ * [batch][kv_heads][head_dim]; q, out: device [batch][q_heads][head_dim].
+ * RA_ERR_CAPACITY as for ra_append_kv.
+ */
+int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                    uint16_t* out, float scale, void* stream);
+
+/*
+ * One decode step of the whole layer stack: ra_decode_layer for l = 0..layers-1,
+ * with q_all [layers][batch][q_heads][d], k_all / v_all [layers][batch][kv_heads][d],
+ * out_all [layers][batch][q_heads][d].  Capacity is checked for every layer first,
+ * so a step that fails changes nothing.
  */
 int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, const uint16_t* v_all,
                    uint16_t* out_all, float scale, void* stream);

@@ -25,8 +25,8 @@ RA_ERR_CUDA = -4
 RA_ERR_DEVICE_TIMEOUT = -5
 RA_ERR_UNSUPPORTED = -6
 RA_MAX_BATCH = 512
-RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN, RA_KERNEL_COMBINE = range(5)
-KERNEL_NAMES = ["append", "select", "compact", "attn", "combine"]
+RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN = range(4)
+KERNEL_NAMES = ["append", "select", "compact", "attn"]
 
 # Exported C symbols and their ctypes signatures (kept in the order of include/ra.h).
 _vp, _i, _u64, _sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint64, ctypes.c_size_t
@@ -46,6 +46,7 @@ SIGNATURES = {
     "ra_evict": (_i, [_vp, _i, _ip, _vp]),
     "ra_decode_attn": (_i, [_vp, _i, _vp, _vp, ctypes.c_float, _vp]),
     "ra_decode_attn_noalloc": (_i, [_vp, _i, _vp, _vp, ctypes.c_float, _vp]),
+    "ra_decode_layer": (_i, [_vp, _i, _vp, _vp, _vp, _vp, ctypes.c_float, _vp]),
     "ra_decode_step": (_i, [_vp, _vp, _vp, _vp, _vp, ctypes.c_float, _vp]),
     "ra_get_counters": (_i, [_vp, _i, _i, _i32p, _i32p, _i32p]),
     "ra_get_positions": (_i, [_vp, _i, _i, _i, _i32p, _i, _ip, _vp]),
@@ -153,6 +154,11 @@ def ra_decode_attn(ctx, layer, q_ptr, out_ptr, scale=0.0, stream=None):
 
 def ra_decode_attn_noalloc(ctx, layer, q_ptr, out_ptr, scale=0.0, stream=None):
     return _check(lib().ra_decode_attn_noalloc(ctx, layer, q_ptr, out_ptr, float(scale), _stream_ptr(stream)), ctx)
+
+
+def ra_decode_layer(ctx, layer, q_ptr, k_ptr, v_ptr, out_ptr, scale=0.0, stream=None):
+    return _check(lib().ra_decode_layer(ctx, layer, q_ptr, k_ptr, v_ptr, out_ptr, float(scale), _stream_ptr(stream)),
+                  ctx)
 
 
 def ra_decode_step(ctx, q_ptr, k_ptr, v_ptr, out_ptr, scale=0.0, stream=None):

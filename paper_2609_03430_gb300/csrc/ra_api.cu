@@ -53,8 +53,8 @@ struct ra_ctx {
     long long gen_rows = 0;
     int regions = 0;
     // arena layout (byte offsets)
-    size_t off_k, off_v, off_pos, off_region, off_spare, off_cnt, off_lp, off_poff, off_plan, off_partial, off_err,
-        bytes;
+    size_t off_k, off_v, off_pos, off_region, off_spare, off_cnt, off_lp, off_poff, off_plan, off_partial, off_arrive,
+        off_err, bytes;
     // binding
     bool bound = false;
     int device = -1;
@@ -198,6 +198,47 @@ int make_tmap(ra_ctx* ctx, CUtensorMap* map, void* base, int box_rows)
     return RA_OK;
 }
 
+void fill_active(const ra_ctx* ctx, uint32_t* mask)
+{
+    for (int i = 0; i < RA_MAX_BATCH / 32; ++i) mask[i] = 0;
+    for (int b = 0; b < ctx->B; ++b)
+        if (ctx->active[b]) mask[b >> 5] |= 1u << (b & 31);
+}
+
+// Work split of one layer's attention from the host mirror: head lengths (prompt + cached
+// generated rows, + 1 for a fused new token), their prefix, and slots per warp.
+int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas)
+{
+    fill_active(ctx, p->active);
+    long long acc = 0;
+    int na = 0;
+    p->seq_base[0] = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (ctx->active[b]) {
+            acc += (long long)ctx->KVH * (ctx->lp[b] + ctx->c[(size_t)layer * ctx->B + b] + fused);
+            ++na;
+        }
+        p->seq_base[b + 1] = (int32_t)acc;
+    }
+    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 slots");
+    p->total = (int)acc;
+    const int wpc = attn_warps_per_cta(ctx->G);
+    const long long nwarps_max = (long long)ctx->sms * wpc;
+    long long W = (acc + nwarps_max - 1) / nwarps_max;
+    if (W < kMinSlotsPerWarp) W = kMinSlotsPerWarp;
+    p->W = (int)W;
+    const long long warps = (acc + W - 1) / W;
+    *ctas = (int)((warps + wpc - 1) / wpc);
+    *n_active = na;
+    return RA_OK;
+}
+
+void set_scale(AttnParams* p, float scale)
+{
+    const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)kHeadDim);
+    p->qk_scale_log2 = sc * 1.4426950408889634f;
+}
+
 }  // namespace
 
 extern "C" {
@@ -268,6 +309,7 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_poff = take((size_t)batch * 4);
     ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
     ctx->off_partial = take((size_t)(kMaxSMs * kMaxAttnWarps + batch * kv_heads) * partial_stride(ctx->G) * 4);
+    ctx->off_arrive = take((size_t)batch * kv_heads * 4);
     ctx->off_err = take(256);
     ctx->bytes = o;
     ctx->g.assign((size_t)layers * batch, 0);
@@ -319,6 +361,7 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.seq_poff = (int32_t*)(a + ctx->off_poff);
     Ly.plan = (int32_t*)(a + ctx->off_plan);
     Ly.partial = (float*)(a + ctx->off_partial);
+    Ly.arrive = (int32_t*)(a + ctx->off_arrive);
     Ly.err = (int32_t*)(a + ctx->off_err);
     Ly.prompt_rows_per_layer = ctx->prompt_rows_per_layer;
     Ly.gen_row0 = ctx->prompt_rows_per_layer * ctx->L;
@@ -346,7 +389,8 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
             cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.seq_lp, ctx->lp.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.seq_poff, ctx->poff.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess)
         return cuda_fail(ctx, e, "table initialisation");
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(ctx, e, "table initialisation sync");
 
@@ -435,13 +479,6 @@ int ra_set_active(ra_ctx* ctx, int seq, int active)
     return RA_OK;
 }
 
-static void fill_active(const ra_ctx* ctx, uint32_t* mask)
-{
-    for (int i = 0; i < RA_MAX_BATCH / 32; ++i) mask[i] = 0;
-    for (int b = 0; b < ctx->B; ++b)
-        if (ctx->active[b]) mask[b >> 5] |= 1u << (b & 31);
-}
-
 int ra_append_kv(ra_ctx* ctx, int layer, const uint16_t* k_new, const uint16_t* v_new, void* stream)
 {
     int rc;
@@ -486,6 +523,7 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
     EvictParams p{};
     p.lay = ctx->lay;
     p.layer = layer;
+    p.pending = 0;
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
@@ -534,43 +572,101 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     p.layer = layer;
     p.q = q;
     p.out = out;
-    fill_active(ctx, p.active);
-    long long acc = 0;
+    p.partial = ctx->lay.partial;
+    p.arrive = ctx->lay.arrive;
     int n_active = 0;
-    p.seq_base[0] = 0;
-    for (int b = 0; b < ctx->B; ++b) {
-        if (ctx->active[b]) {
-            acc += (long long)ctx->KVH * (ctx->lp[b] + ctx->c[(size_t)layer * ctx->B + b]);
-            ++n_active;
-        }
-        p.seq_base[b + 1] = (int32_t)acc;
-    }
-    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 slots");
+    int ctas = 0;
+    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
-    const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)kHeadDim);
-    p.qk_scale_log2 = sc * 1.4426950408889634f;
-    p.total = (int)acc;
-    const int wpc = attn_warps_per_cta(ctx->G);
-    const long long nwarps_max = (long long)ctx->sms * wpc;
-    long long W = (acc + nwarps_max - 1) / nwarps_max;
-    if (W < kMinSlotsPerWarp) W = kMinSlotsPerWarp;
-    p.W = (int)W;
+    set_scale(&p, scale);
+    cudaStream_t s = (cudaStream_t)stream;
+    ProfScope ps(ctx, RA_KERNEL_ATTN, (double)p.total * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes, s);
+    cudaError_t e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+    ps.done();
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
+    return RA_OK;
+}
+
+int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                    uint16_t* out, float scale, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!q || !out || !k_new || !v_new || !aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
+        return fail(ctx, RA_ERR_INVALID_ARG, "q/k_new/v_new/out must be non-NULL and 16-byte aligned");
+    const size_t base = (size_t)layer * ctx->B;
+    for (int b = 0; b < ctx->B; ++b)
+        if (ctx->active[b] && ctx->c[base + b] >= ctx->Cmax)
+            return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d already caches K + 2r = %d generated tokens", layer, b,
+                        ctx->Cmax);
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
-    if (acc > 0) {
-        const long long warps = (acc + W - 1) / W;
-        const int ctas = (int)((warps + wpc - 1) / wpc);
-        ProfScope ps(ctx, RA_KERNEL_ATTN, (double)acc * 2 * kRowBytes + (double)n_active * ctx->H * kRowBytes, s);
+    // 1. Eviction first, with the step's token pending: it is the newest slot, so it is never a
+    //    candidate, and evicting before writing it gives the same state as append-then-evict.
+    EvictParams ep{};
+    ep.lay = ctx->lay;
+    ep.layer = layer;
+    ep.pending = 1;
+    int n = 0;
+    double moved = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (!ctx->active[b]) continue;
+        const int g1 = ctx->g[base + b] + 1, c1 = ctx->c[base + b] + 1;
+        if (g1 % ctx->r == 0 && c1 - ctx->r > ctx->K) {
+            ep.trig[n++] = (int16_t)b;
+            moved += (double)(ctx->K + ctx->r - 1) * ctx->KVH;
+        }
+    }
+    if (n > 0) {
+        ep.n_trig = n;
+        {
+            ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
+            e = launch_select(ep, s);
+            ps.done();
+        }
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
+        {
+            ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
+            e = launch_compact(ep, s);
+            ps.done();
+        }
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
+        for (int i = 0; i < n; ++i) {
+            const int b = ep.trig[i];
+            ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written
+            ctx->nev[base + b] += 1;
+        }
+    }
+    // 2. Fused append + attention (+ merge of the split pieces).
+    AttnParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    p.q = q;
+    p.out = out;
+    p.k_new = k_new;
+    p.v_new = v_new;
+    p.partial = ctx->lay.partial;
+    p.arrive = ctx->lay.arrive;
+    int n_active = 0, ctas = 0;
+    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas)) != RA_OK) return rc;
+    if (n_active == 0) return RA_OK;
+    for (int b = 0; b < ctx->B; ++b) p.seq_g[b] = ctx->g[base + b];
+    set_scale(&p, scale);
+    {
+        ProfScope ps(ctx, RA_KERNEL_ATTN,
+                     (double)p.total * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes +
+                         (double)n_active * ctx->KVH * 2 * kRowBytes,
+                     s);
         e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
         ps.done();
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
     }
-    {
-        ProfScope ps(ctx, RA_KERNEL_COMBINE, (double)n_active * ctx->H * kRowBytes, s);
-        e = launch_combine(p, s);
-        ps.done();
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
+    for (int b = 0; b < ctx->B; ++b) {
+        if (!ctx->active[b]) continue;
+        ctx->c[base + b] += 1;
+        ctx->g[base + b] += 1;
     }
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "combine launch");
     return RA_OK;
 }
 
@@ -586,11 +682,10 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
             if (ctx->active[b] && ctx->c[(size_t)l * ctx->B + b] >= ctx->Cmax)
                 return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d is full (evict not called)", l, b);
     const size_t qs = (size_t)ctx->B * ctx->H * kHeadDim, ks = (size_t)ctx->B * ctx->KVH * kHeadDim;
-    for (int l = 0; l < ctx->L; ++l) {
-        if ((rc = ra_append_kv(ctx, l, k_all + l * ks, v_all + l * ks, stream)) != RA_OK) return rc;
-        if ((rc = ra_evict(ctx, l, nullptr, stream)) != RA_OK) return rc;
-        if ((rc = ra_decode_attn(ctx, l, q_all + l * qs, out_all + l * qs, scale, stream)) != RA_OK) return rc;
-    }
+    for (int l = 0; l < ctx->L; ++l)
+        if ((rc = ra_decode_layer(ctx, l, q_all + l * qs, k_all + l * ks, v_all + l * ks, out_all + l * qs, scale,
+                                  stream)) != RA_OK)
+            return rc;
     return RA_OK;
 }
 
@@ -777,44 +872,27 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     p.layer = layer;
     p.q = q;
     p.out = out;
-    fill_active(ctx, p.active);
-    long long acc = 0;
-    int n_active = 0;
-    p.seq_base[0] = 0;
-    for (int b = 0; b < ctx->B; ++b) {
-        if (ctx->active[b]) {
-            acc += (long long)ctx->KVH * (ctx->lp[b] + ctx->c[(size_t)layer * ctx->B + b]);
-            ++n_active;
-        }
-        p.seq_base[b + 1] = (int32_t)acc;
-    }
-    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 slots");
+    int n_active = 0, ctas = 0;
+    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
-    const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)kHeadDim);
-    p.qk_scale_log2 = sc * 1.4426950408889634f;
-    p.total = (int)acc;
-    const int wpc = attn_warps_per_cta(ctx->G);
-    const long long nwarps_max = (long long)ctx->sms * wpc;
-    long long W = (acc + nwarps_max - 1) / nwarps_max;
-    if (W < kMinSlotsPerWarp) W = kMinSlotsPerWarp;
-    p.W = (int)W;
-    const long long warps = acc > 0 ? (acc + W - 1) / W : 0;
-    // partial records written: one per (warp, head) piece, at index warp + head
-    const size_t need = (size_t)(warps + (long long)ctx->B * ctx->KVH) * partial_stride(ctx->G) * sizeof(float);
+    set_scale(&p, scale);
+    const long long warps = p.total > 0 ? ((long long)p.total + p.W - 1) / p.W : 0;
+    // [arrival counters, one int per (seq, KV head)][partial records, one per (warp, head) piece]
+    const size_t counters = align_up((size_t)ctx->B * ctx->KVH * sizeof(int32_t), kAlign);
+    const size_t need =
+        counters + (size_t)(warps + (long long)ctx->B * ctx->KVH) * partial_stride(ctx->G) * sizeof(float);
     if (need > kNoAllocScratchBytes)
         return fail(ctx, RA_ERR_CAPACITY, "layer needs %zu bytes of split-K scratch; the fixed array holds %zu", need,
                     kNoAllocScratchBytes);
     float* scratch = nullptr;
     if ((rc = noalloc_scratch(ctx, ctx->device, &scratch)) != RA_OK) return rc;
-    p.lay.partial = scratch;
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e;
-    if (acc > 0) {
-        const int ctas = (int)((warps + wpc - 1) / wpc);
-        e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
-    }
-    e = launch_combine(p, s);
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "combine launch");
+    p.arrive = reinterpret_cast<int32_t*>(scratch);
+    p.partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(scratch) + counters);
+    // the counters must start at zero; the array keeps whatever the previous call left
+    cudaError_t e = cudaMemsetAsync(p.arrive, 0, (size_t)ctx->B * ctx->KVH * sizeof(int32_t), s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "scratch counter clear");
+    e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
     return RA_OK;
 }

@@ -8,7 +8,7 @@
 //                   select of the K smallest (score, ordinal) -- Eq. 1 -- and a
 //                   ballot-compacted, ascending list of the evicted ordinals.
 //   compact_kernel  many CTAs per triggered head: order-preserving move of the
-//                   survivors (kept candidates, then the r-token buffer) into
+//                   survivors (kept candidates, then the buffer rows) into
 //                   the head's spare region with coalesced 16-byte copies
 //                   ("keep-sets sorted chronologically ... compacted with a
 //                   gather", Appendix F).  Out of place, so CTAs never wait on
@@ -50,6 +50,8 @@ __device__ __forceinline__ bool bit_on(const uint32_t* mask, int b) { return (ma
 // ----------------------------------------------------------------------------- append
 __global__ void __launch_bounds__(1024) append_kernel(const __grid_constant__ AppendParams p)
 {
+    pdl_launch_dependents();
+    pdl_wait();
     const int b = blockIdx.x;
     if (!bit_on(p.active, b)) return;
     const DevLayout& L = p.lay;
@@ -82,12 +84,16 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     extern __shared__ uint32_t sm[];
     __shared__ uint32_t hist[256];
     __shared__ uint32_t s_bin, s_before, s_total;
+    pdl_launch_dependents();
+    pdl_wait();
     const DevLayout& L = p.lay;
     const int b = p.trig[blockIdx.x], h = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const DevCounters cnt = L.counters[(size_t)p.layer * L.B + b];
-    const int c = cnt.c, g = cnt.g, K = L.K, r = L.r;
-    const int N = c - r, m = N - K;
+    // With a pending token (fused step) the cache holds c rows and the token about to be
+    // appended is the newest slot: candidates and the step count include it.
+    const int c = cnt.c, g = cnt.g + p.pending, K = L.K, r = L.r;
+    const int N = c + p.pending - r, m = N - K;
     const int head_id = b * L.KVH + h;
     int32_t* plan = L.plan + (size_t)head_id * (kPlanHeader + r);
     if (m <= 0 || m > r || N > kMaxCandidates) {  // the host mirror rules this out; never move data on a bad plan
@@ -230,6 +236,9 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
 {
     extern __shared__ int32_t s_ev[];
     __shared__ int32_t s_hdr[4];
+    __shared__ int32_t s_dst[kCompactChunk];
+    pdl_launch_dependents();
+    pdl_wait();
     const DevLayout& L = p.lay;
     const int t = blockIdx.y / L.KVH, h = blockIdx.y % L.KVH;
     const int b = p.trig[t];
@@ -244,6 +253,17 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
     const int s0 = blockIdx.x * kCompactChunk;
     if (s0 >= c) return;
     const int s1 = min(c, s0 + kCompactChunk);
+    // destination of every slot of the chunk: j - #evicted(< j), or -1 if j is evicted
+    for (int t = threadIdx.x; t < s1 - s0; t += kCompactThreads) {
+        const int j = s0 + t;
+        int lo = 0, hi = m;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (s_ev[mid] < j) lo = mid + 1; else hi = mid;
+        }
+        s_dst[t] = (lo < m && s_ev[lo] == j) ? -1 : j - lo;
+    }
+    __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint16_t* sbase = (lane < 16 ? L.kpool : L.vpool) + (L.gen_row0 + (long long)src * L.Cmax) * kHeadDim;
     uint16_t* dbase = (lane < 16 ? L.kpool : L.vpool) + (L.gen_row0 + (long long)dst * L.Cmax) * kHeadDim;
@@ -257,18 +277,10 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
 #pragma unroll
         for (int u = 0; u < kCompactUnroll; ++u) {
             const int j = base + u;
-            dj[u] = -1;
-            if (j < s1) {
-                int lo = 0, hi = m;  // rank = number of evicted ordinals < j
-                while (lo < hi) {
-                    const int mid = (lo + hi) >> 1;
-                    if (s_ev[mid] < j) lo = mid + 1; else hi = mid;
-                }
-                if (!(lo < m && s_ev[lo] == j)) {
-                    dj[u] = j - lo;
-                    val[u] = __ldg(reinterpret_cast<const uint4*>(sbase + (size_t)j * kHeadDim) + part);
-                    if (lane == 0) pv[u] = __ldg(spos + j);
-                }
+            dj[u] = j < s1 ? s_dst[j - s0] : -1;
+            if (dj[u] >= 0) {
+                val[u] = __ldg(reinterpret_cast<const uint4*>(sbase + (size_t)j * kHeadDim) + part);
+                if (lane == 0) pv[u] = __ldg(spos + j);
             }
         }
 #pragma unroll
@@ -316,8 +328,7 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(const __grid_constant__ 
 
 cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s)
 {
-    append_kernel<<<B, p.lay.KVH * 32, 0, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(append_kernel, dim3(B), dim3(p.lay.KVH * 32), 0, s, p);
 }
 
 static size_t select_smem(int N) { return ((size_t)((N + 31) / 32) * 32 + (N + 31) / 32) * sizeof(uint32_t); }
@@ -332,16 +343,15 @@ cudaError_t launch_select(const EvictParams& p, cudaStream_t s)
         if (e != cudaSuccess) return e;
         configured = smem;
     }
-    select_kernel<<<dim3(p.n_trig, p.lay.KVH), kSelThreads, smem, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(select_kernel, dim3(p.n_trig, p.lay.KVH), dim3(kSelThreads), smem, s, p);
 }
 
 cudaError_t launch_compact(const EvictParams& p, cudaStream_t s)
 {
     const int Cmax = p.lay.Cmax;
     const int chunks = (Cmax + kCompactChunk - 1) / kCompactChunk;
-    compact_kernel<<<dim3(chunks, p.n_trig * p.lay.KVH), kCompactThreads, p.lay.r * sizeof(int32_t), s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(compact_kernel, dim3(chunks, p.n_trig * p.lay.KVH), dim3(kCompactThreads),
+                      p.lay.r * sizeof(int32_t), s, p);
 }
 
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s)

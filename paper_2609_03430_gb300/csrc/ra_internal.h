@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "ra.h"
 
 namespace ra {
@@ -41,6 +43,7 @@ struct DevLayout {
     int32_t* seq_poff;     // [B] row offset of a sequence's prompt block inside a layer (KVH * sum lp)
     int32_t* plan;         // [B*KVH][kPlanHeader + r] eviction plan of the current layer
     float* partial;        // attention split partials
+    int32_t* arrive;       // [B*KVH] split-piece arrival counters
     int32_t* err;          // device error word
     long long prompt_rows_per_layer;
     long long gen_row0;    // first row of the generated regions
@@ -59,6 +62,7 @@ struct AppendParams {
 struct EvictParams {
     DevLayout lay;
     int layer;
+    int pending;  // 1 when the step's new token is not yet in the cache (fused step): it counts as the newest slot
     int n_trig;
     int16_t trig[RA_MAX_BATCH];  // triggered sequence ids
 };
@@ -67,12 +71,17 @@ struct AttnParams {
     DevLayout lay;
     int layer;
     const uint16_t* q;      // [B][H][128]
-    uint16_t* out;          // [B][H][128] (combine)
+    uint16_t* out;          // [B][H][128]
+    const uint16_t* k_new;  // fused append: the step's new rows [B][KVH][128]; null = attention only
+    const uint16_t* v_new;
+    float* partial;         // split-K partial records (arena or the no-alloc array)
+    int32_t* arrive;        // [B*KVH] pieces merged so far per head; zero between launches
     int W;                  // slots per warp (stream-K split)
     int total;              // total slots of the layer
     float qk_scale_log2;    // scale * log2(e)
     uint32_t active[RA_MAX_BATCH / 32];
-    int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of (lp + c) over active sequences
+    int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of head lengths over active sequences
+    int32_t seq_g[RA_MAX_BATCH];         // fused append: tokens generated before this one
 };
 
 struct CopyRowsParams {
@@ -97,7 +106,25 @@ int attn_warps_per_cta(int G);
 int attn_tile_rows(int G);
 cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tmap_k, const CUtensorMap* tmap_v, int ctas,
                              cudaStream_t s);
-cudaError_t launch_combine(const AttnParams& p, cudaStream_t s);
 cudaError_t attn_prepare(int G);  // one-time function attributes (dynamic smem)
+
+// Launch with programmatic dependent launch: the kernel may be scheduled while its
+// predecessor on the stream finishes; every kernel waits (griddepcontrol.wait)
+// before touching memory a predecessor writes.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args&&... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 }  // namespace ra

@@ -30,7 +30,7 @@ def check_attention(got_bits, ref, what=""):
 class Runner:
     """A small workload run through the C ABI with an oracle mirror of every head."""
 
-    def __init__(self, L, H, KVH, prompt_lens, K, r, eseed, dseed, key_scale=None, D=128):
+    def __init__(self, L, H, KVH, prompt_lens, K, r, eseed, dseed, key_scale=None, D=128, fused=False):
         import torch
 
         import paper_2609_03430_gb300 as ra
@@ -47,6 +47,7 @@ class Runner:
         self.orc = oracle.OracleCache(L, KVH, self.lp, K, r, eseed)
         self.dev = torch.device("cuda")
         self.step_idx = 0
+        self.fused = fused  # True: one ra_decode_layer call per layer instead of append/evict/attend
         self.active = [True] * self.B
         maxlp = max(max(self.lp), 1)
         for l in range(L):
@@ -90,16 +91,21 @@ class Runner:
                     k[b, h] = self.krows(l, b, h, [pos])[0]
                     v[b, h] = self.vrows(l, b, h, [pos])[0]
             tk, tv = self.up(k), self.up(v)  # keep both alive: a freed temporary would be reused for the next
-            self.ra.ra_append_kv(self.ctx, l, tk.data_ptr(), tv.data_ptr())
-            n = self.ra.ra_evict(self.ctx, l)
-            nf = sum(1 for b in range(self.B) if self.active[b] and self.orc.evict(b, l))
-            assert n == nf, (l, n, nf)
-            fired[l] = n
             q = np.stack([synth.q_rows(self.dseed, l, b, np.arange(self.H), self.step_idx, self.D)
                           for b in range(self.B)])
             out = self.torch.zeros((self.B, self.H, self.D), dtype=self.torch.int16, device=self.dev)
             tq = self.up(q)
-            self.ra.ra_decode_attn(self.ctx, l, tq.data_ptr(), out.data_ptr(), scale)
+            nf = sum(1 for b in range(self.B) if self.active[b] and self.orc.evict(b, l))
+            if self.fused:
+                before = [self.ra.ra_get_counters(self.ctx, b, l)[2] for b in range(self.B)]
+                self.ra.ra_decode_layer(self.ctx, l, tq.data_ptr(), tk.data_ptr(), tv.data_ptr(), out.data_ptr(), scale)
+                n = sum(self.ra.ra_get_counters(self.ctx, b, l)[2] - before[b] for b in range(self.B))
+            else:
+                self.ra.ra_append_kv(self.ctx, l, tk.data_ptr(), tv.data_ptr())
+                n = self.ra.ra_evict(self.ctx, l)
+                self.ra.ra_decode_attn(self.ctx, l, tq.data_ptr(), out.data_ptr(), scale)
+            assert n == nf, (l, n, nf)
+            fired[l] = n
             if l in check_attn_layers:
                 outs[l] = (q, out)
         for l, (q, out) in outs.items():

@@ -12,10 +12,11 @@ from ra_testlib import Runner, check_attention
 pytestmark = [pytest.mark.gpu, pytest.mark.skipif(not cuda_available(), reason="needs a CUDA GPU")]
 
 
-def test_config1_full_run():
+@pytest.mark.parametrize("fused", [False, True], ids=["separate-calls", "fused-layer"])
+def test_config1_full_run(fused):
     """Qwen3-4B attention shape, one layer, batch 1, prompt 128, K=256, r=64, 1024 steps, seed 0:
     eleven evictions; state checked bit-exactly after each, attention every 8th step and at firings."""
-    run = Runner(L=1, H=32, KVH=8, prompt_lens=[128], K=256, r=64, eseed=0, dseed=1)
+    run = Runner(L=1, H=32, KVH=8, prompt_lens=[128], K=256, r=64, eseed=0, dseed=1, fused=fused)
     n_fire = 0
     for step in range(1024):
         g_next = step + 1
@@ -29,10 +30,11 @@ def test_config1_full_run():
     run.close()
 
 
-def test_ragged_batch_layers_and_finishing():
+@pytest.mark.parametrize("fused", [False, True], ids=["separate-calls", "fused-layer"])
+def test_ragged_batch_layers_and_finishing(fused):
     """Ragged prompts (including an empty one), G=5, K not a multiple of r, two layers,
     a sequence that finishes mid-run."""
-    run = Runner(L=2, H=40, KVH=8, prompt_lens=[0, 17, 100, 33, 250], K=100, r=32, eseed=5, dseed=3)
+    run = Runner(L=2, H=40, KVH=8, prompt_lens=[0, 17, 100, 33, 250], K=100, r=32, eseed=5, dseed=3, fused=fused)
     for step in range(420):
         if step == 200:
             run.set_active(3, False)
@@ -45,7 +47,7 @@ def test_ragged_batch_layers_and_finishing():
 
 @pytest.mark.parametrize("G", [1, 2, 3, 4, 6, 7, 8])
 def test_group_sizes(G):
-    run = Runner(L=1, H=2 * G, KVH=2, prompt_lens=[70, 1], K=48, r=16, eseed=G, dseed=10 + G)
+    run = Runner(L=1, H=2 * G, KVH=2, prompt_lens=[70, 1], K=48, r=16, eseed=G, dseed=10 + G, fused=G % 2 == 0)
     for step in range(150):
         fired = run.step(check_attn_layers=(0,) if step % 25 == 0 or step in (95, 96, 97) else ())
         if any(fired.values()):
@@ -55,8 +57,9 @@ def test_group_sizes(G):
 
 def test_degenerate_budgets():
     # K = 0: only the recent buffer survives; r = 1 evicts at every step once the cache exceeds K + 1
-    for K, r in [(0, 8), (5, 1), (3, 2)]:
-        run = Runner(L=1, H=4, KVH=2, prompt_lens=[9], K=K, r=r, eseed=K + r, dseed=2)
+    for (K, r), fused in [((0, 8), False), ((5, 1), False), ((3, 2), False), ((0, 8), True), ((5, 1), True),
+                          ((3, 2), True)]:
+        run = Runner(L=1, H=4, KVH=2, prompt_lens=[9], K=K, r=r, eseed=K + r, dseed=2, fused=fused)
         for step in range(60):
             fired = run.step(check_attn_layers=(0,) if step % 7 == 0 else ())
             if any(fired.values()):
