@@ -18,6 +18,8 @@ SOURCES = ["ra_api.cu", "ra_evict.cu", "ra_attn.cu"]
 HEADERS = ["ra_internal.h", "ra_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include"), "-I" + CSRC]
+# Extra nvcc flags, e.g. -DRA_ATTN_S_LPS=16 ... to build another attention kernel shape.
+EXTRA = os.environ.get("RA_NVCC_FLAGS", "").split()
 
 
 def _inputs():
@@ -37,7 +39,7 @@ def compile_procs():
     procs = []
     for s in SOURCES:
         obj = os.path.join(BUILD, s.replace(".cu", ".o"))
-        cmd = ["nvcc", *ARCH, *FLAGS, "-c", os.path.join(CSRC, s), "-o", obj]
+        cmd = ["nvcc", *ARCH, *FLAGS, *EXTRA, "-c", os.path.join(CSRC, s), "-o", obj]
         procs.append((subprocess.Popen(cmd), obj, cmd))
     return procs
 

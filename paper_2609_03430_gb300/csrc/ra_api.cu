@@ -28,7 +28,6 @@ namespace {
 thread_local std::string g_tls_error = "no error";
 
 constexpr int kMaxSMs = 256;       // partial-buffer sizing bound (the GB300 has 152)
-constexpr int kMaxAttnWarps = 8;   // warps per attention CTA, upper bound
 constexpr int kMinSlotsPerWarp = 64;
 constexpr size_t kAlign = 256;
 
@@ -52,6 +51,7 @@ struct ra_ctx {
     long long total_rows = 0;
     long long gen_rows = 0;
     int regions = 0;
+    size_t partial_records = 0;  // split-K partial records the arena holds
     // arena layout (byte offsets)
     size_t off_k, off_v, off_pos, off_region, off_spare, off_cnt, off_lp, off_poff, off_plan, off_partial, off_arrive,
         off_err, bytes;
@@ -189,10 +189,11 @@ int make_tmap(ra_ctx* ctx, CUtensorMap* map, void* base, int box_rows)
     }
     const cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)ctx->total_rows};
     const cuuint64_t strides[1] = {(cuuint64_t)kRowBytes};
-    const cuuint32_t box[2] = {(cuuint32_t)kHeadDim, (cuuint32_t)box_rows};
+    // boxes of 64 channels (128 bytes) x box_rows rows, stored with the 128-byte swizzle
+    const cuuint32_t box[2] = {(cuuint32_t)(kHeadDim / 2), (cuuint32_t)box_rows};
     const cuuint32_t estr[2] = {1, 1};
     CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(ctx, RA_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
     return RA_OK;
@@ -230,6 +231,9 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     const long long warps = (acc + W - 1) / W;
     *ctas = (int)((warps + wpc - 1) / wpc);
     *n_active = na;
+    // partial records are indexed warp + head: both bounded by what the arena holds
+    if ((size_t)(*ctas) * wpc + (size_t)ctx->B * ctx->KVH > ctx->partial_records)
+        return fail(ctx, RA_ERR_STATE, "attention split needs more partial records than the arena holds");
     return RA_OK;
 }
 
@@ -308,7 +312,8 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_lp = take((size_t)batch * 4);
     ctx->off_poff = take((size_t)batch * 4);
     ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
-    ctx->off_partial = take((size_t)(kMaxSMs * kMaxAttnWarps + batch * kv_heads) * partial_stride(ctx->G) * 4);
+    ctx->partial_records = (size_t)kMaxSMs * attn_warps_per_cta(ctx->G) + (size_t)batch * kv_heads;
+    ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);
     ctx->off_err = take(256);
     ctx->bytes = o;
@@ -392,6 +397,8 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
         (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess)
         return cuda_fail(ctx, e, "table initialisation");
+    // rows that were never written (past a head's cached slots) then read as zeros, never as stale NaNs
+    if ((e = cudaMemsetAsync(a, 0, ctx->off_pos, s)) != cudaSuccess) return cuda_fail(ctx, e, "cache clear");
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(ctx, e, "table initialisation sync");
 
     const int tile = attn_tile_rows(ctx->G);

@@ -21,17 +21,19 @@
 // monotonically through the slot order -- and the last warp to finish a piece
 // of that head (an arrival counter per head) merges all of them.
 //
-// Per-warp compute layout: LPS lanes share one cache row (each lane owns
-// 16 bytes -- 8 channels -- of every LPS-th 16-byte chunk, so a row read is
-// bank-conflict free); the warp works on 32/LPS rows at once.  The G query rows
-// live in fp32 registers; each K row is read once from shared memory and used
-// by all G heads (G flop per byte), with packed two-wide fp32 FMAs.  Partial
-// dot products are summed across the LPS lanes with a butterfly reduce-scatter
-// (each exchange halves the vector), which leaves exactly one (row, head) score
-// per lane.  The softmax is online in base 2 with the scale folded into one
-// multiply; the running max is only raised when a batch exceeds it by more than
-// 2^8 (results are unchanged up to rounding, as softmax is shift invariant), so
-// rescaling the accumulators is rare.
+// Per-warp compute: the contraction of the G query rows with a tile of cache
+// rows runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
+// S = Q K^T takes the query heads as the 16 M rows (G <= 8 used, the rest
+// zero) and 8 cache rows per N tile; O += P V reuses the S accumulator
+// fragments as the A operand (P rounded to bf16).  Q fragments stay in
+// registers for a whole head piece; K and V are read with ldmatrix from TMA
+// tiles stored with the 128-byte swizzle, so the reads are bank-conflict free.
+// Each lane owns one query head (lane / 4): the softmax statistics need only
+// two shuffles per 16 rows, and O needs no cross-lane reduction.  The softmax
+// is online in base 2 with the scale folded into one multiply; the running max
+// is only raised when a batch exceeds it by more than 2^8 (the result is
+// unchanged up to rounding, as softmax is shift invariant), so rescaling the
+// accumulators is rare.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -47,34 +49,40 @@ namespace {
 constexpr float kTau = 8.0f;                       // lazy-rescale threshold (log2 units)
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // bounded mbarrier waits: 2 s
 constexpr int kSmemBudget = 220 * 1024;
+constexpr int kHalfCh = 64;                        // channels per swizzled TMA box (128 bytes)
+
+// Kernel shape: rows per stage (a multiple of 16), stages per warp, warps per CTA
+// (one CTA per SM; the warp count is capped by what fits in shared memory).
+#ifndef RA_ATTN_TILE
+#define RA_ATTN_TILE 16
+#endif
+#ifndef RA_ATTN_SPW
+#define RA_ATTN_SPW 3
+#endif
+#ifndef RA_ATTN_WARPS
+#define RA_ATTN_WARPS 8
+#endif
 
 template <int G>
 struct Cfg {
-    static constexpr int GP = G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8));  // G padded to a power of two
-    static constexpr int LPS = G <= 4 ? 8 : 16;                              // lanes per cache row
-    static constexpr int SG = 32 / LPS;                                      // rows per warp step
-    static constexpr int NB = LPS / GP;                                      // steps per reduce batch
-    static constexpr int BATCH = SG * NB;                                    // rows per batch
-    static constexpr int NCH = 16 / LPS;                                     // 16-byte chunks per lane per row
-    static constexpr int CPL = NCH * 8;                                      // channels per lane
-    static constexpr int CP2 = CPL / 2;                                      // channel pairs per lane
-    static constexpr int TILE = BATCH > 16 ? BATCH : 16;                     // rows per stage
-    static constexpr int KV_BYTES = TILE * kRowBytes;
+    static constexpr int TILE = RA_ATTN_TILE;                                // rows per stage
+    static constexpr int HALF_BYTES = TILE * 128;                            // one 64-channel half of K or V
+    static constexpr int KV_BYTES = 2 * HALF_BYTES;                          // a K (or V) tile
     static constexpr int Q_BYTES = G * kRowBytes;
-    static constexpr int STAGE_BYTES = ((2 * KV_BYTES + Q_BYTES) + 127) / 128 * 128;
-    static constexpr int W3 = kSmemBudget / (3 * STAGE_BYTES);
-    static constexpr int SPW = W3 >= 6 ? 3 : 2;
-    static constexpr int WARPS_RAW = SPW == 3 ? W3 : kSmemBudget / (2 * STAGE_BYTES);
-    static constexpr int WARPS = WARPS_RAW > 8 ? 8 : WARPS_RAW;
+    static constexpr int STAGE_BYTES = (2 * KV_BYTES + Q_BYTES + 1023) / 1024 * 1024;
+    static constexpr int SPW = RA_ATTN_SPW;
+    static constexpr int WARPS_FIT = kSmemBudget / (SPW * STAGE_BYTES);
+    static constexpr int WARPS = WARPS_FIT < RA_ATTN_WARPS ? WARPS_FIT : RA_ATTN_WARPS;
     static constexpr int NSTAGE = WARPS * SPW;
-    static constexpr size_t SMEM = 128 + (size_t)NSTAGE * STAGE_BYTES + (size_t)NSTAGE * (16 + 8);
+    static constexpr size_t SMEM = 1024 + (size_t)NSTAGE * STAGE_BYTES + (size_t)NSTAGE * (16 + 8);
     // merge layout: LG lanes per query head, MCH channels per lane
+    static constexpr int GP = G <= 1 ? 1 : (G <= 2 ? 2 : (G <= 4 ? 4 : 8));
     static constexpr int LG = 32 / GP;
     static constexpr int MCH = kHeadDim / LG;
-    static_assert(LPS == NB * GP, "one reduced score per lane");
-    static_assert(TILE % BATCH == 0, "tile holds whole batches");
-    static_assert(WARPS >= 4, "shared-memory budget too small");
-    static_assert(STAGE_BYTES % 128 == 0, "TMA destinations stay 128-byte aligned");
+    static_assert(G >= 1 && G <= 8, "the 16-row MMA holds up to 8 query heads");
+    static_assert(TILE % 16 == 0 && TILE <= 256, "whole 16-row MMA batches; TMA box rows <= 256");
+    static_assert(HALF_BYTES % 1024 == 0, "128-byte-swizzled TMA boxes start 1024-byte aligned");
+    static_assert(WARPS >= 2, "shared-memory budget too small");
     static_assert(SMEM <= 232448, "fits the 227 KB opt-in shared memory of sm_100+");
 };
 
@@ -165,12 +173,40 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, int tile, TileDesc&
     return true;
 }
 
-__device__ __forceinline__ void unpack8(const uint4 u, float2* f)
+// Byte offset of (row j, 16-byte chunk c of 16) inside a swizzled K or V tile:
+// two boxes of 64 channels; within a box the chunk index is xored with j mod 8.
+template <int G>
+__device__ __forceinline__ uint32_t swz(int j, int c)
 {
-    f[0] = make_float2(bf16lo(u.x), bf16hi(u.x));
-    f[1] = make_float2(bf16lo(u.y), bf16hi(u.y));
-    f[2] = make_float2(bf16lo(u.z), bf16hi(u.z));
-    f[3] = make_float2(bf16lo(u.w), bf16hi(u.w));
+    return (uint32_t)((c >> 3) * Cfg<G>::HALF_BYTES + j * 128 + (((c & 7) ^ (j & 7)) << 4));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+// D[16x8] += A[16x16] B[16x8], bf16 inputs, fp32 accumulators.  Only rows 0..7 of A
+// (the query heads) are nonzero, so only c0/c1 of the accumulator are kept.
+__device__ __forceinline__ void mma_rows8(float& c0, float& c1, uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1)
+{
+    float d2, d3;
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%10, %11, %12, %13};"
+        : "=f"(c0), "=f"(c1), "=f"(d2), "=f"(d3)
+        : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1), "f"(c0), "f"(c1), "f"(0.f), "f"(0.f));
+    (void)d2;  // rows 8..15 of the product: padding
+    (void)d3;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
@@ -230,10 +266,10 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
 {
     using C = Cfg<G>;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t* wstage = smem + (size_t)warp * C::SPW * C::STAGE_BYTES;
-    // [stages (128-byte aligned)][tile headers, 16 bytes each][mbarriers, 8 bytes each]
+    // [stages (1024-byte aligned)][tile headers, 16 bytes each][mbarriers, 8 bytes each]
     int4* hdrs = reinterpret_cast<int4*>(smem + (size_t)C::NSTAGE * C::STAGE_BYTES) + warp * C::SPW;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)C::NSTAGE * C::STAGE_BYTES + C::NSTAGE * 16) + warp * C::SPW;
 
@@ -267,13 +303,17 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             const uint32_t kv = (d.flags & kNewTok) ? 2u * kRowBytes : 2u * C::KV_BYTES;
             mbar_arrive_expect_tx(&bars[s], kv + (first ? (uint32_t)C::Q_BYTES : 0u));
             const int b = d.hid / p.lay.KVH, h = d.hid - b * p.lay.KVH;
-            if (d.flags & kNewTok) {  // the step's new token comes from the caller's rows
+            if (d.flags & kNewTok) {  // the step's new token comes from the caller's rows (row 0, unswizzled)
                 const size_t src = ((size_t)b * p.lay.KVH + h) * kHeadDim;
-                bulk_load(st, p.k_new + src, (uint32_t)kRowBytes, &bars[s]);
-                bulk_load(st + C::KV_BYTES, p.v_new + src, (uint32_t)kRowBytes, &bars[s]);
+                bulk_load(st, p.k_new + src, 128u, &bars[s]);
+                bulk_load(st + C::HALF_BYTES, p.k_new + src + kHalfCh, 128u, &bars[s]);
+                bulk_load(st + C::KV_BYTES, p.v_new + src, 128u, &bars[s]);
+                bulk_load(st + C::KV_BYTES + C::HALF_BYTES, p.v_new + src + kHalfCh, 128u, &bars[s]);
             } else {
                 tma_load_2d(st, &tk, 0, (int)d.row, &bars[s]);
+                tma_load_2d(st + C::HALF_BYTES, &tk, kHalfCh, (int)d.row, &bars[s]);
                 tma_load_2d(st + C::KV_BYTES, &tv, 0, (int)d.row, &bars[s]);
+                tma_load_2d(st + C::KV_BYTES + C::HALF_BYTES, &tv, kHalfCh, (int)d.row, &bars[s]);
             }
             if (first)
                 bulk_load(st + 2 * C::KV_BYTES, p.q + ((size_t)b * p.lay.H + (size_t)h * G) * kHeadDim,
@@ -287,18 +327,15 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         if (more) ++issued;
     }
 
-    const int k = lane % C::LPS;
-    const int grp = lane / C::LPS;
-    const int g_own = lane % C::GP;
-    const int i_own = k / C::GP;
+    const int gq = lane >> 2;  // this lane's query head (rows >= G are padding)
+    const int tq = lane & 3;
+    const int mi = lane >> 3, ri = lane & 7;  // ldmatrix: matrix and row this lane addresses
 
-    float2 qf[G][C::CP2];
-    float2 O[G][C::CP2];
-    float m_own = -INFINITY, l_own = 0.f;
+    uint32_t qa[8][2];  // A fragments of Q (rows 0..7) for the 8 k-steps of 16 channels
+    float O[16][2];     // O[head gq][n-tile * 8 + 2 tq + {0, 1}]
+    float m_run = -INFINITY, l_run = 0.f;
 #pragma unroll
-    for (int g = 0; g < G; ++g)
-#pragma unroll
-        for (int c = 0; c < C::CP2; ++c) O[g][c] = make_float2(0.f, 0.f);
+    for (int nt = 0; nt < 16; ++nt) O[nt][0] = O[nt][1] = 0.f;
 
     for (int t = 0; t < issued; ++t) {
         const int s = t % C::SPW;
@@ -311,98 +348,77 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         }
         const int4 hd = hdrs[s];
         const int n = hd.x;
-        const uint8_t* Ks = wstage + (size_t)s * C::STAGE_BYTES;
-        const uint8_t* Vs = Ks + C::KV_BYTES;
-        if (hd.y & kFirst) {  // first tile of a head piece: fresh query rows
+        uint8_t* Ks = wstage + (size_t)s * C::STAGE_BYTES;
+        uint8_t* Vs = Ks + C::KV_BYTES;
+        const uint32_t ks = smem_u32(Ks), vs = smem_u32(Vs);
+        if (hd.y & kFirst) {  // first tile of a head piece: fresh query fragments
             const uint8_t* Qs = Vs + C::KV_BYTES;
 #pragma unroll
-            for (int g = 0; g < G; ++g)
-#pragma unroll
-                for (int cc = 0; cc < C::NCH; ++cc) unpack8(lds128(Qs + g * kRowBytes + (k + cc * C::LPS) * 16), &qf[g][cc * 4]);
+            for (int kk = 0; kk < 8; ++kk) {
+                qa[kk][0] = gq < G ? *reinterpret_cast<const uint32_t*>(Qs + gq * kRowBytes + (16 * kk + 2 * tq) * 2) : 0u;
+                qa[kk][1] = gq < G ? *reinterpret_cast<const uint32_t*>(Qs + gq * kRowBytes + (16 * kk + 8 + 2 * tq) * 2) : 0u;
+            }
+        }
+        if (n < C::TILE) {  // rows past the valid ones hold stale data: zero V there so 0 * V stays 0
+            const int nb = (n + 15) & ~15;  // only rows inside the last used 16-row batch matter
+            for (int idx = lane; idx < (nb - n) * 16; idx += 32) {
+                const int j = n + (idx >> 4), c = idx & 15;
+                *reinterpret_cast<uint4*>(Vs + swz<G>(j, c)) = make_uint4(0u, 0u, 0u, 0u);
+            }
+            __syncwarp();
         }
 
-        for (int bs = 0; bs < n; bs += C::BATCH) {
-            float vals[C::LPS];
+        for (int bs = 0; bs < n; bs += 16) {
+            // S = Q K^T for rows bs..bs+15: n-tile 0 = rows bs..bs+7, n-tile 1 = rows bs+8..bs+15
+            float s0a = 0.f, s0b = 0.f, s1a = 0.f, s1b = 0.f;
 #pragma unroll
-            for (int i = 0; i < C::NB; ++i) {
-                const int slot = bs + i * C::SG + grp;
-                const int row = slot < n ? slot : n - 1;
-                float2 acc[G];
-#pragma unroll
-                for (int g = 0; g < G; ++g) acc[g] = make_float2(0.f, 0.f);
-#pragma unroll
-                for (int cc = 0; cc < C::NCH; ++cc) {
-                    float2 kf[4];
-                    unpack8(lds128(Ks + row * kRowBytes + (k + cc * C::LPS) * 16), kf);
-#pragma unroll
-                    for (int e = 0; e < 4; ++e)
-#pragma unroll
-                        for (int g = 0; g < G; ++g) acc[g] = __ffma2_rn(qf[g][cc * 4 + e], kf[e], acc[g]);
-                }
-#pragma unroll
-                for (int g = 0; g < C::GP; ++g) vals[i * C::GP + g] = g < G ? acc[g < G ? g : 0].x + acc[g < G ? g : 0].y : 0.f;
+            for (int kk = 0; kk < 8; ++kk) {
+                uint32_t b[4];
+                ldsm_x4(b, ks + swz<G>(bs + (mi >> 1) * 8 + ri, 2 * kk + (mi & 1)));
+                mma_rows8(s0a, s0b, qa[kk][0], qa[kk][1], b[0], b[1]);
+                mma_rows8(s1a, s1b, qa[kk][0], qa[kk][1], b[2], b[3]);
             }
-            // Butterfly reduce-scatter over the LPS lanes of a row group:
-            // afterwards lane k holds the full dot product of value k = (i_own, g_own).
-#pragma unroll
-            for (int msk = C::LPS / 2; msk >= 1; msk >>= 1) {
-                const bool up = (lane & msk) != 0;
-#pragma unroll
-                for (int t2 = 0; t2 < msk; ++t2) {
-                    const float send = up ? vals[t2] : vals[t2 + msk];
-                    const float keep = up ? vals[t2 + msk] : vals[t2];
-                    vals[t2] = keep + __shfl_xor_sync(0xffffffffu, send, msk);
-                }
-            }
-            float sc = vals[0] * p.qk_scale_log2;
-            const int slot_own = bs + i_own * C::SG + grp;
-            if (slot_own >= n || g_own >= G) sc = -INFINITY;
-            float bm = sc;
-#pragma unroll
-            for (int msk = C::GP; msk < 32; msk <<= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, msk));
-            const bool need = bm > m_own + kTau;
+            // this lane: head gq, rows bs + 2tq + {0,1} and bs + 8 + 2tq + {0,1}
+            const int r0 = bs + 2 * tq;
+            const float sl = p.qk_scale_log2;
+            float sc[4] = {r0 < n ? s0a * sl : -INFINITY, r0 + 1 < n ? s0b * sl : -INFINITY,
+                           r0 + 8 < n ? s1a * sl : -INFINITY, r0 + 9 < n ? s1b * sl : -INFINITY};
+            float bm = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
+            bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 1));
+            bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 2));
+            const bool need = bm > m_run + kTau;
             if (__any_sync(0xffffffffu, need)) {
-                const float m_new = need ? bm : m_own;
-                const float a_own = (m_new == m_own) ? 1.f : exp2f(m_own - m_new);
-                l_own *= a_own;
-                m_own = m_new;
+                const float m_new = need ? bm : m_run;
+                const float a = (m_new == m_run) ? 1.f : exp2f(m_run - m_new);
+                l_run *= a;
+                m_run = m_new;
 #pragma unroll
-                for (int g = 0; g < G; ++g) {
-                    const float a = __shfl_sync(0xffffffffu, a_own, g);
-                    const float2 a2 = make_float2(a, a);
-#pragma unroll
-                    for (int c = 0; c < C::CP2; ++c) O[g][c] = __fmul2_rn(O[g][c], a2);
+                for (int nt = 0; nt < 16; ++nt) {
+                    O[nt][0] *= a;
+                    O[nt][1] *= a;
                 }
             }
-            const float pr = (g_own < G) ? exp2f(sc - m_own) : 0.f;
-            l_own += pr;
+            float pr[4];
 #pragma unroll
-            for (int i = 0; i < C::NB; ++i) {
-                const int slot = bs + i * C::SG + grp;
-                const int row = slot < n ? slot : n - 1;
-                float2 pb[G];
+            for (int e = 0; e < 4; ++e) pr[e] = exp2f(sc[e] - m_run);  // masked rows: exp2(-inf) = 0
+            l_run += (pr[0] + pr[1]) + (pr[2] + pr[3]);
+            const uint32_t pa0 = pack_bf16x2(pr[0], pr[1]), pa2 = pack_bf16x2(pr[2], pr[3]);
+            // O += P V: 16 n-tiles of 8 channels, k = the 16 rows
 #pragma unroll
-                for (int g = 0; g < G; ++g) {
-                    const float pg = __shfl_sync(0xffffffffu, pr, grp * C::LPS + i * C::GP + g);
-                    pb[g] = make_float2(pg, pg);
-                }
-#pragma unroll
-                for (int cc = 0; cc < C::NCH; ++cc) {
-                    float2 vf[4];
-                    unpack8(lds128(Vs + row * kRowBytes + (k + cc * C::LPS) * 16), vf);
-#pragma unroll
-                    for (int e = 0; e < 4; ++e)
-#pragma unroll
-                        for (int g = 0; g < G; ++g) O[g][cc * 4 + e] = __ffma2_rn(pb[g], vf[e], O[g][cc * 4 + e]);
-                }
+            for (int np = 0; np < 8; ++np) {
+                uint32_t b[4];
+                ldsm_x4_t(b, vs + swz<G>(bs + (mi & 1) * 8 + ri, 2 * np + (mi >> 1)));
+                mma_rows8(O[2 * np][0], O[2 * np][1], pa0, pa2, b[0], b[1]);
+                mma_rows8(O[2 * np + 1][0], O[2 * np + 1][1], pa0, pa2, b[2], b[3]);
             }
         }
 
         if (hd.y & kNewTok) {  // fused append: the new token's K/V row and position go into the cache
             const int b = hd.z / p.lay.KVH, h = hd.z - b * p.lay.KVH;
             const long long row = hd.w;
-            const uint4 v = lds128((lane < 16 ? Ks : Vs) + (lane & 15) * 16);
-            reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[lane & 15] = v;
+            const int c = lane & 15;  // row 0 of the tile is unswizzled: chunk c of the (c >> 3) half
+            const uint4 v = lds128((lane < 16 ? Ks : Vs) + (c >> 3) * C::HALF_BYTES + (c & 7) * 16);
+            reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[c] = v;
             if (lane == 0) {
                 const long long slot = row - p.lay.gen_row0;  // region * Cmax + cached index
                 const int g0 = p.seq_g[b];
@@ -416,61 +432,31 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         }
 
         if (hd.y & kLast) {  // last tile of the piece
-            float l = l_own;
-#pragma unroll
-            for (int msk = C::GP; msk < 32; msk <<= 1) l += __shfl_xor_sync(0xffffffffu, l, msk);
-#pragma unroll
-            for (int g = 0; g < G; ++g)
-#pragma unroll
-                for (int c = 0; c < C::CP2; ++c)
-#pragma unroll
-                    for (int msk = C::LPS; msk < 32; msk <<= 1) {
-                        O[g][c].x += __shfl_xor_sync(0xffffffffu, O[g][c].x, msk);
-                        O[g][c].y += __shfl_xor_sync(0xffffffffu, O[g][c].y, msk);
-                    }
+            float l = l_run;
+            l += __shfl_xor_sync(0xffffffffu, l, 1);
+            l += __shfl_xor_sync(0xffffffffu, l, 2);
             const int hid = hd.z;
             const int b = hid / p.lay.KVH, h = hid - b * p.lay.KVH;
             const int hl = seq_head_len(p, b);
             const long long A = p.seq_base[b] + (long long)h * hl;
             const int w0 = (int)(A / p.W), w1 = (int)((A + hl - 1) / p.W);
-            // l of head g sits in lane g (lanes 0..G-1 have g_own = lane)
-            float lg[G];
-#pragma unroll
-            for (int g = 0; g < G; ++g) lg[g] = __shfl_sync(0xffffffffu, l, g);
             if (w0 == w1) {  // the whole head was this warp's: normalise and write the output
-                if (grp == 0) {
+                if (gq < G) {
+                    const float inv = 1.f / l;
+                    uint32_t* out = reinterpret_cast<uint32_t*>(p.out + ((size_t)b * p.lay.H + (size_t)h * G + gq) * kHeadDim);
 #pragma unroll
-                    for (int g = 0; g < G; ++g) {
-                        const float inv = 1.f / lg[g];
-                        uint16_t* out = p.out + ((size_t)b * p.lay.H + (size_t)h * G + g) * kHeadDim;
-#pragma unroll
-                        for (int cc = 0; cc < C::NCH; ++cc) {
-                            const float2* o = &O[g][cc * 4];
-                            uint4 w;
-                            w.x = pack_bf16x2(o[0].x * inv, o[0].y * inv);
-                            w.y = pack_bf16x2(o[1].x * inv, o[1].y * inv);
-                            w.z = pack_bf16x2(o[2].x * inv, o[2].y * inv);
-                            w.w = pack_bf16x2(o[3].x * inv, o[3].y * inv);
-                            reinterpret_cast<uint4*>(out)[k + cc * C::LPS] = w;
-                        }
-                    }
+                    for (int nt = 0; nt < 16; ++nt) out[nt * 4 + tq] = pack_bf16x2(O[nt][0] * inv, O[nt][1] * inv);
                 }
             } else {
                 float* rec = p.partial + (size_t)(gw + hid) * partial_stride(G);
-                if (grp == 0) {
+                if (gq < G) {
 #pragma unroll
-                    for (int g = 0; g < G; ++g)
-#pragma unroll
-                        for (int cc = 0; cc < C::NCH; ++cc) {
-                            float4* dst = reinterpret_cast<float4*>(rec + g * kHeadDim + (k + cc * C::LPS) * 8);
-                            const float2* o = &O[g][cc * 4];
-                            dst[0] = make_float4(o[0].x, o[0].y, o[1].x, o[1].y);
-                            dst[1] = make_float4(o[2].x, o[2].y, o[3].x, o[3].y);
-                        }
-                }
-                if (lane < G) {
-                    rec[G * kHeadDim + lane] = m_own;
-                    rec[G * kHeadDim + G + lane] = l;
+                    for (int nt = 0; nt < 16; ++nt)
+                        *reinterpret_cast<float2*>(rec + gq * kHeadDim + nt * 8 + 2 * tq) = make_float2(O[nt][0], O[nt][1]);
+                    if (tq == 0) {
+                        rec[G * kHeadDim + gq] = m_run;
+                        rec[G * kHeadDim + G + gq] = l;
+                    }
                 }
                 __threadfence();
                 __syncwarp();
@@ -483,12 +469,10 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
                     if (lane == 0) p.arrive[hid] = 0;  // ready for the next launch
                 }
             }
-            m_own = -INFINITY;
-            l_own = 0.f;
+            m_run = -INFINITY;
+            l_run = 0.f;
 #pragma unroll
-            for (int g = 0; g < G; ++g)
-#pragma unroll
-                for (int c = 0; c < C::CP2; ++c) O[g][c] = make_float2(0.f, 0.f);
+            for (int nt = 0; nt < 16; ++nt) O[nt][0] = O[nt][1] = 0.f;
         }
 
         __syncwarp();

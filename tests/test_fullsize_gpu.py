@@ -1,0 +1,91 @@
+"""Parity at the full workload sizes, in the launch configuration bench.py times.
+
+Each workload is set up exactly as the benchmark does (steady-state caches
+filled on the device by the seeded generator, ``ra_decode_step`` over the whole
+layer stack), then run for r + 2 steps, so that every sequence evicts once,
+with step inputs generated for their true positions.  The oracle replays the
+sampled heads from the same start state: their survivor positions and their
+cached K/V bytes must match bit-exactly, and the last step's attention output
+of sampled (sequence, layer, KV head) slices must be within tolerance of the
+fp64 oracle.
+"""
+import numpy as np
+import pytest
+
+from conftest import cuda_available
+from ra_testlib import check_attention
+
+pytestmark = [pytest.mark.gpu, pytest.mark.skipif(not cuda_available(), reason="needs a CUDA GPU")]
+
+
+def _samples(w, n_heads, n_attn, seed):
+    rng = np.random.default_rng(seed)
+    heads = {(int(rng.integers(w["B"])), int(rng.integers(w["L"])), int(rng.integers(w["KVH"])))
+             for _ in range(n_heads)}
+    heads |= {(0, 0, 0), (w["B"] - 1, w["L"] - 1, w["KVH"] - 1)}
+    attn = sorted(heads)[:n_attn]
+    return sorted(heads), attn
+
+
+@pytest.mark.parametrize("cfg", [2, 3, 4, 5])
+def test_workload_parity_sampled(cfg):
+    import torch
+
+    import bench
+    import oracle
+    import paper_2609_03430_gb300 as ra
+    import synth
+    import synth.gpu as sg
+
+    torch.cuda.set_device(0)
+    wl = bench.Workload(cfg, ring=1)
+    w = wl.w
+    L, B, H, KVH, K, r, D = wl.L, wl.B, wl.H, wl.KVH, wl.K, wl.r, 128
+    G = H // KVH
+    heads, attn_heads = _samples(w, 64, 8, cfg)
+    orc = oracle.OracleCache(L, KVH, wl.lp, K, r, wl.eseed, heads=heads)
+    for (b, l, h) in heads:
+        c, g = wl.c0[b], wl.g0[b]
+        orc.gen[(b, l, h)] = np.arange(wl.lp[b] + g - c, wl.lp[b] + g, dtype=np.int32)
+        orc.g[b, l] = g
+    dev = wl.dev
+    q = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((L, B, KVH, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    out = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    steps = r + 2
+    for t in range(steps):
+        qpos = torch.full((B, H, 1), t, dtype=torch.int32, device=dev)
+        npos = torch.tensor([[wl.lp[b] + wl.g0[b] + t] * KVH for b in range(B)], dtype=torch.int32,
+                            device=dev).reshape(B, KVH, 1)
+        for l in range(L):
+            sg.fill_rows(q[l].view(B, H, 1, D), qpos, wl.dseed, 2, l, 0)
+            sg.fill_rows(kn[l].view(B, KVH, 1, D), npos, wl.dseed, 0, l, 0, wl._scale(l))
+            sg.fill_rows(vn[l].view(B, KVH, 1, D), npos, wl.dseed, 1, l, 0)
+        ra.ra_decode_step(wl.ctx, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), out.data_ptr(), 0.0)
+        for (b, l) in sorted({(b, l) for (b, l, _) in heads}):
+            orc.append(b, l)
+            orc.evict(b, l)
+    torch.cuda.synchronize()
+    ra.ra_check_device(wl.ctx)
+    fired = 0
+    for (b, l, h) in heads:
+        g, c, nev = ra.ra_get_counters(wl.ctx, b, l)
+        assert g == orc.g[b, l] and c == orc.gen[(b, l, h)].size
+        fired += nev > 0
+        got = ra.ra_get_positions(wl.ctx, l, b, h, K + 2 * r)
+        np.testing.assert_array_equal(got, orc.gen[(b, l, h)], err_msg=f"positions {(b, l, h)}")
+    assert fired == len(heads)  # every sampled head evicted at least once
+    sc_np = None if wl.key_scale is None else wl.key_scale.cpu().numpy()
+    got_out = out.cpu().numpy()
+    for (b, l, h) in attn_heads:
+        pos = orc.positions(b, l, h)
+        krow = synth.kv_rows(wl.dseed, 0, l, b, h, pos, D, None if sc_np is None else sc_np[l, h])
+        vrow = synth.kv_rows(wl.dseed, 1, l, b, h, pos, D)
+        kk, vv = ra.ra_get_kv(wl.ctx, l, b, h, wl.lp[b] + K + 2 * r)
+        np.testing.assert_array_equal(kk, krow, err_msg=f"K rows {(b, l, h)}")
+        np.testing.assert_array_equal(vv, vrow, err_msg=f"V rows {(b, l, h)}")
+        qv = synth.q_rows(wl.dseed, l, b, np.arange(h * G, (h + 1) * G), steps - 1, D)
+        ref = oracle.attend(qv, krow, vrow)
+        check_attention(got_out[l, b, h * G:(h + 1) * G], ref, f"cfg {cfg} slice {(b, l, h)}")
+    wl.cache.close()
