@@ -3,7 +3,7 @@
 // Owns the host mirror of every per-(layer, sequence) counter, so that trigger
 // decisions (section 2: every r steps once the candidates exceed K), capacity
 // checks and the attention work split are made on the host without reading
-// device memory; the kernels keep identical counters on the device.  No call
+// device memory; kernels receive the counts they need as launch parameters.  No call
 // allocates device memory or synchronises, except the debug getters.
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -28,7 +28,10 @@ namespace {
 thread_local std::string g_tls_error = "no error";
 
 constexpr int kMaxSMs = 256;       // partial-buffer sizing bound (the GB300 has 152)
-constexpr int kMinSlotsPerWarp = 64;
+#ifndef RA_ATTN_CHUNKS_PER_WARP
+#define RA_ATTN_CHUNKS_PER_WARP 1
+#endif
+constexpr int kChunksPerWarp = RA_ATTN_CHUNKS_PER_WARP;  // chunks per warp on average: room for stealing
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -52,8 +55,9 @@ struct ra_ctx {
     long long gen_rows = 0;
     int regions = 0;
     size_t partial_records = 0;  // split-K partial records the arena holds
+    unsigned long long ticket_base = 0;  // first chunk ticket of the next attention launch
     // arena layout (byte offsets)
-    size_t off_k, off_v, off_pos, off_region, off_spare, off_cnt, off_lp, off_poff, off_plan, off_partial, off_arrive,
+    size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_poff, off_plan, off_partial, off_arrive, off_ticket,
         off_err, bytes;
     // binding
     bool bound = false;
@@ -206,35 +210,54 @@ void fill_active(const ra_ctx* ctx, uint32_t* mask)
         if (ctx->active[b]) mask[b >> 5] |= 1u << (b & 31);
 }
 
-// Work split of one layer's attention from the host mirror: head lengths (prompt + cached
-// generated rows, + 1 for a fused new token), their prefix, and slots per warp.
-int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas)
+// Work split of one layer's attention from the host mirror, in tiles: a head has
+// ceil(lp / TILE) prompt tiles and ceil(gen / TILE) tiles of generated rows, where gen is
+// the cached generated rows plus one for a fused new token.  *slots = rows attended.
+int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots)
 {
     fill_active(ctx, p->active);
-    long long acc = 0;
+    const int T = attn_tile_rows(ctx->G);
+    p->tile = T;
+    long long acc = 0, rows = 0;
     int na = 0;
     p->seq_base[0] = 0;
     for (int b = 0; b < ctx->B; ++b) {
+        const int gen = ctx->c[(size_t)layer * ctx->B + b] + fused;
+        p->seq_gen[b] = gen;
+        p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b];
         if (ctx->active[b]) {
-            acc += (long long)ctx->KVH * (ctx->lp[b] + ctx->c[(size_t)layer * ctx->B + b] + fused);
+            acc += (long long)ctx->KVH * ((ctx->lp[b] + T - 1) / T + (gen + T - 1) / T);
+            rows += (long long)ctx->KVH * (ctx->lp[b] + gen);
             ++na;
         }
         p->seq_base[b + 1] = (int32_t)acc;
     }
-    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 slots");
+    if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 tiles");
     p->total = (int)acc;
     const int wpc = attn_warps_per_cta(ctx->G);
     const long long nwarps_max = (long long)ctx->sms * wpc;
-    long long W = (acc + nwarps_max - 1) / nwarps_max;
-    if (W < kMinSlotsPerWarp) W = kMinSlotsPerWarp;
+    long long W = (acc + kChunksPerWarp * nwarps_max - 1) / (kChunksPerWarp * nwarps_max);
+    if (W < 1) W = 1;
     p->W = (int)W;
-    const long long warps = (acc + W - 1) / W;
-    *ctas = (int)((warps + wpc - 1) / wpc);
+    const long long nchunks = (acc + W - 1) / W;
+    p->nchunks = (int)nchunks;
+    *ctas = (int)std::min<long long>(ctx->sms, (nchunks + wpc - 1) / wpc);
+    p->nwarps = *ctas * wpc;
+    if (nchunks <= p->nwarps) p->ticket = nullptr;  // every chunk has a warp of its own: no stealing
     *n_active = na;
-    // partial records are indexed warp + head: both bounded by what the arena holds
-    if ((size_t)(*ctas) * wpc + (size_t)ctx->B * ctx->KVH > ctx->partial_records)
+    *slots = (double)rows;
+    // partial records are indexed chunk + head: both bounded by what the arena holds
+    if ((size_t)nchunks + (size_t)ctx->B * ctx->KVH > ctx->partial_records)
         return fail(ctx, RA_ERR_STATE, "attention split needs more partial records than the arena holds");
     return RA_OK;
+}
+
+// Chunk tickets one launch takes: every stolen chunk, plus one failed take per warp that ran.
+unsigned long long tickets_taken(const AttnParams& p)
+{
+    if (!p.ticket) return 0;
+    const long long stolen = std::max(0, p.nchunks - p.nwarps);
+    return (unsigned long long)(stolen + std::min(p.nchunks, p.nwarps));
 }
 
 void set_scale(AttnParams* p, float scale)
@@ -308,13 +331,15 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_pos = take((size_t)ctx->regions * ctx->Cmax * 4);
     ctx->off_region = take((size_t)layers * batch * kv_heads * 4);
     ctx->off_spare = take((size_t)batch * kv_heads * 4);
-    ctx->off_cnt = take((size_t)layers * batch * sizeof(DevCounters));
     ctx->off_lp = take((size_t)batch * 4);
     ctx->off_poff = take((size_t)batch * 4);
     ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
-    ctx->partial_records = (size_t)kMaxSMs * attn_warps_per_cta(ctx->G) + (size_t)batch * kv_heads;
+    // chunks of the attention split: about kChunksPerWarp per warp (at least one tile each)
+    const size_t max_chunks = (size_t)kChunksPerWarp * kMaxSMs * attn_warps_per_cta(ctx->G) + 1;
+    ctx->partial_records = max_chunks + (size_t)batch * kv_heads;
     ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);
+    ctx->off_ticket = take(sizeof(unsigned long long));
     ctx->off_err = take(256);
     ctx->bytes = o;
     ctx->g.assign((size_t)layers * batch, 0);
@@ -361,12 +386,12 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.pos = (int32_t*)(a + ctx->off_pos);
     Ly.region = (int32_t*)(a + ctx->off_region);
     Ly.spare = (int32_t*)(a + ctx->off_spare);
-    Ly.counters = (DevCounters*)(a + ctx->off_cnt);
     Ly.seq_lp = (int32_t*)(a + ctx->off_lp);
     Ly.seq_poff = (int32_t*)(a + ctx->off_poff);
     Ly.plan = (int32_t*)(a + ctx->off_plan);
     Ly.partial = (float*)(a + ctx->off_partial);
     Ly.arrive = (int32_t*)(a + ctx->off_arrive);
+    Ly.ticket = (unsigned long long*)(a + ctx->off_ticket);
     Ly.err = (int32_t*)(a + ctx->off_err);
     Ly.prompt_rows_per_layer = ctx->prompt_rows_per_layer;
     Ly.gen_row0 = ctx->prompt_rows_per_layer * ctx->L;
@@ -385,17 +410,15 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     std::vector<int32_t> region((size_t)ctx->L * BH), spare(BH);
     for (size_t i = 0; i < region.size(); ++i) region[i] = (int32_t)i;
     for (int i = 0; i < BH; ++i) spare[i] = ctx->L * BH + i;
-    std::vector<DevCounters> cnt((size_t)ctx->L * ctx->B, DevCounters{0, 0, 0, 0});
     int32_t zero = 0;
     // Pageable host sources: cudaMemcpyAsync returns once the data is staged, so the vectors may die here.
     if ((e = cudaMemcpyAsync(Ly.region, region.data(), region.size() * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.spare, spare.data(), spare.size() * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(Ly.counters, cnt.data(), cnt.size() * sizeof(DevCounters), cudaMemcpyHostToDevice, s)) !=
-            cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.seq_lp, ctx->lp.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.seq_poff, ctx->poff.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess)
+        (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess ||
+        (e = cudaMemsetAsync(Ly.ticket, 0, sizeof(unsigned long long), s)) != cudaSuccess)
         return cuda_fail(ctx, e, "table initialisation");
     // rows that were never written (past a head's cached slots) then read as zeros, never as stale NaNs
     if ((e = cudaMemsetAsync(a, 0, ctx->off_pos, s)) != cudaSuccess) return cuda_fail(ctx, e, "cache clear");
@@ -407,6 +430,7 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     if ((rc = make_tmap(ctx, &ctx->tmap_v, Ly.vpool, tile)) != RA_OK) return rc;
     if ((e = attn_prepare(ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
 
+    ctx->ticket_base = 0;
     ctx->arena = a;
     ctx->device = dev;
     ctx->sms = sms;
@@ -461,16 +485,9 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
     p.v = v;
     p.pos = pos;
     p.row_stride = row_stride;
-    std::vector<DevCounters> cnt(ctx->B);
-    for (int b = 0; b < ctx->B; ++b) {
-        p.n_rows[b] = c_host[b];
-        cnt[b] = DevCounters{c_host[b], g_host[b], ctx->nev[(size_t)layer * ctx->B + b], 0};
-    }
+    for (int b = 0; b < ctx->B; ++b) p.n_rows[b] = c_host[b];
     cudaError_t e;
     if (maxc > 0 && (e = launch_restore(p, s)) != cudaSuccess) return cuda_fail(ctx, e, "restore launch");
-    if ((e = cudaMemcpyAsync(ctx->lay.counters + (size_t)layer * ctx->B, cnt.data(), cnt.size() * sizeof(DevCounters),
-                             cudaMemcpyHostToDevice, s)) != cudaSuccess)
-        return cuda_fail(ctx, e, "restore counters");
     for (int b = 0; b < ctx->B; ++b) {
         ctx->g[(size_t)layer * ctx->B + b] = g_host[b];
         ctx->c[(size_t)layer * ctx->B + b] = c_host[b];
@@ -508,6 +525,10 @@ int ra_append_kv(ra_ctx* ctx, int layer, const uint16_t* k_new, const uint16_t* 
     p.k_new = k_new;
     p.v_new = v_new;
     fill_active(ctx, p.active);
+    for (int b = 0; b < ctx->B; ++b) {
+        p.seq_c[b] = ctx->c[(size_t)layer * ctx->B + b];
+        p.seq_g[b] = ctx->g[(size_t)layer * ctx->B + b];
+    }
     cudaStream_t s = (cudaStream_t)stream;
     ProfScope ps(ctx, RA_KERNEL_APPEND, 2.0 * n_active * ctx->KVH * kRowBytes * 2, s);
     cudaError_t e = launch_append(p, ctx->B, s);
@@ -530,7 +551,6 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
     EvictParams p{};
     p.lay = ctx->lay;
     p.layer = layer;
-    p.pending = 0;
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
@@ -538,7 +558,11 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
         const int g = ctx->g[(size_t)layer * ctx->B + b], c = ctx->c[(size_t)layer * ctx->B + b];
         // section 2 / Appendix F trigger: every r steps, once the candidates exceed the budget
         if (g > 0 && g % ctx->r == 0 && c - ctx->r > ctx->K) {
-            p.trig[n++] = (int16_t)b;
+            p.trig[n] = (int16_t)b;
+            p.trig_c[n] = c;
+            p.trig_n[n] = c - ctx->r;
+            p.trig_g[n] = g;
+            ++n;
             moved += (double)(ctx->K + ctx->r) * ctx->KVH;
         }
     }
@@ -581,16 +605,20 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     p.out = out;
     p.partial = ctx->lay.partial;
     p.arrive = ctx->lay.arrive;
+    p.ticket = ctx->lay.ticket;
+    p.ticket_base = ctx->ticket_base;
     int n_active = 0;
     int ctas = 0;
-    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas)) != RA_OK) return rc;
+    double rows = 0;
+    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
     cudaStream_t s = (cudaStream_t)stream;
-    ProfScope ps(ctx, RA_KERNEL_ATTN, (double)p.total * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes, s);
+    ProfScope ps(ctx, RA_KERNEL_ATTN, rows * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes, s);
     cudaError_t e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
+    if (p.total > 0) ctx->ticket_base += tickets_taken(p);
     return RA_OK;
 }
 
@@ -614,14 +642,17 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     EvictParams ep{};
     ep.lay = ctx->lay;
     ep.layer = layer;
-    ep.pending = 1;
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
         if (!ctx->active[b]) continue;
         const int g1 = ctx->g[base + b] + 1, c1 = ctx->c[base + b] + 1;
         if (g1 % ctx->r == 0 && c1 - ctx->r > ctx->K) {
-            ep.trig[n++] = (int16_t)b;
+            ep.trig[n] = (int16_t)b;
+            ep.trig_c[n] = c1 - 1;
+            ep.trig_n[n] = c1 - ctx->r;
+            ep.trig_g[n] = g1;
+            ++n;
             moved += (double)(ctx->K + ctx->r - 1) * ctx->KVH;
         }
     }
@@ -655,20 +686,30 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     p.v_new = v_new;
     p.partial = ctx->lay.partial;
     p.arrive = ctx->lay.arrive;
+    p.ticket = ctx->lay.ticket;
+    p.ticket_base = ctx->ticket_base;
     int n_active = 0, ctas = 0;
-    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas)) != RA_OK) return rc;
+    double rows = 0;
+    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
-    for (int b = 0; b < ctx->B; ++b) p.seq_g[b] = ctx->g[base + b];
     set_scale(&p, scale);
+    // The kernel may request its first K/V tiles before its predecessor finishes when that
+    // predecessor cannot be writing this layer's cache or tables: no eviction of this layer at
+    // this step (else it is this layer's compaction) and more than one layer (else it is this
+    // layer's previous step).  Kernels let successors start only after their own wait, so
+    // everything older than the predecessor has completed.
+    p.early = (n == 0 && ctx->L >= 2 && p.ticket == nullptr) ? 1 : 0;
     {
+        // rows read (the new token's from the caller), its row written, q read, out written
         ProfScope ps(ctx, RA_KERNEL_ATTN,
-                     (double)p.total * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes +
+                     rows * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes +
                          (double)n_active * ctx->KVH * 2 * kRowBytes,
                      s);
         e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
         ps.done();
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
+    if (p.total > 0) ctx->ticket_base += tickets_taken(p);
     for (int b = 0; b < ctx->B; ++b) {
         if (!ctx->active[b]) continue;
         ctx->c[base + b] += 1;
@@ -880,24 +921,26 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     p.q = q;
     p.out = out;
     int n_active = 0, ctas = 0;
-    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas)) != RA_OK) return rc;
+    double rows = 0;
+    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
-    const long long warps = p.total > 0 ? ((long long)p.total + p.W - 1) / p.W : 0;
-    // [arrival counters, one int per (seq, KV head)][partial records, one per (warp, head) piece]
-    const size_t counters = align_up((size_t)ctx->B * ctx->KVH * sizeof(int32_t), kAlign);
+    // [chunk ticket][arrival counters, one int per (seq, KV head)][partial records, one per (chunk, head) piece]
+    const size_t counters = align_up(sizeof(unsigned long long) + (size_t)ctx->B * ctx->KVH * sizeof(int32_t), kAlign);
     const size_t need =
-        counters + (size_t)(warps + (long long)ctx->B * ctx->KVH) * partial_stride(ctx->G) * sizeof(float);
+        counters + (size_t)(p.nchunks + (long long)ctx->B * ctx->KVH) * partial_stride(ctx->G) * sizeof(float);
     if (need > kNoAllocScratchBytes)
         return fail(ctx, RA_ERR_CAPACITY, "layer needs %zu bytes of split-K scratch; the fixed array holds %zu", need,
                     kNoAllocScratchBytes);
     float* scratch = nullptr;
     if ((rc = noalloc_scratch(ctx, ctx->device, &scratch)) != RA_OK) return rc;
     cudaStream_t s = (cudaStream_t)stream;
-    p.arrive = reinterpret_cast<int32_t*>(scratch);
+    p.ticket = reinterpret_cast<unsigned long long*>(scratch);
+    p.ticket_base = 0;
+    p.arrive = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(scratch) + sizeof(unsigned long long));
     p.partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(scratch) + counters);
-    // the counters must start at zero; the array keeps whatever the previous call left
-    cudaError_t e = cudaMemsetAsync(p.arrive, 0, (size_t)ctx->B * ctx->KVH * sizeof(int32_t), s);
+    // the ticket and the counters must start at zero; the array keeps whatever the previous call left
+    cudaError_t e = cudaMemsetAsync(scratch, 0, counters, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "scratch counter clear");
     e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");

@@ -4,22 +4,25 @@
 //     o = sum_i softmax_i(scale * q . k_i) v_i
 // over the prompt rows and the cached generated rows of (b, h) -- section 2
 // ("Notation"), with the grouped-query sharing of Appendix F.  In the fused
-// form the step's new token (Appendix F: appended post-RoPE every step) is one
-// more slot: it is read from the caller's k_new/v_new rows, attended, and
-// written into the cache by the warp that consumes it.
+// form the step's new token (Appendix F: appended post-RoPE every step) is the
+// last generated row: it is read from the caller's k_new/v_new rows, placed in
+// its head's last tile, attended, and written into the cache by the warp that
+// consumes that tile.
 //
-// Work split ("stream-K" by warp): the slots of all heads of the layer are laid
-// end to end (sequence-major, then KV head; within a head the prompt rows, the
-// cached generated rows, then the new token) and every warp of the grid takes
-// one contiguous range of W slots.  A warp runs its own pipeline: lane 0
-// streams tiles of TILE rows of K and of V (and, at the first tile of each head
-// piece, the G query rows) into a ring of SPW shared-memory stages with 2-D TMA
-// loads completing on per-stage mbarriers; all 32 lanes consume.  A head that
-// fits in one warp's range is finished in registers.  Otherwise each (head,
-// warp) piece writes an fp32 partial (unnormalised o, running max m, sum l) to
-// slot `warp + head` -- unique because warps and heads both advance
-// monotonically through the slot order -- and the last warp to finish a piece
-// of that head (an arrival counter per head) merges all of them.
+// Work split: every head is cut into tiles of TILE rows (its prompt rows, then
+// its generated rows); the tiles of all heads of the layer are laid end to end
+// (sequence-major, then KV head) and cut into equal chunks of W tiles, one per
+// warp, so every warp makes the same number of pipeline trips.  (A warp may
+// steal further chunks from an atomic ticket when chunks outnumber warps.)  A
+// warp runs its own pipeline: lane 0 streams the tiles of K and V -- each as
+// two 64-channel boxes stored with the 128-byte swizzle -- plus, at the first
+// tile of each head piece, the G query rows, into a ring of SPW shared-memory
+// stages with 2-D TMA loads completing on per-stage mbarriers; all 32 lanes
+// consume.  A head that fits in one chunk is finished in registers.  Otherwise
+// each (head, chunk) piece writes an fp32 partial (unnormalised o, running max
+// m, sum l) to record `chunk + head` -- unique because chunks and heads both
+// advance monotonically through the tile order -- and the last warp to finish
+// a piece of that head (an arrival counter per head) merges all of them.
 //
 // Per-warp compute: the contraction of the G query rows with a tile of cache
 // rows runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
@@ -54,13 +57,13 @@ constexpr int kHalfCh = 64;                        // channels per swizzled TMA 
 // Kernel shape: rows per stage (a multiple of 16), stages per warp, warps per CTA
 // (one CTA per SM; the warp count is capped by what fits in shared memory).
 #ifndef RA_ATTN_TILE
-#define RA_ATTN_TILE 16
+#define RA_ATTN_TILE 64
 #endif
 #ifndef RA_ATTN_SPW
-#define RA_ATTN_SPW 3
+#define RA_ATTN_SPW 2
 #endif
 #ifndef RA_ATTN_WARPS
-#define RA_ATTN_WARPS 8
+#define RA_ATTN_WARPS 3
 #endif
 
 template <int G>
@@ -69,7 +72,8 @@ struct Cfg {
     static constexpr int HALF_BYTES = TILE * 128;                            // one 64-channel half of K or V
     static constexpr int KV_BYTES = 2 * HALF_BYTES;                          // a K (or V) tile
     static constexpr int Q_BYTES = G * kRowBytes;
-    static constexpr int STAGE_BYTES = (2 * KV_BYTES + Q_BYTES + 1023) / 1024 * 1024;
+    static constexpr int NT_OFF = 2 * KV_BYTES + Q_BYTES;  // the fused new token's K and V rows (unswizzled)
+    static constexpr int STAGE_BYTES = (NT_OFF + 2 * kRowBytes + 1023) / 1024 * 1024;
     static constexpr int SPW = RA_ATTN_SPW;
     static constexpr int WARPS_FIT = kSmemBudget / (SPW * STAGE_BYTES);
     static constexpr int WARPS = WARPS_FIT < RA_ATTN_WARPS ? WARPS_FIT : RA_ATTN_WARPS;
@@ -88,21 +92,24 @@ struct Cfg {
 
 constexpr int kFirst = 1, kLast = 2, kNewTok = 4;
 
-// Producer-side walk over the warp's slot range.
+// Producer-side walk over the warp's chunks (chunks and cursors count tiles).
 struct TileIter {
-    int f, end;           // flattened cursor and end of the warp's range
-    int b, h, pos;        // current sequence, KV head, slot within the head
-    int hl, lp, cg;       // head length, prompt length, cached generated rows (excl. a fused new token)
-    long long prow, grow; // first prompt row / first generated row of the head
+    int chunk;                       // current chunk (-1: none yet)
+    unsigned long long next_ticket;  // lane 0: ticket taken ahead for the chunk after this one
+    int f, end;                      // flattened tile cursor and end of the current chunk
+    int b, h, k;                     // current sequence, KV head, tile within the head
+    int nt, tp;                      // tiles in the head, prompt tiles among them
+    int lp, gen;                     // prompt rows, generated rows (incl. a fused new token)
+    long long prow, grow;            // first prompt row / first generated row of the head
     bool piece_start;
 };
 
 struct TileDesc {
-    long long row;  // first cache row (TMA) or the cache row the new token goes to
-    int n, hid, flags;
+    long long row;  // first cache row of the tile
+    int n, hid, flags, chunk;
 };
 
-__device__ __forceinline__ int seq_head_len(const AttnParams& p, int b)
+__device__ __forceinline__ int seq_head_tiles(const AttnParams& p, int b)
 {
     return (p.seq_base[b + 1] - p.seq_base[b]) / p.lay.KVH;
 }
@@ -110,10 +117,10 @@ __device__ __forceinline__ int seq_head_len(const AttnParams& p, int b)
 __device__ __forceinline__ void enter_head(TileIter& it, const AttnParams& p)
 {
     const DevLayout& L = p.lay;
-    const int lp = L.seq_lp[it.b];
-    it.lp = lp < it.hl ? lp : it.hl;
-    it.cg = it.hl - it.lp - (p.k_new ? 1 : 0);
-    it.prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[it.b] + (long long)it.h * lp;
+    it.lp = L.seq_lp[it.b];
+    it.gen = p.seq_gen[it.b];
+    it.tp = (it.lp + p.tile - 1) / p.tile;
+    it.prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[it.b] + (long long)it.h * it.lp;
     const int reg = L.region[((size_t)p.layer * L.B + it.b) * L.KVH + it.h];
     it.grow = L.gen_row0 + (long long)reg * L.Cmax;
     it.piece_start = true;
@@ -131,43 +138,63 @@ __device__ void iter_init(TileIter& it, const AttnParams& p, int R0, int R1)
     int b = lo;
     while (b < p.lay.B && p.seq_base[b + 1] <= R0) ++b;
     it.b = b;
-    it.hl = seq_head_len(p, b);
+    it.nt = seq_head_tiles(p, b);
     const int off = R0 - p.seq_base[b];
-    it.h = off / it.hl;
-    it.pos = off - it.h * it.hl;
+    it.h = off / it.nt;
+    it.k = off - it.h * it.nt;
     enter_head(it, p);
 }
 
-__device__ bool iter_next(TileIter& it, const AttnParams& p, int tile, TileDesc& d)
+// Next chunk of this warp: its own index first, then stolen ones; false when none is left.
+// Called by all lanes together (lane 0 takes the tickets).
+__device__ bool iter_next_chunk(TileIter& it, const AttnParams& p, int warp_id, int lane)
 {
-    if (it.f >= it.end) return false;
-    const int gen_end = it.lp + it.cg;  // slots [gen_end, hl) hold the fused new token
-    const int seg_end = it.pos < it.lp ? it.lp : (it.pos < gen_end ? gen_end : it.hl);
-    const int rem = it.end - it.f;
-    const int piece_end = (it.hl - it.pos < rem) ? it.hl : it.pos + rem;
-    int n = (seg_end < piece_end ? seg_end : piece_end) - it.pos;
-    if (n > tile) n = tile;
-    d.flags = (it.piece_start ? kFirst : 0) | (it.pos + n == piece_end ? kLast : 0);
-    if (it.pos < it.lp) {
-        d.row = it.prow + it.pos;
+    int c;
+    if (it.chunk < 0) {
+        c = warp_id;
     } else {
-        d.row = it.grow + (it.pos - it.lp);
-        if (it.pos >= gen_end) d.flags |= kNewTok;  // row = its destination slot in the cache
+        if (!p.ticket) return false;  // every chunk has a warp of its own: nothing to steal
+        const unsigned long long raw = __shfl_sync(0xffffffffu, it.next_ticket, 0);
+        c = p.nwarps + (int)(raw - p.ticket_base);
     }
-    d.n = n;
+    if (c >= p.nchunks) return false;
+    // Take the ticket for the chunk after this one now: its latency hides behind this chunk's loads.
+    if (lane == 0 && p.ticket) it.next_ticket = atomicAdd(p.ticket, 1ull);
+    it.chunk = c;
+    const int R0 = c * p.W;
+    iter_init(it, p, R0, min(p.total, R0 + p.W));
+    return true;
+}
+
+__device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int warp_id, int lane)
+{
+    if (it.f >= it.end && !iter_next_chunk(it, p, warp_id, lane)) return false;
+    const int T = p.tile;
+    d.flags = it.piece_start ? kFirst : 0;
+    if (it.k < it.tp) {
+        d.row = it.prow + (long long)it.k * T;
+        d.n = min(T, it.lp - it.k * T);
+    } else {
+        const int kg = it.k - it.tp;
+        d.row = it.grow + (long long)kg * T;
+        d.n = min(T, it.gen - kg * T);
+        if (p.k_new && kg * T + d.n == it.gen) d.flags |= kNewTok;  // its last row is the step's new token
+    }
+    if (it.k + 1 == it.nt || it.f + 1 == it.end) d.flags |= kLast;
     d.hid = it.b * p.lay.KVH + it.h;
+    d.chunk = it.chunk;
     it.piece_start = false;
-    it.pos += n;
-    it.f += n;
-    if (it.pos == it.hl && it.f < it.end) {  // next head (skipping finished sequences)
+    ++it.k;
+    ++it.f;
+    if (it.k == it.nt && it.f < it.end) {  // next head (skipping finished sequences)
         if (++it.h == p.lay.KVH) {
             it.h = 0;
             do {
                 ++it.b;
-            } while (seq_head_len(p, it.b) == 0);
-            it.hl = seq_head_len(p, it.b);
+            } while (seq_head_tiles(p, it.b) == 0);
+            it.nt = seq_head_tiles(p, it.b);
         }
-        it.pos = 0;
+        it.k = 0;
         enter_head(it, p);
     }
     return true;
@@ -215,47 +242,62 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi)) << 16);
 }
 
-// Merge every piece of head `hid` (pieces are partial records w0 + p + hid, p < P)
+// Merge every piece of head `hid` (pieces are partial records c0 + q + hid, q < P)
 // into the bf16 output rows of its G query heads.  One warp; lanes split as
-// (query head, channel block).  Partials come from other SMs: read through L2.
+// (query head g, sub-lane).  The sub-lanes of a head load the statistics of up
+// to LG pieces at once and the O loads of those pieces are all independent, so
+// each group of LG pieces costs about one round of L2 latency.  Partials come
+// from other SMs: read through L2.
 template <int G>
-__device__ void merge_head(const AttnParams& p, int hid, int w0, int P, int lane)
+__device__ void merge_head(const AttnParams& p, int hid, int c0, int P, int lane)
 {
     using C = Cfg<G>;
-    const int g = lane / C::LG;
-    const int c0 = (lane % C::LG) * C::MCH;
-    if (g >= G) return;
+    const int g = lane / C::LG, sub = lane % C::LG;
+    const int gg = g < G ? g : 0;  // lanes of padding heads shadow head 0 (results unused)
+    const int ch0 = sub * C::MCH;
     const size_t rs = (size_t)partial_stride(G);
-    const float* base = p.partial + (size_t)(w0 + hid) * rs;
+    const float* base = p.partial + (size_t)(c0 + hid) * rs;
     float M = -INFINITY;
-#pragma unroll 4
-    for (int q = 0; q < P; ++q) M = fmaxf(M, __ldcg(base + q * rs + G * kHeadDim + g));
+    for (int q = sub; q < P; q += C::LG) M = fmaxf(M, __ldcg(base + q * rs + G * kHeadDim + gg));
+#pragma unroll
+    for (int o = 1; o < C::LG; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
     float Lsum = 0.f;
     float4 acc[C::MCH / 4];
 #pragma unroll
     for (int j = 0; j < C::MCH / 4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 2
-    for (int q = 0; q < P; ++q) {
-        const float* rec = base + q * rs;
-        const float a = exp2f(__ldcg(rec + G * kHeadDim + g) - M);
-        Lsum = fmaf(a, __ldcg(rec + G * kHeadDim + G + g), Lsum);
-        const float4* o = reinterpret_cast<const float4*>(rec + g * kHeadDim + c0);
+    for (int q0 = 0; q0 < P; q0 += C::LG) {
+        float a = 0.f;
+        if (q0 + sub < P) {
+            const float* rec = base + (q0 + sub) * rs;
+            a = exp2f(__ldcg(rec + G * kHeadDim + gg) - M);
+            Lsum = fmaf(a, __ldcg(rec + G * kHeadDim + G + gg), Lsum);
+        }
 #pragma unroll
-        for (int j = 0; j < C::MCH / 4; ++j) {
-            const float4 v = __ldcg(o + j);
-            acc[j].x = fmaf(a, v.x, acc[j].x);
-            acc[j].y = fmaf(a, v.y, acc[j].y);
-            acc[j].z = fmaf(a, v.z, acc[j].z);
-            acc[j].w = fmaf(a, v.w, acc[j].w);
+        for (int j = 0; j < C::LG; ++j) {
+            const float aj = __shfl_sync(0xffffffffu, a, g * C::LG + j);
+            if (q0 + j < P) {
+                const float4* o = reinterpret_cast<const float4*>(base + (q0 + j) * rs + gg * kHeadDim + ch0);
+#pragma unroll
+                for (int k = 0; k < C::MCH / 4; ++k) {
+                    const float4 v = __ldcg(o + k);
+                    acc[k].x = fmaf(aj, v.x, acc[k].x);
+                    acc[k].y = fmaf(aj, v.y, acc[k].y);
+                    acc[k].z = fmaf(aj, v.z, acc[k].z);
+                    acc[k].w = fmaf(aj, v.w, acc[k].w);
+                }
+            }
         }
     }
+#pragma unroll
+    for (int o = 1; o < C::LG; o <<= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
+    if (g >= G) return;
     const float inv = 1.f / Lsum;
     const int b = hid / p.lay.KVH, h = hid - b * p.lay.KVH;
-    uint16_t* out = p.out + ((size_t)b * p.lay.H + (size_t)h * G + g) * kHeadDim + c0;
+    uint16_t* out = p.out + ((size_t)b * p.lay.H + (size_t)h * G + g) * kHeadDim + ch0;
 #pragma unroll
-    for (int j = 0; j < C::MCH / 4; ++j) {
-        const uint2 w = make_uint2(pack_bf16x2(acc[j].x * inv, acc[j].y * inv), pack_bf16x2(acc[j].z * inv, acc[j].w * inv));
-        *reinterpret_cast<uint2*>(out + 4 * j) = w;
+    for (int k = 0; k < C::MCH / 4; ++k) {
+        const uint2 w = make_uint2(pack_bf16x2(acc[k].x * inv, acc[k].y * inv), pack_bf16x2(acc[k].z * inv, acc[k].w * inv));
+        *reinterpret_cast<uint2*>(out + 4 * k) = w;
     }
 }
 
@@ -273,12 +315,12 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
     int4* hdrs = reinterpret_cast<int4*>(smem + (size_t)C::NSTAGE * C::STAGE_BYTES) + warp * C::SPW;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)C::NSTAGE * C::STAGE_BYTES + C::NSTAGE * 16) + warp * C::SPW;
 
-    pdl_launch_dependents();
     const int gw = blockIdx.x * C::WARPS + warp;
-    const long long R0l = (long long)gw * p.W;
-    if (R0l >= p.total) return;
-    const int R0 = (int)R0l;
-    const int R1 = (int)min((long long)p.total, R0l + p.W);
+    if (gw >= p.nchunks) {  // no chunk for this warp (it takes no ticket either)
+        pdl_wait();
+        pdl_launch_dependents();
+        return;
+    }
 
     if (lane == 0) {
         for (int s = 0; s < C::SPW; ++s) mbar_init(&bars[s], 1);
@@ -287,45 +329,61 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         prefetch_tensormap(&tv);
     }
     __syncwarp();
-    pdl_wait();  // the cache, the region table and the inputs may come from the previous kernel
+    // The cache, the region table and the inputs may come from the previous kernel.  With
+    // p.early (the host has checked that the previous kernel writes none of this layer's
+    // cache or tables) the first tiles' K and V are requested before waiting; the query
+    // rows and the new token's row, which the caller may have just produced, come after.
+    if (!p.early) pdl_wait();
 
     TileIter it;
-    iter_init(it, p, R0, R1);
+    it.chunk = -1;
+    it.next_ticket = 0;
+    it.f = it.end = 0;
     int issued = 0;
-    auto issue = [&](int t) -> bool {
+    // The caller's rows of a stage: the query rows (first tile of a piece), the new token's row.
+    auto issue_inputs = [&](int s) {
+        const int4 hd = hdrs[s];
+        uint8_t* st = wstage + (size_t)s * C::STAGE_BYTES;
+        const int b = hd.z / p.lay.KVH, h = hd.z - b * p.lay.KVH;
+        if (hd.y & kNewTok) {
+            const size_t src = ((size_t)b * p.lay.KVH + h) * kHeadDim;
+            bulk_load(st + C::NT_OFF, p.k_new + src, (uint32_t)kRowBytes, &bars[s]);
+            bulk_load(st + C::NT_OFF + kRowBytes, p.v_new + src, (uint32_t)kRowBytes, &bars[s]);
+        }
+        if (hd.y & kFirst)
+            bulk_load(st + 2 * C::KV_BYTES, p.q + ((size_t)b * p.lay.H + (size_t)h * G) * kHeadDim,
+                      (uint32_t)C::Q_BYTES, &bars[s]);
+    };
+    auto issue = [&](int t, bool inputs) -> bool {
         TileDesc d;
-        if (!iter_next(it, p, C::TILE, d)) return false;
+        if (!iter_next(it, p, d, gw, lane)) return false;
         const int s = t % C::SPW;
         if (lane == 0) {
             uint8_t* st = wstage + (size_t)s * C::STAGE_BYTES;
-            hdrs[s] = make_int4(d.n, d.flags, d.hid, (int)d.row);
+            hdrs[s] = make_int4(d.n, d.flags | (d.chunk << 3), d.hid, (int)d.row);
             const bool first = d.flags & kFirst;
-            const uint32_t kv = (d.flags & kNewTok) ? 2u * kRowBytes : 2u * C::KV_BYTES;
-            mbar_arrive_expect_tx(&bars[s], kv + (first ? (uint32_t)C::Q_BYTES : 0u));
-            const int b = d.hid / p.lay.KVH, h = d.hid - b * p.lay.KVH;
-            if (d.flags & kNewTok) {  // the step's new token comes from the caller's rows (row 0, unswizzled)
-                const size_t src = ((size_t)b * p.lay.KVH + h) * kHeadDim;
-                bulk_load(st, p.k_new + src, 128u, &bars[s]);
-                bulk_load(st + C::HALF_BYTES, p.k_new + src + kHalfCh, 128u, &bars[s]);
-                bulk_load(st + C::KV_BYTES, p.v_new + src, 128u, &bars[s]);
-                bulk_load(st + C::KV_BYTES + C::HALF_BYTES, p.v_new + src + kHalfCh, 128u, &bars[s]);
-            } else {
-                tma_load_2d(st, &tk, 0, (int)d.row, &bars[s]);
-                tma_load_2d(st + C::HALF_BYTES, &tk, kHalfCh, (int)d.row, &bars[s]);
-                tma_load_2d(st + C::KV_BYTES, &tv, 0, (int)d.row, &bars[s]);
-                tma_load_2d(st + C::KV_BYTES + C::HALF_BYTES, &tv, kHalfCh, (int)d.row, &bars[s]);
-            }
-            if (first)
-                bulk_load(st + 2 * C::KV_BYTES, p.q + ((size_t)b * p.lay.H + (size_t)h * G) * kHeadDim,
-                          (uint32_t)C::Q_BYTES, &bars[s]);
+            const bool newtok = d.flags & kNewTok;
+            mbar_arrive_expect_tx(&bars[s], 2u * C::KV_BYTES + (first ? (uint32_t)C::Q_BYTES : 0u) +
+                                                (newtok ? 2u * kRowBytes : 0u));
+            tma_load_2d(st, &tk, 0, (int)d.row, &bars[s]);
+            tma_load_2d(st + C::HALF_BYTES, &tk, kHalfCh, (int)d.row, &bars[s]);
+            tma_load_2d(st + C::KV_BYTES, &tv, 0, (int)d.row, &bars[s]);
+            tma_load_2d(st + C::KV_BYTES + C::HALF_BYTES, &tv, kHalfCh, (int)d.row, &bars[s]);
+            if (inputs) issue_inputs(s);
         }
         return true;
     };
     bool more = true;
     for (int t = 0; t < C::SPW && more; ++t) {
-        more = issue(t);
+        more = issue(t, !p.early);
         if (more) ++issued;
     }
+    if (p.early) {
+        pdl_wait();
+        if (lane == 0)
+            for (int t = 0; t < issued; ++t) issue_inputs(t);
+    }
+    pdl_launch_dependents();  // only now: the successor may assume our predecessor has completed
 
     const int gq = lane >> 2;  // this lane's query head (rows >= G are padding)
     const int tq = lane & 3;
@@ -358,6 +416,16 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
                 qa[kk][0] = gq < G ? *reinterpret_cast<const uint32_t*>(Qs + gq * kRowBytes + (16 * kk + 2 * tq) * 2) : 0u;
                 qa[kk][1] = gq < G ? *reinterpret_cast<const uint32_t*>(Qs + gq * kRowBytes + (16 * kk + 8 + 2 * tq) * 2) : 0u;
             }
+        }
+        if (hd.y & kNewTok) {  // fused append: put the new token in row n-1 of the tile and into the cache
+            const int b = hd.z / p.lay.KVH;
+            const int c = lane & 15;
+            const uint4 v = lds128(Ks + C::NT_OFF + (lane >> 4) * kRowBytes + c * 16);
+            *reinterpret_cast<uint4*>((lane < 16 ? Ks : Vs) + swz<G>(n - 1, c)) = v;
+            const long long row = (long long)hd.w + n - 1;
+            reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[c] = v;
+            if (lane == 0) p.lay.pos[row - p.lay.gen_row0] = p.lay.seq_lp[b] + p.seq_g[b];
+            __syncwarp();
         }
         if (n < C::TILE) {  // rows past the valid ones hold stale data: zero V there so 0 * V stays 0
             const int nb = (n + 15) & ~15;  // only rows inside the last used 16-row batch matter
@@ -413,33 +481,15 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             }
         }
 
-        if (hd.y & kNewTok) {  // fused append: the new token's K/V row and position go into the cache
-            const int b = hd.z / p.lay.KVH, h = hd.z - b * p.lay.KVH;
-            const long long row = hd.w;
-            const int c = lane & 15;  // row 0 of the tile is unswizzled: chunk c of the (c >> 3) half
-            const uint4 v = lds128((lane < 16 ? Ks : Vs) + (c >> 3) * C::HALF_BYTES + (c & 7) * 16);
-            reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[c] = v;
-            if (lane == 0) {
-                const long long slot = row - p.lay.gen_row0;  // region * Cmax + cached index
-                const int g0 = p.seq_g[b];
-                p.lay.pos[slot] = p.lay.seq_lp[b] + g0;
-                if (h == 0) {
-                    DevCounters* cnt = p.lay.counters + (size_t)p.layer * p.lay.B + b;
-                    cnt->c = (int)(slot % p.lay.Cmax) + 1;
-                    cnt->g = g0 + 1;
-                }
-            }
-        }
-
         if (hd.y & kLast) {  // last tile of the piece
             float l = l_run;
             l += __shfl_xor_sync(0xffffffffu, l, 1);
             l += __shfl_xor_sync(0xffffffffu, l, 2);
             const int hid = hd.z;
             const int b = hid / p.lay.KVH, h = hid - b * p.lay.KVH;
-            const int hl = seq_head_len(p, b);
-            const long long A = p.seq_base[b] + (long long)h * hl;
-            const int w0 = (int)(A / p.W), w1 = (int)((A + hl - 1) / p.W);
+            const int nth = seq_head_tiles(p, b);
+            const long long A = p.seq_base[b] + (long long)h * nth;
+            const int w0 = (int)(A / p.W), w1 = (int)((A + nth - 1) / p.W);
             if (w0 == w1) {  // the whole head was this warp's: normalise and write the output
                 if (gq < G) {
                     const float inv = 1.f / l;
@@ -448,7 +498,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
                     for (int nt = 0; nt < 16; ++nt) out[nt * 4 + tq] = pack_bf16x2(O[nt][0] * inv, O[nt][1] * inv);
                 }
             } else {
-                float* rec = p.partial + (size_t)(gw + hid) * partial_stride(G);
+                float* rec = p.partial + (size_t)((hd.y >> 3) + hid) * partial_stride(G);
                 if (gq < G) {
 #pragma unroll
                     for (int nt = 0; nt < 16; ++nt)
@@ -478,7 +528,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         __syncwarp();
         if (more) {  // refill the stage just consumed with the tile SPW ahead
             if (lane == 0) fence_proxy_async_smem();
-            more = issue(t + C::SPW);
+            more = issue(t + C::SPW, true);
             if (more) ++issued;
         }
     }
@@ -488,8 +538,8 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
 // attend over nothing: their output rows are zero.
 __global__ void __launch_bounds__(256) zero_empty_kernel(const __grid_constant__ AttnParams p)
 {
-    pdl_launch_dependents();
     pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     if (!((p.active[b >> 5] >> (b & 31)) & 1u) || p.seq_base[b + 1] != p.seq_base[b]) return;
     uint16_t* out = p.out + (size_t)b * p.lay.H * kHeadDim;

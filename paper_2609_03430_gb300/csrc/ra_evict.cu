@@ -50,14 +50,13 @@ __device__ __forceinline__ bool bit_on(const uint32_t* mask, int b) { return (ma
 // ----------------------------------------------------------------------------- append
 __global__ void __launch_bounds__(1024) append_kernel(const __grid_constant__ AppendParams p)
 {
-    pdl_launch_dependents();
     pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     if (!bit_on(p.active, b)) return;
     const DevLayout& L = p.lay;
     const int h = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    DevCounters* cnt = L.counters + (size_t)p.layer * L.B + b;
-    const int c = cnt->c, g = cnt->g;
+    const int c = p.seq_c[b], g = p.seq_g[b];
     const int reg = L.region[((size_t)p.layer * L.B + b) * L.KVH + h];
     const long long row = L.gen_row0 + (long long)reg * L.Cmax + c;
     const size_t src = ((size_t)b * L.KVH + h) * kHeadDim;
@@ -69,11 +68,6 @@ __global__ void __launch_bounds__(1024) append_kernel(const __grid_constant__ Ap
         reinterpret_cast<uint4*>(L.vpool + row * kHeadDim)[lane - 16] = v;
     }
     if (lane == 0) L.pos[(size_t)reg * L.Cmax + c] = L.seq_lp[b] + g;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        cnt->c = c + 1;
-        cnt->g = g + 1;
-    }
 }
 
 // ----------------------------------------------------------------------------- select
@@ -84,19 +78,19 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     extern __shared__ uint32_t sm[];
     __shared__ uint32_t hist[256];
     __shared__ uint32_t s_bin, s_before, s_total;
-    pdl_launch_dependents();
     pdl_wait();
+    pdl_launch_dependents();
     const DevLayout& L = p.lay;
     const int b = p.trig[blockIdx.x], h = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const DevCounters cnt = L.counters[(size_t)p.layer * L.B + b];
     // With a pending token (fused step) the cache holds c rows and the token about to be
-    // appended is the newest slot: candidates and the step count include it.
-    const int c = cnt.c, g = cnt.g + p.pending, K = L.K, r = L.r;
-    const int N = c + p.pending - r, m = N - K;
+    // appended is the newest slot: the candidate count and the step include it.
+    const int c = p.trig_c[blockIdx.x], N = p.trig_n[blockIdx.x], g = p.trig_g[blockIdx.x];
+    const int K = L.K, r = L.r;
+    const int m = N - K;
     const int head_id = b * L.KVH + h;
     int32_t* plan = L.plan + (size_t)head_id * (kPlanHeader + r);
-    if (m <= 0 || m > r || N > kMaxCandidates) {  // the host mirror rules this out; never move data on a bad plan
+    if (m <= 0 || m > r || N > kMaxCandidates || N > c) {  // the host mirror rules this out; never move data on a bad plan
         if (tid == 0) {
             atomicExch(L.err, kDeviceErrPlan);
             plan[3] = 0;
@@ -237,8 +231,8 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
     extern __shared__ int32_t s_ev[];
     __shared__ int32_t s_hdr[4];
     __shared__ int32_t s_dst[kCompactChunk];
-    pdl_launch_dependents();
     pdl_wait();
+    pdl_launch_dependents();
     const DevLayout& L = p.lay;
     const int t = blockIdx.y / L.KVH, h = blockIdx.y % L.KVH;
     const int b = p.trig[t];
@@ -290,11 +284,6 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
                 if (lane == 0) dpos[dj[u]] = pv[u];
             }
         }
-    }
-    if (blockIdx.x == 0 && h == 0 && threadIdx.x == 0) {
-        DevCounters* cnt = L.counters + (size_t)p.layer * L.B + b;
-        cnt->c = c - m;
-        cnt->nev = cnt->nev + 1;
     }
 }
 

@@ -23,14 +23,6 @@ __host__ __device__ constexpr int partial_stride(int G) { return G * 128 + ((2 *
 constexpr int kDeviceErrTimeout = 1;     // values of the device error word
 constexpr int kDeviceErrPlan = 2;
 
-// Device-side per-(layer, seq) counters (mirrored on the host).
-struct DevCounters {
-    int32_t c;    // cached generated tokens
-    int32_t g;    // generated tokens appended
-    int32_t nev;  // evictions so far
-    int32_t pad;
-};
-
 // Pointers into the bound arena plus the static shape of a context.
 struct DevLayout {
     uint16_t* kpool;       // [total_rows][128] bf16: prompt rows of every layer, then generated regions
@@ -38,12 +30,12 @@ struct DevLayout {
     int32_t* pos;          // [regions][Cmax] positions of generated slots
     int32_t* region;       // [L][B][KVH] region index currently holding a head's generated slots
     int32_t* spare;        // [B][KVH] the free region that a head's next compaction writes into
-    DevCounters* counters; // [L][B]
     int32_t* seq_lp;       // [B] prompt length
     int32_t* seq_poff;     // [B] row offset of a sequence's prompt block inside a layer (KVH * sum lp)
     int32_t* plan;         // [B*KVH][kPlanHeader + r] eviction plan of the current layer
     float* partial;        // attention split partials
     int32_t* arrive;       // [B*KVH] split-piece arrival counters
+    unsigned long long* ticket;  // attention chunk-stealing counter
     int32_t* err;          // device error word
     long long prompt_rows_per_layer;
     long long gen_row0;    // first row of the generated regions
@@ -51,36 +43,50 @@ struct DevLayout {
     uint64_t seed;
 };
 
+// Per-sequence counts come from the host mirror (the single source of truth) as launch parameters.
 struct AppendParams {
     DevLayout lay;
     int layer;
     const uint16_t* k_new;  // [B][KVH][128]
     const uint16_t* v_new;
     uint32_t active[RA_MAX_BATCH / 32];
+    int32_t seq_c[RA_MAX_BATCH];  // cached generated rows before the append
+    int32_t seq_g[RA_MAX_BATCH];  // generated tokens before the append (position = lp + g)
 };
 
 struct EvictParams {
     DevLayout lay;
     int layer;
-    int pending;  // 1 when the step's new token is not yet in the cache (fused step): it counts as the newest slot
     int n_trig;
-    int16_t trig[RA_MAX_BATCH];  // triggered sequence ids
+    int16_t trig[RA_MAX_BATCH];    // triggered sequence ids
+    int32_t trig_c[RA_MAX_BATCH];  // rows in the cache (a pending new token is not among them)
+    int32_t trig_n[RA_MAX_BATCH];  // candidates (all rows but the newest r, counting a pending token)
+    int32_t trig_g[RA_MAX_BATCH];  // step of the draw: generated tokens including this step's
 };
 
+// Attention work is counted in tiles of TILE rows: a head has ceil(lp / TILE) prompt tiles and
+// ceil(gen / TILE) tiles of generated rows (gen includes a fused new token, its last row).
 struct AttnParams {
     DevLayout lay;
     int layer;
+    int tile;               // rows per tile
     const uint16_t* q;      // [B][H][128]
     uint16_t* out;          // [B][H][128]
     const uint16_t* k_new;  // fused append: the step's new rows [B][KVH][128]; null = attention only
     const uint16_t* v_new;
     float* partial;         // split-K partial records (arena or the no-alloc array)
     int32_t* arrive;        // [B*KVH] pieces merged so far per head; zero between launches
-    int W;                  // slots per warp (stream-K split)
-    int total;              // total slots of the layer
+    int W;                  // tiles per chunk of the split (a warp's first chunk is its index, later ones are stolen)
+    int total;              // total tiles of the layer
+    int nchunks;            // ceil(total / W)
+    int nwarps;             // warps launched
+    unsigned long long* ticket;  // chunk-stealing counter (never reset: this launch's tickets start at ticket_base)
+    unsigned long long ticket_base;
     float qk_scale_log2;    // scale * log2(e)
+    int early;              // 1: the first tiles' K/V may be loaded before the predecessor kernel finishes
     uint32_t active[RA_MAX_BATCH / 32];
-    int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of head lengths over active sequences
+    int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of tiles per head over active sequences
+    int32_t seq_gen[RA_MAX_BATCH];       // generated rows attended per head (incl. a fused new token)
     int32_t seq_g[RA_MAX_BATCH];         // fused append: tokens generated before this one
 };
 
@@ -109,8 +115,10 @@ cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tmap_k, con
 cudaError_t attn_prepare(int G);  // one-time function attributes (dynamic smem)
 
 // Launch with programmatic dependent launch: the kernel may be scheduled while its
-// predecessor on the stream finishes; every kernel waits (griddepcontrol.wait)
-// before touching memory a predecessor writes.
+// predecessor on the stream finishes.  Every kernel waits (griddepcontrol.wait)
+// before touching memory its predecessor may write, and lets its successor be
+// scheduled only after that wait -- so when a kernel starts, every kernel before
+// its predecessor has completed.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args&&... args)
 {
