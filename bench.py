@@ -239,6 +239,24 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(inside)}
 
 
+def profiled_traffic(cfg):
+    """DRAM bytes per attention launch from the committed ncu record, if it was taken on the
+    current kernel source for this workload's layer shape; else None."""
+    import hashlib
+
+    try:
+        with open(os.path.join(ROOT, "profiles", "attn_kernel_traffic.json")) as f:
+            rec = json.load(f)
+        src = os.path.join(ROOT, "paper_2609_03430_gb300", "csrc", "ra_attn.cu")
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if rec.get("kernel_source_sha256") != digest:
+            return None
+        per_cfg = rec.get("traffic_bytes_per_launch", {})
+        return per_cfg.get(str(cfg))
+    except Exception:
+        return None
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -449,7 +467,10 @@ def run_ours(args, w):
                 "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
                 else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
                 "algorithmic_bytes_per_launch": by_launch, "us_per_launch": a["us_per_launch"],
-                "traffic": args.traffic}
+                "traffic": args.traffic if args.traffic is not None else profiled_traffic(args.config),
+                "timing": "CUDA events around every attention launch on its stream, in a second pass of "
+                          "the same number of steps (events between launches defeat their overlap, so "
+                          "this duration is an upper bound)"}
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)
@@ -459,7 +480,11 @@ def run_ours(args, w):
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_dict(w, args),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                 "clocks": clocks.summary(wall0, wall1), "kernels": kern,
-                "attn_cache_bytes_per_step": attn_bytes_before}
+                "attn_cache_bytes_per_step": attn_bytes_before,
+                "step_effective": {"GBps": attn_bytes_before / (ms_step * 1e-3) / 1e9,
+                                   "frac": attn_bytes_before / (ms_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                                   "what": "cache bytes streamed per step / device time per step "
+                                           "(all kernels of the step, launches overlapped)"}}
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
