@@ -115,6 +115,24 @@ int ra_prefill(ra_ctx* ctx, int layer, const uint16_t* k, const uint16_t* v, int
 int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_host, const int32_t* pos,
                const uint16_t* k, const uint16_t* v, int row_stride, void* stream);
 
+/*
+ * Candidate scoring policy (default RA_POLICY_RANDOM, the method).  The others
+ * are the controls the paper contrasts with it, kept through the same Eq. 1
+ * top-K and compaction:
+ *   RA_POLICY_SHARED   one draw per (sequence, layer) used by every KV head --
+ *                      the shared-draw control (section 5, Appendix D);
+ *   RA_POLICY_RECENCY  keep the K newest candidates -- protected recency, the
+ *                      prompt plus a contiguous recent window (section 4.1, 5);
+ *   RA_POLICY_BLOCK    one draw per block of `block` consecutive positions, so
+ *                      the history is kept in contiguous blocks (section 5).
+ * Takes effect from the next eviction; `block` >= 1 is used by RA_POLICY_BLOCK.
+ */
+#define RA_POLICY_RANDOM 0
+#define RA_POLICY_SHARED 1
+#define RA_POLICY_RECENCY 2
+#define RA_POLICY_BLOCK 3
+int ra_set_policy(ra_ctx* ctx, int policy, int block);
+
 /* Mark sequence `seq` active (1) or finished (0); finished ones are skipped by every call. */
 int ra_set_active(ra_ctx* ctx, int seq, int active);
 

@@ -67,6 +67,14 @@ def _load():
         lib.ora_evict_head.restype = ctypes.c_int
         lib.ora_attend.argtypes = [u16p, u16p, u16p, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                    ctypes.c_double, f64p]
+        lib.ora_policy_key.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_uint32,
+                                       ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32,
+                                       ctypes.c_uint32, ctypes.c_int32, ctypes.c_int32]
+        lib.ora_policy_key.restype = ctypes.c_uint32
+        lib.ora_evict_head_policy.argtypes = [i32p, ctypes.POINTER(ctypes.c_int), ctypes.c_int, ctypes.c_int,
+                                              ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int,
+                                              ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, i32p]
+        lib.ora_evict_head_policy.restype = ctypes.c_int
         lib.ora_attend.restype = None
         _lib = lib
     return _lib
@@ -125,6 +133,23 @@ def evict_head(gen: np.ndarray, g: int, K: int, r: int, seed: int, layer: int, h
     return buf[: c.value].copy(), ev[:m].copy()
 
 
+POLICY_RANDOM, POLICY_SHARED, POLICY_RECENCY, POLICY_BLOCK = 0, 1, 2, 3
+
+
+def evict_head_policy(gen, g, K, r, seed, layer, seq, kv_heads, h, policy, block=1):
+    """One eviction round under a policy variant (random / shared / recency / block)."""
+    buf = np.ascontiguousarray(gen, dtype=np.int32).copy()
+    c = ctypes.c_int(int(buf.size))
+    ev = np.zeros(max(int(buf.size), 1), dtype=np.int32)
+    if buf.size == 0:
+        return buf, ev[:0]
+    m = _load().ora_evict_head_policy(_ptr(buf, ctypes.c_int32), ctypes.byref(c), g, K, r, seed, layer, seq,
+                                      kv_heads, h, policy, block, _ptr(ev, ctypes.c_int32))
+    if m < 0:
+        raise RuntimeError("ora_evict_head_policy failed")
+    return buf[: c.value].copy(), ev[:m].copy()
+
+
 def attend(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float = 0.0) -> np.ndarray:
     """fp64 decode attention of a GQA group: q [G][d], k/v [n][d] bf16 bits -> [G][d] float64."""
     q = np.ascontiguousarray(q, dtype=np.uint16)
@@ -159,7 +184,7 @@ class OracleCache:
     fix the order within a step).
     """
 
-    def __init__(self, layers, kv_heads, prompt_lens, K, r, seed, heads=None):
+    def __init__(self, layers, kv_heads, prompt_lens, K, r, seed, heads=None, policy=0, block=1):
         self.L = layers
         self.KVH = kv_heads
         self.prompt_lens = [int(x) for x in prompt_lens]
@@ -167,6 +192,7 @@ class OracleCache:
         self.K = K
         self.r = r
         self.seed = seed
+        self.policy, self.block = policy, block
         self.g = np.zeros((self.B, layers), dtype=np.int64)
         # heads: iterable of (seq, layer, kv_head) to track; None = all
         if heads is None:
@@ -208,7 +234,11 @@ class OracleCache:
             cur = self.gen[key]
             if not should_evict(g, int(cur.size), self.K, self.r):
                 continue
-            new, ev = evict_head(cur, g, self.K, self.r, self.seed, layer, seq * self.KVH + h)
+            if self.policy == POLICY_RANDOM:
+                new, ev = evict_head(cur, g, self.K, self.r, self.seed, layer, seq * self.KVH + h)
+            else:
+                new, ev = evict_head_policy(cur, g, self.K, self.r, self.seed, layer, seq, self.KVH, h,
+                                            self.policy, self.block)
             self.gen[key] = new
             fired[h] = ev
         if fired:

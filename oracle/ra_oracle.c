@@ -86,6 +86,34 @@ uint32_t ora_random_key(uint64_t seed, uint32_t layer, uint32_t head_id, uint32_
     return out[0];
 }
 
+/*
+ * Scores of the policy variants the paper contrasts with Random Attention
+ * (section 5 and Appendix D), all kept through the same Eq. 1 top-K:
+ *   0 random   -- the method: an independent draw per KV head (see above);
+ *   1 shared   -- the shared-draw control: one draw per (sequence, layer) that
+ *                 every KV head uses (head_id = seq * kv_heads for all heads);
+ *   2 recency  -- protected recency: the prompt plus the most recent window,
+ *                 i.e. the K newest candidates (score N - 1 - j);
+ *   3 block    -- history kept in contiguous blocks: every candidate of one
+ *                 block of `block` consecutive positions shares one draw
+ *                 (counter word 0 = position / block).
+ * Ties of equal score go to the lower ordinal, as everywhere.
+ */
+uint32_t ora_policy_key(int policy, uint64_t seed, uint32_t layer, uint32_t seq, uint32_t kv_heads, uint32_t h,
+                        uint32_t step, uint32_t j, uint32_t n_cand, int32_t position, int32_t block)
+{
+    switch (policy) {
+        case 1:
+            return ora_random_key(seed, layer, seq * kv_heads, step, j);
+        case 2:
+            return n_cand - 1u - j;
+        case 3:
+            return ora_random_key(seed, layer, seq * kv_heads + h, step, (uint32_t)(position / block));
+        default:
+            return ora_random_key(seed, layer, seq * kv_heads + h, step, j);
+    }
+}
+
 /* ------------------------------------------------------------------------- */
 /* Selection: Eq. 1, S_t = top-K over the candidates of s_i.                 */
 /* ------------------------------------------------------------------------- */
@@ -170,6 +198,48 @@ int ora_evict_head(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int
     }
     for (int j = 0; j < n; ++j)
         keys[j] = ora_random_key(seed, (uint32_t)layer, (uint32_t)head_id, (uint32_t)g, (uint32_t)j);
+    if (ora_select_keep(keys, n, K, keep) != 0) {
+        free(keys); free(keep); free(next);
+        return -1;
+    }
+    int m = 0, ki = 0;
+    for (int j = 0; j < n; ++j) {
+        if (ki < K && keep[ki] == j) {
+            next[ki] = gen[j];
+            ++ki;
+        } else {
+            if (evicted_out) evicted_out[m] = j;
+            ++m;
+        }
+    }
+    for (int i = 0; i < r; ++i) next[K + i] = gen[n + i];
+    memcpy(gen, next, sizeof(int32_t) * (size_t)(K + r));
+    *c = K + r;
+    free(keys); free(keep); free(next);
+    return m;
+}
+
+/*
+ * One eviction round under a policy variant (see ora_policy_key); same trigger,
+ * candidates and compaction as ora_evict_head.
+ */
+int ora_evict_head_policy(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int layer, int seq,
+                          int kv_heads, int h, int policy, int block, int32_t* evicted_out)
+{
+    int cc = *c;
+    if (!ora_should_evict(g, cc, K, r)) return 0;
+    if (policy == 3 && block < 1) return -1;
+    int n = cc - r;
+    uint32_t* keys = (uint32_t*)malloc(sizeof(uint32_t) * (size_t)n);
+    int32_t* keep = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
+    int32_t* next = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K + r));
+    if (!keys || !keep || !next) {
+        free(keys); free(keep); free(next);
+        return -1;
+    }
+    for (int j = 0; j < n; ++j)
+        keys[j] = ora_policy_key(policy, seed, (uint32_t)layer, (uint32_t)seq, (uint32_t)kv_heads, (uint32_t)h,
+                                 (uint32_t)g, (uint32_t)j, (uint32_t)n, gen[j], block);
     if (ora_select_keep(keys, n, K, keep) != 0) {
         free(keys); free(keep); free(next);
         return -1;

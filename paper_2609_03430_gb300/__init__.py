@@ -41,6 +41,7 @@ SIGNATURES = {
     "ra_bind": (_i, [_vp, _vp, _sz, _vp]),
     "ra_prefill": (_i, [_vp, _i, _vp, _vp, _i, _vp]),
     "ra_restore": (_i, [_vp, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp]),
+    "ra_set_policy": (_i, [_vp, _i, _i]),
     "ra_set_active": (_i, [_vp, _i, _i]),
     "ra_append_kv": (_i, [_vp, _i, _vp, _vp, _vp]),
     "ra_evict": (_i, [_vp, _i, _ip, _vp]),
@@ -132,6 +133,13 @@ def ra_restore(ctx, layer, g_list, c_list, pos_ptr, k_ptr, v_ptr, row_stride, st
     g = (ctypes.c_int32 * n)(*[int(x) for x in g_list])
     c = (ctypes.c_int32 * n)(*[int(x) for x in c_list])
     return _check(lib().ra_restore(ctx, layer, g, c, pos_ptr, k_ptr, v_ptr, row_stride, _stream_ptr(stream)), ctx)
+
+
+RA_POLICY_RANDOM, RA_POLICY_SHARED, RA_POLICY_RECENCY, RA_POLICY_BLOCK = 0, 1, 2, 3
+
+
+def ra_set_policy(ctx, policy, block=1):
+    return _check(lib().ra_set_policy(ctx, int(policy), int(block)), ctx)
 
 
 def ra_set_active(ctx, seq, active):

@@ -69,6 +69,8 @@ struct ra_ctx {
     // host mirror
     std::vector<int32_t> g, c, nev;  // [L][B]
     std::vector<uint8_t> active;     // [B]
+    int policy = RA_POLICY_RANDOM;   // candidate scoring (ra_set_policy)
+    int block = 1;
     // profiling
     bool prof = false;
     std::vector<ProfRec> pending;
@@ -495,6 +497,17 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
     return RA_OK;
 }
 
+int ra_set_policy(ra_ctx* ctx, int policy, int block)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (policy < RA_POLICY_RANDOM || policy > RA_POLICY_BLOCK)
+        return fail(ctx, RA_ERR_INVALID_ARG, "unknown policy %d", policy);
+    if (policy == RA_POLICY_BLOCK && block < 1) return fail(ctx, RA_ERR_INVALID_ARG, "block must be >= 1");
+    ctx->policy = policy;
+    ctx->block = policy == RA_POLICY_BLOCK ? block : 1;
+    return RA_OK;
+}
+
 int ra_set_active(ra_ctx* ctx, int seq, int active)
 {
     if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
@@ -551,6 +564,8 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
     EvictParams p{};
     p.lay = ctx->lay;
     p.layer = layer;
+    p.policy = ctx->policy;
+    p.block = ctx->block;
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
@@ -642,6 +657,8 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     EvictParams ep{};
     ep.lay = ctx->lay;
     ep.layer = layer;
+    ep.policy = ctx->policy;
+    ep.block = ctx->block;
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {

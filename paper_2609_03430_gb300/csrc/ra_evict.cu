@@ -4,8 +4,10 @@
 //                   and its position go to slot c of the head's region
 //                   (Appendix F: keys stored post-RoPE, cumulative counter).
 //   select_kernel   one CTA per triggered (seq, KV head): Philox4x32-10 score
-//                   per candidate (section 3's i.i.d. uniform draw), radix
-//                   select of the K smallest (score, ordinal) -- Eq. 1 -- and a
+//                   per candidate (section 3's i.i.d. uniform draw; or one of
+//                   the variants the paper contrasts: a draw shared by all heads,
+//                   protected recency, block-contiguous draws), radix select of
+//                   the K smallest (score, ordinal) -- Eq. 1 -- and a
 //                   ballot-compacted, ascending list of the evicted ordinals.
 //   compact_kernel  many CTAs per triggered head: order-preserving move of the
 //                   survivors (kept candidates, then the buffer rows) into
@@ -102,8 +104,18 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     uint32_t* evbits = sm + nwords * 32; // [nwords]
 
     const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
-    for (int j = tid; j < N; j += kSelThreads)
-        keys[j] = philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)p.layer, (uint32_t)head_id, k0, k1);
+    if (p.policy == RA_POLICY_RECENCY) {  // protected recency: the K newest candidates score lowest
+        for (int j = tid; j < N; j += kSelThreads) keys[j] = (uint32_t)(N - 1 - j);
+    } else if (p.policy == RA_POLICY_BLOCK) {  // one draw per block of consecutive positions
+        const int32_t* pos = L.pos + (size_t)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
+        for (int j = tid; j < N; j += kSelThreads)
+            keys[j] = philox4x32_10_w0((uint32_t)(pos[j] / p.block), (uint32_t)g, (uint32_t)p.layer, (uint32_t)head_id,
+                                       k0, k1);
+    } else {  // random: an independent draw per KV head; shared: one draw for all heads of the sequence
+        const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
+        for (int j = tid; j < N; j += kSelThreads)
+            keys[j] = philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)p.layer, id, k0, k1);
+    }
     __syncthreads();
 
     // Radix select of the element at rank K (0-based) of the (key, ordinal) order:

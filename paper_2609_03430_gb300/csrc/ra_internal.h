@@ -57,6 +57,8 @@ struct AppendParams {
 struct EvictParams {
     DevLayout lay;
     int layer;
+    int policy;  // RA_POLICY_*: how candidates are scored
+    int block;   // RA_POLICY_BLOCK: positions per block
     int n_trig;
     int16_t trig[RA_MAX_BATCH];    // triggered sequence ids
     int32_t trig_c[RA_MAX_BATCH];  // rows in the cache (a pending new token is not among them)

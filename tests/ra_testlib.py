@@ -30,7 +30,8 @@ def check_attention(got_bits, ref, what=""):
 class Runner:
     """A small workload run through the C ABI with an oracle mirror of every head."""
 
-    def __init__(self, L, H, KVH, prompt_lens, K, r, eseed, dseed, key_scale=None, D=128, fused=False):
+    def __init__(self, L, H, KVH, prompt_lens, K, r, eseed, dseed, key_scale=None, D=128, fused=False, policy=0,
+                 block=1):
         import torch
 
         import paper_2609_03430_gb300 as ra
@@ -44,7 +45,9 @@ class Runner:
         self.key_scale = key_scale  # fp32 [L][KVH][D] or None
         self.cache = ra.RandomAttentionCache(L, H, KVH, D, self.lp, K, r, eseed)
         self.ctx = self.cache.ctx
-        self.orc = oracle.OracleCache(L, KVH, self.lp, K, r, eseed)
+        self.orc = oracle.OracleCache(L, KVH, self.lp, K, r, eseed, policy=policy, block=block)
+        if policy:
+            ra.ra_set_policy(self.ctx, policy, block)
         self.dev = torch.device("cuda")
         self.step_idx = 0
         self.fused = fused  # True: one ra_decode_layer call per layer instead of append/evict/attend

@@ -55,6 +55,19 @@ def test_group_sizes(G):
     run.close()
 
 
+@pytest.mark.parametrize("policy,block,fused", [(1, 1, True), (2, 1, False), (3, 4, True), (3, 16, False)],
+                         ids=["shared-draw", "recency", "block4", "block16"])
+def test_policy_variants(policy, block, fused):
+    """The controls the paper contrasts with the method, run by the same kernels: survivors bit-exact."""
+    run = Runner(L=2, H=16, KVH=4, prompt_lens=[30, 0, 77], K=96, r=32, eseed=11, dseed=6, fused=fused,
+                 policy=policy, block=block)
+    for step in range(330):
+        fired = run.step(check_attn_layers=(1,) if step % 60 == 0 else ())
+        if any(fired.values()):
+            run.check_state()
+    run.close()
+
+
 def test_degenerate_budgets():
     # K = 0: only the recent buffer survives; r = 1 evicts at every step once the cache exceeds K + 1
     for (K, r), fused in [((0, 8), False), ((5, 1), False), ((3, 2), False), ((0, 8), True), ((5, 1), True),
