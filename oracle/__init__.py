@@ -14,7 +14,9 @@ Paper sections followed (Random Attention, arXiv 2609.03430):
   * Appendix F "Engine details" -- every r=64 steps once the cache exceeds
     K+r; keep-sets sorted chronologically; GQA query groups share their KV
     head's keep-set; keys stored post-RoPE (so attention applies no rotation);
-  * section 2 "Notation" -- o_t = sum_i softmax_i(q.k_i/sqrt(d)) v_i.
+  * section 2 "Notation" -- o_t = sum_i softmax_i(q.k_i/sqrt(d)) v_i;
+  * section 2 "Baselines as choices of s" -- the SnapKV window score of the
+    scored comparator (window attention, max-pooled, top-K, prompt pinned).
 
 Budget convention: ``K`` here counts retained *generated* tokens; the paper's
 budget includes the prompt (K_paper = prompt_len + K), see
@@ -76,6 +78,16 @@ def _load():
                                               ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, i32p]
         lib.ora_evict_head_policy.restype = ctypes.c_int
         lib.ora_attend.restype = None
+        lib.ora_window_scores.argtypes = [u16p, i32p, ctypes.c_int, ctypes.c_int, u16p, i32p, ctypes.c_int,
+                                          ctypes.c_int, ctypes.c_double, f64p]
+        lib.ora_window_scores.restype = None
+        lib.ora_max_pool.argtypes = [f64p, ctypes.c_int, ctypes.c_int, f64p]
+        lib.ora_max_pool.restype = None
+        lib.ora_select_top.argtypes = [f64p, ctypes.c_int, ctypes.c_int, i32p]
+        lib.ora_select_top.restype = ctypes.c_int
+        lib.ora_evict_head_scored.argtypes = [i32p, ctypes.POINTER(ctypes.c_int), ctypes.c_int, ctypes.c_int,
+                                              ctypes.c_int, f64p, ctypes.c_int, i32p]
+        lib.ora_evict_head_scored.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -133,7 +145,8 @@ def evict_head(gen: np.ndarray, g: int, K: int, r: int, seed: int, layer: int, h
     return buf[: c.value].copy(), ev[:m].copy()
 
 
-POLICY_RANDOM, POLICY_SHARED, POLICY_RECENCY, POLICY_BLOCK = 0, 1, 2, 3
+POLICY_RANDOM, POLICY_SHARED, POLICY_RECENCY, POLICY_BLOCK, POLICY_SNAPKV = 0, 1, 2, 3, 4
+SNAPKV_POOL_RADIUS = 3  # max-pool width 7: the paper gives no width, this is the library's stated choice
 
 
 def evict_head_policy(gen, g, K, r, seed, layer, seq, kv_heads, h, policy, block=1):
@@ -162,6 +175,57 @@ def attend(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float = 0.0) -> n
     _load().ora_attend(_ptr(q, ctypes.c_uint16), _ptr(k, ctypes.c_uint16), _ptr(v, ctypes.c_uint16),
                        n, G, d, float(scale), _ptr(out, ctypes.c_double))
     return out
+
+
+def window_scores(q: np.ndarray, q_pos, k: np.ndarray, k_pos, scale: float = 0.0) -> np.ndarray:
+    """SnapKV window score of every key (section 2): attention from the window queries
+    q [n_q][G][d] (bf16 bits) at positions q_pos, summed over queries and heads, each
+    query seeing the keys k [n_k][d] whose positions k_pos are not after its own."""
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    qp = np.ascontiguousarray(q_pos, dtype=np.int32)
+    kp = np.ascontiguousarray(k_pos, dtype=np.int32)
+    n_q, G, d = q.shape
+    n_k = k.shape[0]
+    assert k.shape == (n_k, d) and qp.shape == (n_q,) and kp.shape == (n_k,)
+    out = np.zeros(max(n_k, 1), dtype=np.float64)
+    _load().ora_window_scores(_ptr(q, ctypes.c_uint16), _ptr(qp, ctypes.c_int32), n_q, G, _ptr(k, ctypes.c_uint16),
+                              _ptr(kp, ctypes.c_int32), n_k, d, float(scale), _ptr(out, ctypes.c_double))
+    return out[:n_k].copy()
+
+
+def max_pool(s, radius: int = SNAPKV_POOL_RADIUS) -> np.ndarray:
+    """Max over the window |j - i| <= radius, clipped to the ends."""
+    s = np.ascontiguousarray(s, dtype=np.float64)
+    out = np.zeros(max(s.size, 1), dtype=np.float64)
+    _load().ora_max_pool(_ptr(s, ctypes.c_double), int(s.size), int(radius), _ptr(out, ctypes.c_double))
+    return out[: s.size].copy()
+
+
+def select_top(s, K: int) -> np.ndarray:
+    """Indices of the K largest scores (ties: lower index first), ascending."""
+    s = np.ascontiguousarray(s, dtype=np.float64)
+    out = np.zeros(max(K, 1), dtype=np.int32)
+    if _load().ora_select_top(_ptr(s, ctypes.c_double), int(s.size), int(K), _ptr(out, ctypes.c_int32)) != 0:
+        raise ValueError("ora_select_top: bad arguments")
+    return out[:K].copy()
+
+
+def evict_head_scored(gen, g, K, r, raw_scores, radius=SNAPKV_POOL_RADIUS):
+    """One scored eviction round: raw_scores[j] ranks candidate j (j < c - r) after max-pooling."""
+    buf = np.ascontiguousarray(gen, dtype=np.int32).copy()
+    raw = np.ascontiguousarray(raw_scores, dtype=np.float64)
+    c = ctypes.c_int(int(buf.size))
+    ev = np.zeros(max(int(buf.size), 1), dtype=np.int32)
+    if not should_evict(g, int(buf.size), K, r):
+        return buf, ev[:0]
+    if raw.size != buf.size - r:
+        raise ValueError(f"need {buf.size - r} candidate scores, got {raw.size}")
+    m = _load().ora_evict_head_scored(_ptr(buf, ctypes.c_int32), ctypes.byref(c), g, K, r,
+                                      _ptr(raw, ctypes.c_double), int(radius), _ptr(ev, ctypes.c_int32))
+    if m < 0:
+        raise RuntimeError("ora_evict_head_scored failed")
+    return buf[: c.value].copy(), ev[:m].copy()
 
 
 def paper_budget_to_generated(K_paper: int, prompt_len: int) -> int:
@@ -223,8 +287,11 @@ class OracleCache:
         self.g[seq, layer] += 1
         return pos
 
-    def evict(self, seq, layer):
-        """Returns {kv_head: evicted ordinals} for the tracked heads if the trigger fired."""
+    def evict(self, seq, layer, scorer=None):
+        """Returns {kv_head: evicted ordinals} for the tracked heads if the trigger fired.
+
+        Under the scored policy, scorer(seq, layer, kv_head, cached_positions) returns the raw
+        window score of each candidate (all cached generated slots but the newest r)."""
         g = int(self.g[seq, layer])
         fired = {}
         for h in range(self.KVH):
@@ -236,6 +303,8 @@ class OracleCache:
                 continue
             if self.policy == POLICY_RANDOM:
                 new, ev = evict_head(cur, g, self.K, self.r, self.seed, layer, seq * self.KVH + h)
+            elif self.policy == POLICY_SNAPKV:
+                new, ev = evict_head_scored(cur, g, self.K, self.r, scorer(seq, layer, h, cur))
             else:
                 new, ev = evict_head_policy(cur, g, self.K, self.r, self.seed, layer, seq, self.KVH, h,
                                             self.policy, self.block)

@@ -24,11 +24,16 @@
  *   - Decode attention o = sum_i softmax_i(q.k_i / sqrt(d)) v_i in fp64
  *     (section 2 "Notation"), grouped-query: a KV head's keep-set serves
  *     every query head of its group (Appendix F).
+ *   - The scored comparator (section 2, "Baselines as choices of s"): the
+ *     SnapKV score -- attention received from the last w queries, summed
+ *     over the query heads of the group, max-pooled over neighbouring
+ *     positions -- and a top-K by that score, with the prompt pinned.
  *
  * Parity status: every function here is pinned by the "not gpu" tests
  * (Philox against an independent Philox implementation, selection by brute
  * force and by the paper's closed-form survival law, attention by closed
- * forms and an independent library softmax).
+ * forms and an independent library softmax, window scores by closed forms
+ * and a brute-force softmax, pooling and top-K by hand-worked cases).
  */
 #include <math.h>
 #include <stdint.h>
@@ -303,4 +308,136 @@ void ora_attend(const uint16_t* q, const uint16_t* k, const uint16_t* v, int n, 
         for (int c = 0; c < d; ++c) o[c] /= den;
     }
     free(s);
+}
+
+/* ------------------------------------------------------------------------- */
+/* Scored comparator (section 2, "Baselines as choices of s"): the SnapKV     */
+/* score, the attention that the last w queries give each cached position,    */
+/* max-pooled over neighbouring positions, then the K best kept.  The prompt  */
+/* stays pinned and the buffer unscored, as in Random Attention, so the two   */
+/* policies differ only in how candidates are ranked.                         */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * score[i] = sum over window queries u and query heads g of alpha_i(u, g), with
+ *   alpha_i(u, g) = exp(scale * q_ug . k_i) / sum_{i': pos_i' <= qpos_u} exp(scale * q_ug . k_i')
+ * when pos_i <= qpos_u (a decoding query sees no later position) and 0
+ * otherwise.  q [n_q][G][d] and k [n_k][d] are bf16 bit patterns; q_pos [n_q]
+ * and k_pos [n_k] are token positions; score [n_k] is fp64.  scale <= 0 means
+ * 1/sqrt(d).  Every key, the prompt's included, takes part in the softmax;
+ * the caller reads the entries of the candidates.
+ */
+void ora_window_scores(const uint16_t* q, const int32_t* q_pos, int n_q, int G, const uint16_t* k,
+                       const int32_t* k_pos, int n_k, int d, double scale, double* score)
+{
+    if (scale <= 0.0) scale = 1.0 / sqrt((double)d);
+    for (int i = 0; i < n_k; ++i) score[i] = 0.0;
+    double* logit = (double*)malloc(sizeof(double) * (size_t)(n_k > 0 ? n_k : 1));
+    if (!logit) return;
+    for (int u = 0; u < n_q; ++u) {
+        for (int g = 0; g < G; ++g) {
+            const uint16_t* qr = q + ((size_t)u * G + g) * d;
+            double mx = -INFINITY;
+            for (int i = 0; i < n_k; ++i) {
+                if (k_pos[i] > q_pos[u]) continue;
+                double dot = 0.0;
+                for (int c = 0; c < d; ++c)
+                    dot += ora_bf16_to_double(qr[c]) * ora_bf16_to_double(k[(size_t)i * d + c]);
+                logit[i] = scale * dot;
+                if (logit[i] > mx) mx = logit[i];
+            }
+            if (mx == -INFINITY) continue; /* the query sees no key */
+            double den = 0.0;
+            for (int i = 0; i < n_k; ++i)
+                if (k_pos[i] <= q_pos[u]) den += exp(logit[i] - mx);
+            for (int i = 0; i < n_k; ++i)
+                if (k_pos[i] <= q_pos[u]) score[i] += exp(logit[i] - mx) / den;
+        }
+    }
+    free(logit);
+}
+
+/* out[i] = max of s[j] over |j - i| <= radius, 0 <= j < n (a window clipped at the ends). */
+void ora_max_pool(const double* s, int n, int radius, double* out)
+{
+    for (int i = 0; i < n; ++i) {
+        double m = s[i];
+        for (int j = i - radius; j <= i + radius; ++j)
+            if (j >= 0 && j < n && s[j] > m) m = s[j];
+        out[i] = m;
+    }
+}
+
+typedef struct {
+    double s;
+    int32_t i;
+} ora_scored;
+
+static int ora_cmp_scored(const void* a, const void* b)
+{
+    const ora_scored* x = (const ora_scored*)a;
+    const ora_scored* y = (const ora_scored*)b;
+    if (x->s != y->s) return x->s > y->s ? -1 : 1; /* larger score first */
+    return (x->i > y->i) - (x->i < y->i);           /* then the earlier position */
+}
+
+/*
+ * Top-K by score: the K largest of s[0..n), equal scores going to the lower
+ * index.  keep_out receives the K indices in ascending (chronological) order.
+ * Returns 0, or -1 on bad arguments.
+ */
+int ora_select_top(const double* s, int n, int K, int32_t* keep_out)
+{
+    if (n < 0 || K < 0 || K > n) return -1;
+    ora_scored* a = (ora_scored*)malloc(sizeof(ora_scored) * (size_t)(n > 0 ? n : 1));
+    if (!a) return -1;
+    for (int i = 0; i < n; ++i) {
+        a[i].s = s[i];
+        a[i].i = i;
+    }
+    qsort(a, (size_t)n, sizeof(ora_scored), ora_cmp_scored);
+    for (int i = 0; i < K; ++i) keep_out[i] = a[i].i;
+    free(a);
+    qsort(keep_out, (size_t)K, sizeof(int32_t), ora_cmp_i32);
+    return 0;
+}
+
+/*
+ * One scored eviction round of one head, the same cadence and compaction as
+ * ora_evict_head but ranked by score: raw[0..n) holds the window score of each
+ * candidate (n = c - r), pooled over +-radius neighbours; the K best survive.
+ * Returns the number evicted (0 when the trigger does not fire), -1 on error.
+ */
+int ora_evict_head_scored(int32_t* gen, int* c, int g, int K, int r, const double* raw, int radius,
+                          int32_t* evicted_out)
+{
+    const int cc = *c;
+    if (!ora_should_evict(g, cc, K, r)) return 0;
+    const int n = cc - r;
+    double* pooled = (double*)malloc(sizeof(double) * (size_t)n);
+    int32_t* keep = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
+    int32_t* next = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K + r));
+    if (!pooled || !keep || !next) {
+        free(pooled); free(keep); free(next);
+        return -1;
+    }
+    ora_max_pool(raw, n, radius, pooled);
+    if (ora_select_top(pooled, n, K, keep) != 0) {
+        free(pooled); free(keep); free(next);
+        return -1;
+    }
+    int m = 0, ki = 0;
+    for (int j = 0; j < n; ++j) {
+        if (ki < K && keep[ki] == j) {
+            next[ki++] = gen[j];
+        } else {
+            if (evicted_out) evicted_out[m] = j;
+            ++m;
+        }
+    }
+    for (int i = 0; i < r; ++i) next[K + i] = gen[n + i];
+    memcpy(gen, next, sizeof(int32_t) * (size_t)(K + r));
+    *c = K + r;
+    free(pooled); free(keep); free(next);
+    return m;
 }
