@@ -69,7 +69,9 @@ enum ra_kernel_kind {
     RA_KERNEL_SELECT = 1,
     RA_KERNEL_COMPACT = 2,
     RA_KERNEL_ATTN = 3,
-    RA_KERNEL_KINDS = 4
+    RA_KERNEL_SCORE_STATS = 4, /* scored comparator, pass 1: softmax statistics of the window queries */
+    RA_KERNEL_SCORE_SUM = 5,   /* scored comparator, pass 2: attention summed per candidate */
+    RA_KERNEL_KINDS = 6
 };
 
 /*
@@ -125,13 +127,47 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
  *                      prompt plus a contiguous recent window (section 4.1, 5);
  *   RA_POLICY_BLOCK    one draw per block of `block` consecutive positions, so
  *                      the history is kept in contiguous blocks (section 5).
+ *   RA_POLICY_SNAPKV   the scored comparator: a candidate's score is the
+ *                      attention it receives from the window of the last r
+ *                      decode queries, summed over the query heads of its KV
+ *                      group and max-pooled over the 3 candidates on either
+ *                      side (SnapKV as section 2 writes it, with the prompt
+ *                      pinned and the buffer unscored as for the method); the
+ *                      K best survive, ties to the earlier position.  Each
+ *                      window query attends with scale 1/sqrt(head_dim) to the
+ *                      keys at positions up to its own.
  * Takes effect from the next eviction; `block` >= 1 is used by RA_POLICY_BLOCK.
+ *
+ * The scored policy needs a per-layer window of recent queries, which the
+ * attention calls record: set it BEFORE ra_device_bytes / ra_bind (the arena
+ * then also holds the window, the scores and their scratch, and the context
+ * keeps recording the window under every policy); on a context bound without
+ * them it fails with RA_ERR_STATE.  It requires r * G <= 512.
  */
 #define RA_POLICY_RANDOM 0
 #define RA_POLICY_SHARED 1
 #define RA_POLICY_RECENCY 2
 #define RA_POLICY_BLOCK 3
+#define RA_POLICY_SNAPKV 4
 int ra_set_policy(ra_ctx* ctx, int policy, int block);
+
+/*
+ * Scored policy, warm start: load the query window of layer `layer` from q,
+ * device [batch][q_heads][r][head_dim] bf16, where row u of (b, qh) is the
+ * query of decode step g_b - r + 1 + u (g_b = the sequence's generated count,
+ * so row r - 1 is the latest step).  Steps before the first are never read.
+ * RA_ERR_STATE unless the context was bound with the scored policy's buffers.
+ */
+int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, void* stream);
+
+/*
+ * Debug (scored policy): copy the raw window scores (before pooling) that the
+ * latest scored eviction of (layer, seq, kv_head) computed, one fp32 per
+ * candidate in slot order, to host (synchronises).  *n = the candidate count
+ * of that eviction (0 if none happened yet); capacity must be >= *n.
+ */
+int ra_get_scores(ra_ctx* ctx, int layer, int seq, int kv_head, float* host_scores, int capacity, int* n,
+                  void* stream);
 
 /* Mark sequence `seq` active (1) or finished (0); finished ones are skipped by every call. */
 int ra_set_active(ra_ctx* ctx, int seq, int active);

@@ -25,8 +25,8 @@ RA_ERR_CUDA = -4
 RA_ERR_DEVICE_TIMEOUT = -5
 RA_ERR_UNSUPPORTED = -6
 RA_MAX_BATCH = 512
-RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN = range(4)
-KERNEL_NAMES = ["append", "select", "compact", "attn"]
+RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN, RA_KERNEL_SCORE_STATS, RA_KERNEL_SCORE_SUM = range(6)
+KERNEL_NAMES = ["append", "select", "compact", "attn", "score_stats", "score_sum"]
 
 # Exported C symbols and their ctypes signatures (kept in the order of include/ra.h).
 _vp, _i, _u64, _sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint64, ctypes.c_size_t
@@ -42,6 +42,8 @@ SIGNATURES = {
     "ra_prefill": (_i, [_vp, _i, _vp, _vp, _i, _vp]),
     "ra_restore": (_i, [_vp, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp]),
     "ra_set_policy": (_i, [_vp, _i, _i]),
+    "ra_restore_queries": (_i, [_vp, _i, _vp, _vp]),
+    "ra_get_scores": (_i, [_vp, _i, _i, _i, ctypes.POINTER(ctypes.c_float), _i, _ip, _vp]),
     "ra_set_active": (_i, [_vp, _i, _i]),
     "ra_append_kv": (_i, [_vp, _i, _vp, _vp, _vp]),
     "ra_evict": (_i, [_vp, _i, _ip, _vp]),
@@ -135,11 +137,25 @@ def ra_restore(ctx, layer, g_list, c_list, pos_ptr, k_ptr, v_ptr, row_stride, st
     return _check(lib().ra_restore(ctx, layer, g, c, pos_ptr, k_ptr, v_ptr, row_stride, _stream_ptr(stream)), ctx)
 
 
-RA_POLICY_RANDOM, RA_POLICY_SHARED, RA_POLICY_RECENCY, RA_POLICY_BLOCK = 0, 1, 2, 3
+RA_POLICY_RANDOM, RA_POLICY_SHARED, RA_POLICY_RECENCY, RA_POLICY_BLOCK, RA_POLICY_SNAPKV = 0, 1, 2, 3, 4
 
 
 def ra_set_policy(ctx, policy, block=1):
     return _check(lib().ra_set_policy(ctx, int(policy), int(block)), ctx)
+
+
+def ra_restore_queries(ctx, layer, q_ptr, stream=None):
+    return _check(lib().ra_restore_queries(ctx, layer, q_ptr, _stream_ptr(stream)), ctx)
+
+
+def ra_get_scores(ctx, layer, seq, kv_head, capacity, stream=None):
+    import numpy as np
+
+    buf = np.zeros(max(capacity, 1), dtype=np.float32)
+    n = ctypes.c_int(0)
+    _check(lib().ra_get_scores(ctx, layer, seq, kv_head, buf.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), capacity,
+                               ctypes.byref(n), _stream_ptr(stream)), ctx)
+    return buf[: n.value].copy()
 
 
 def ra_set_active(ctx, seq, active):
@@ -230,7 +246,8 @@ def ra_destroy(ctx):
 class RandomAttentionCache:
     """Owns a context and its torch-allocated device arena (uint8 CUDA tensor)."""
 
-    def __init__(self, layers, q_heads, kv_heads, head_dim, prompt_lens, K, r=64, seed=0, device=None, stream=None):
+    def __init__(self, layers, q_heads, kv_heads, head_dim, prompt_lens, K, r=64, seed=0, device=None, stream=None,
+                 policy=RA_POLICY_RANDOM, block=1):
         import torch
 
         if isinstance(prompt_lens, int):
@@ -239,6 +256,8 @@ class RandomAttentionCache:
         self.L, self.H, self.KVH, self.D = layers, q_heads, kv_heads, head_dim
         self.B, self.K, self.r, self.seed = len(self.prompt_lens), K, r, seed
         self.ctx = ra_create_batched(layers, q_heads, kv_heads, head_dim, self.prompt_lens, K, r, seed)
+        if policy != RA_POLICY_RANDOM:  # before sizing: the scored policy adds buffers to the arena
+            ra_set_policy(self.ctx, policy, block)
         self.nbytes = ra_device_bytes(self.ctx)
         dev = torch.device("cuda") if device is None else torch.device(device)
         self.arena = torch.empty(self.nbytes + 256, dtype=torch.uint8, device=dev)

@@ -14,7 +14,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libra.so")
-SOURCES = ["ra_api.cu", "ra_evict.cu", "ra_attn.cu"]
+SOURCES = ["ra_api.cu", "ra_evict.cu", "ra_attn.cu", "ra_score.cu"]
 HEADERS = ["ra_internal.h", "ra_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include"), "-I" + CSRC]

@@ -59,6 +59,10 @@ struct ra_ctx {
     // arena layout (byte offsets)
     size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_poff, off_plan, off_partial, off_arrive, off_ticket,
         off_err, bytes;
+    // scored policy: query window, scores and pass-1 statistics after the base arena
+    bool scoring = false;
+    size_t base_bytes = 0, off_qring = 0, off_scores = 0, off_stats = 0;
+    int stats_chunks = 0;
     // binding
     bool bound = false;
     int device = -1;
@@ -66,11 +70,13 @@ struct ra_ctx {
     uint8_t* arena = nullptr;
     DevLayout lay{};
     CUtensorMap tmap_k{}, tmap_v{};
+    CUtensorMap tmap_ks{};  // kpool in kScoreTile-row boxes (scoring kernels)
     // host mirror
     std::vector<int32_t> g, c, nev;  // [L][B]
     std::vector<uint8_t> active;     // [B]
     int policy = RA_POLICY_RANDOM;   // candidate scoring (ra_set_policy)
     int block = 1;
+    std::vector<int32_t> score_n;    // [L][B] candidates of the latest scored round
     // profiling
     bool prof = false;
     std::vector<ProfRec> pending;
@@ -262,6 +268,98 @@ unsigned long long tickets_taken(const AttnParams& p)
     return (unsigned long long)(stolen + std::min(p.nchunks, p.nwarps));
 }
 
+// Arena size with (or without) the scored policy's buffers after the base layout.
+void layout_scoring(ra_ctx* ctx)
+{
+    if (!ctx->scoring) {
+        ctx->bytes = ctx->base_bytes;
+        return;
+    }
+    const size_t heads = (size_t)ctx->B * ctx->KVH;
+    const size_t M = (size_t)ctx->r * ctx->G;
+    size_t o = ctx->base_bytes;
+    ctx->off_qring = o;
+    o = align_up(o + (size_t)ctx->L * heads * M * kRowBytes, kAlign);
+    ctx->off_scores = o;
+    o = align_up(o + (size_t)ctx->L * heads * ctx->Cmax * sizeof(float), kAlign);
+    ctx->off_stats = o;
+    o = align_up(o + heads * ctx->stats_chunks * M * 2 * sizeof(float), kAlign);
+    ctx->bytes = o;
+}
+
+// Launch shape of the two scoring passes of one eviction round, from the host mirror:
+// about two waves of CTAs (one per SM when the window needs more than half the shared
+// memory), each taking a run of consecutive tiles of one head.
+void plan_scoring(ra_ctx* ctx, EvictParams* p, double* bytes1, double* bytes2)
+{
+    const int r = ctx->r, M = r * ctx->G;
+    const int per_sm = score_row_tiles_per_warp(M) <= 2 ? 2 : 1;
+    long long w1 = 0, w2 = 0;
+    int max1 = 1, max2 = 1;
+    double rows1 = 0, rows2 = 0;
+    for (int i = 0; i < p->n_trig; ++i) {
+        const int b = p->trig[i], N = p->trig_n[i], lp = ctx->lp[b];
+        const int t1 = (lp + kScoreTile - 1) / kScoreTile + (N + r - 1 + kScoreTile - 1) / kScoreTile;
+        const int t2 = (N + kScoreTile - 1) / kScoreTile;
+        w1 += (long long)ctx->KVH * t1;
+        w2 += (long long)ctx->KVH * t2;
+        max1 = std::max(max1, t1);
+        max2 = std::max(max2, t2);
+        rows1 += (double)ctx->KVH * (lp + N + r - 1);
+        rows2 += (double)ctx->KVH * N;
+        ctx->score_n[(size_t)p->layer * ctx->B + b] = N;
+    }
+    const long long target = (long long)ctx->sms * per_sm;
+    long long ch1 = std::max<long long>((w1 + target - 1) / target, (max1 + ctx->stats_chunks - 1) / ctx->stats_chunks);
+    long long ch2 = (w2 + target - 1) / target;
+    ch1 = std::max<long long>(ch1, 1);
+    ch2 = std::max<long long>(ch2, 1);
+    p->ch1 = (int)ch1;
+    p->ch2 = (int)ch2;
+    p->nch1 = (int)((max1 + ch1 - 1) / ch1);
+    p->nch2 = (int)((max2 + ch2 - 1) / ch2);
+    p->qk_scale_log2 = 1.4426950408889634f / sqrtf((float)kHeadDim);
+    // key rows read once and the window once per head; pass 2 also writes one score per candidate
+    const double win = (double)p->n_trig * ctx->KVH * M * kRowBytes;
+    *bytes1 = rows1 * kRowBytes + win;
+    *bytes2 = rows2 * (kRowBytes + 4) + win;
+}
+
+// One eviction round of the triggered sequences in p: [score passes,] select, compact.
+int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s)
+{
+    cudaError_t e;
+    if (p.policy == RA_POLICY_SNAPKV) {
+        double b1 = 0, b2 = 0;
+        plan_scoring(ctx, &p, &b1, &b2);
+        {
+            ProfScope ps(ctx, RA_KERNEL_SCORE_STATS, b1, s);
+            e = launch_score(p, 1, &ctx->tmap_ks, s);
+            ps.done();
+        }
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "score pass 1 launch");
+        {
+            ProfScope ps(ctx, RA_KERNEL_SCORE_SUM, b2, s);
+            e = launch_score(p, 2, &ctx->tmap_ks, s);
+            ps.done();
+        }
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "score pass 2 launch");
+    }
+    {
+        ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
+        e = launch_select(p, s);
+        ps.done();
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
+    {
+        ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
+        e = launch_compact(p, s);
+        ps.done();
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
+    return RA_OK;
+}
+
 void set_scale(AttnParams* p, float scale)
 {
     const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)kHeadDim);
@@ -343,11 +441,19 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);
     ctx->off_ticket = take(sizeof(unsigned long long));
     ctx->off_err = take(256);
-    ctx->bytes = o;
+    ctx->base_bytes = o;
+    int maxlp = 0;
+    for (int b = 0; b < batch; ++b) maxlp = std::max(maxlp, (int)prompt_lens[b]);
+    // pass-1 chunks per head: at most one per tile of the longest head, capped (the host
+    // then takes chunks of several tiles)
+    const int tiles1 = (maxlp + kScoreTile - 1) / kScoreTile + (ctx->Cmax + kScoreTile - 1) / kScoreTile;
+    ctx->stats_chunks = std::min(tiles1, 64);
+    layout_scoring(ctx);
     ctx->g.assign((size_t)layers * batch, 0);
     ctx->c.assign((size_t)layers * batch, 0);
     ctx->nev.assign((size_t)layers * batch, 0);
     ctx->active.assign(batch, 1);
+    ctx->score_n.assign((size_t)layers * batch, 0);
     *out = ctx;
     return RA_OK;
 }
@@ -395,6 +501,10 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.arrive = (int32_t*)(a + ctx->off_arrive);
     Ly.ticket = (unsigned long long*)(a + ctx->off_ticket);
     Ly.err = (int32_t*)(a + ctx->off_err);
+    Ly.qring = ctx->scoring ? (uint16_t*)(a + ctx->off_qring) : nullptr;
+    Ly.scores = ctx->scoring ? (float*)(a + ctx->off_scores) : nullptr;
+    Ly.stats = ctx->scoring ? (float*)(a + ctx->off_stats) : nullptr;
+    Ly.stats_chunks = ctx->stats_chunks;
     Ly.prompt_rows_per_layer = ctx->prompt_rows_per_layer;
     Ly.gen_row0 = ctx->prompt_rows_per_layer * ctx->L;
     Ly.L = ctx->L;
@@ -424,6 +534,9 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
         return cuda_fail(ctx, e, "table initialisation");
     // rows that were never written (past a head's cached slots) then read as zeros, never as stale NaNs
     if ((e = cudaMemsetAsync(a, 0, ctx->off_pos, s)) != cudaSuccess) return cuda_fail(ctx, e, "cache clear");
+    // an empty query window and no scores yet
+    if (ctx->scoring && (e = cudaMemsetAsync(a + ctx->off_qring, 0, ctx->off_stats - ctx->off_qring, s)) != cudaSuccess)
+        return cuda_fail(ctx, e, "query window clear");
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(ctx, e, "table initialisation sync");
 
     const int tile = attn_tile_rows(ctx->G);
@@ -431,6 +544,10 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     if ((rc = make_tmap(ctx, &ctx->tmap_k, Ly.kpool, tile)) != RA_OK) return rc;
     if ((rc = make_tmap(ctx, &ctx->tmap_v, Ly.vpool, tile)) != RA_OK) return rc;
     if ((e = attn_prepare(ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
+    if (ctx->scoring) {
+        if ((rc = make_tmap(ctx, &ctx->tmap_ks, Ly.kpool, kScoreTile)) != RA_OK) return rc;
+        if ((e = score_prepare()) != cudaSuccess) return cuda_fail(ctx, e, "score kernel attributes");
+    }
 
     ctx->ticket_base = 0;
     ctx->arena = a;
@@ -440,6 +557,7 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     std::fill(ctx->g.begin(), ctx->g.end(), 0);
     std::fill(ctx->c.begin(), ctx->c.end(), 0);
     std::fill(ctx->nev.begin(), ctx->nev.end(), 0);
+    std::fill(ctx->score_n.begin(), ctx->score_n.end(), 0);
     return RA_OK;
 }
 
@@ -500,9 +618,18 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
 int ra_set_policy(ra_ctx* ctx, int policy, int block)
 {
     if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
-    if (policy < RA_POLICY_RANDOM || policy > RA_POLICY_BLOCK)
+    if (policy < RA_POLICY_RANDOM || policy > RA_POLICY_SNAPKV)
         return fail(ctx, RA_ERR_INVALID_ARG, "unknown policy %d", policy);
     if (policy == RA_POLICY_BLOCK && block < 1) return fail(ctx, RA_ERR_INVALID_ARG, "block must be >= 1");
+    if (policy == RA_POLICY_SNAPKV && !ctx->scoring) {
+        if (ctx->bound)
+            return fail(ctx, RA_ERR_STATE, "the scored policy must be set before ra_device_bytes / ra_bind");
+        if (ctx->r * ctx->G > kScoreMaxRows)
+            return fail(ctx, RA_ERR_UNSUPPORTED, "scored policy needs r * G <= %d (have %d)", kScoreMaxRows,
+                        ctx->r * ctx->G);
+        ctx->scoring = true;
+        layout_scoring(ctx);
+    }
     ctx->policy = policy;
     ctx->block = policy == RA_POLICY_BLOCK ? block : 1;
     return RA_OK;
@@ -514,6 +641,17 @@ int ra_set_active(ra_ctx* ctx, int seq, int active)
     if (seq < 0 || seq >= ctx->B) return fail(ctx, RA_ERR_INVALID_ARG, "seq %d out of range", seq);
     ctx->active[seq] = active ? 1 : 0;
     return RA_OK;
+}
+
+int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (!ctx->scoring) return fail(ctx, RA_ERR_STATE, "context bound without the scored policy's query window");
+    if (!q || !aligned16(q)) return fail(ctx, RA_ERR_INVALID_ARG, "q must be non-NULL and 16-byte aligned");
+    cudaError_t e = launch_restore_queries(ctx->lay, layer, q, ctx->g.data() + (size_t)layer * ctx->B, (cudaStream_t)stream);
+    return e == cudaSuccess ? RA_OK : cuda_fail(ctx, e, "query window restore launch");
 }
 
 int ra_append_kv(ra_ctx* ctx, int layer, const uint16_t* k_new, const uint16_t* v_new, void* stream)
@@ -583,20 +721,7 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
     }
     if (n == 0) return RA_OK;
     p.n_trig = n;
-    cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e;
-    {
-        ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
-        e = launch_select(p, s);
-        ps.done();
-    }
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
-    {
-        ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
-        e = launch_compact(p, s);
-        ps.done();
-    }
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
+    if ((rc = run_eviction(ctx, p, moved, (cudaStream_t)stream)) != RA_OK) return rc;
     for (int i = 0; i < n; ++i) {
         const int b = p.trig[i];
         ctx->c[(size_t)layer * ctx->B + b] = ctx->K + ctx->r;
@@ -622,6 +747,8 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     p.arrive = ctx->lay.arrive;
     p.ticket = ctx->lay.ticket;
     p.ticket_base = ctx->ticket_base;
+    p.qring = ctx->lay.qring;
+    p.ring_off = -1;  // the step's token is already appended: its query is step g
     int n_active = 0;
     int ctas = 0;
     double rows = 0;
@@ -675,18 +802,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     }
     if (n > 0) {
         ep.n_trig = n;
-        {
-            ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
-            e = launch_select(ep, s);
-            ps.done();
-        }
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
-        {
-            ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
-            e = launch_compact(ep, s);
-            ps.done();
-        }
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
+        if ((rc = run_eviction(ctx, ep, moved, s)) != RA_OK) return rc;
         for (int i = 0; i < n; ++i) {
             const int b = ep.trig[i];
             ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written
@@ -705,6 +821,8 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     p.arrive = ctx->lay.arrive;
     p.ticket = ctx->lay.ticket;
     p.ticket_base = ctx->ticket_base;
+    p.qring = ctx->lay.qring;
+    p.ring_off = 0;  // the query of step g + 1
     int n_active = 0, ctas = 0;
     double rows = 0;
     if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
@@ -826,6 +944,26 @@ int ra_get_kv(ra_ctx* ctx, int layer, int seq, int kv_head, uint16_t* host_k, ui
     return RA_OK;
 }
 
+int ra_get_scores(ra_ctx* ctx, int layer, int seq, int kv_head, float* host_scores, int capacity, int* n,
+                  void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
+    if (seq < 0 || seq >= ctx->B || kv_head < 0 || kv_head >= ctx->KVH || !n)
+        return fail(ctx, RA_ERR_INVALID_ARG, "seq/kv_head out of range or n NULL");
+    if (!ctx->scoring) return fail(ctx, RA_ERR_STATE, "context bound without the scored policy's buffers");
+    const int N = ctx->score_n[(size_t)layer * ctx->B + seq];
+    *n = N;
+    if (capacity < N || (N > 0 && !host_scores)) return fail(ctx, RA_ERR_INVALID_ARG, "capacity %d < %d", capacity, N);
+    cudaError_t e;
+    if ((e = cudaStreamSynchronize((cudaStream_t)stream)) != cudaSuccess) return cuda_fail(ctx, e, "stream sync");
+    const float* src = ctx->lay.scores + (((size_t)layer * ctx->B + seq) * ctx->KVH + kv_head) * ctx->Cmax;
+    if (N > 0 && (e = cudaMemcpy(host_scores, src, (size_t)N * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_fail(ctx, e, "scores read");
+    return RA_OK;
+}
+
 int ra_check_device(ra_ctx* ctx, void* stream)
 {
     int rc;
@@ -937,6 +1075,8 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     p.layer = layer;
     p.q = q;
     p.out = out;
+    p.qring = ctx->lay.qring;
+    p.ring_off = -1;
     int n_active = 0, ctas = 0;
     double rows = 0;
     if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;

@@ -24,6 +24,9 @@
 // advance monotonically through the tile order -- and the last warp to finish
 // a piece of that head (an arrival counter per head) merges all of them.
 //
+// With the scored comparator's buffers bound, the warp that consumes a head's
+// first tile also copies the head's G query rows into the query window.
+//
 // Per-warp compute: the contraction of the G query rows with a tile of cache
 // rows runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
 // S = Q K^T takes the query heads as the 16 M rows (G <= 8 used, the rest
@@ -90,7 +93,8 @@ struct Cfg {
     static_assert(SMEM <= 232448, "fits the 227 KB opt-in shared memory of sm_100+");
 };
 
-constexpr int kFirst = 1, kLast = 2, kNewTok = 4;
+// Tile header flags; the chunk index sits above them (<< kFlagBits).
+constexpr int kFirst = 1, kLast = 2, kNewTok = 4, kHead0 = 8, kFlagBits = 4;
 
 // Producer-side walk over the warp's chunks (chunks and cursors count tiles).
 struct TileIter {
@@ -170,7 +174,7 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int wa
 {
     if (it.f >= it.end && !iter_next_chunk(it, p, warp_id, lane)) return false;
     const int T = p.tile;
-    d.flags = it.piece_start ? kFirst : 0;
+    d.flags = (it.piece_start ? kFirst : 0) | (it.k == 0 ? kHead0 : 0);
     if (it.k < it.tp) {
         d.row = it.prow + (long long)it.k * T;
         d.n = min(T, it.lp - it.k * T);
@@ -360,7 +364,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         const int s = t % C::SPW;
         if (lane == 0) {
             uint8_t* st = wstage + (size_t)s * C::STAGE_BYTES;
-            hdrs[s] = make_int4(d.n, d.flags | (d.chunk << 3), d.hid, (int)d.row);
+            hdrs[s] = make_int4(d.n, d.flags | (d.chunk << kFlagBits), d.hid, (int)d.row);
             const bool first = d.flags & kFirst;
             const bool newtok = d.flags & kNewTok;
             mbar_arrive_expect_tx(&bars[s], 2u * C::KV_BYTES + (first ? (uint32_t)C::Q_BYTES : 0u) +
@@ -415,6 +419,14 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             for (int kk = 0; kk < 8; ++kk) {
                 qa[kk][0] = gq < G ? *reinterpret_cast<const uint32_t*>(Qs + gq * kRowBytes + (16 * kk + 2 * tq) * 2) : 0u;
                 qa[kk][1] = gq < G ? *reinterpret_cast<const uint32_t*>(Qs + gq * kRowBytes + (16 * kk + 8 + 2 * tq) * 2) : 0u;
+            }
+            if ((hd.y & kHead0) && p.qring) {  // the scored policy's window: this step's query rows of the head
+                const int b = hd.z / p.lay.KVH, h = hd.z - b * p.lay.KVH, r = p.lay.r;
+                int slot = (p.seq_g[b] + p.ring_off) % r;
+                if (slot < 0) slot += r;
+                uint4* dst = reinterpret_cast<uint4*>(
+                    p.qring + ((((size_t)p.layer * p.lay.B + b) * p.lay.KVH + h) * r + slot) * (size_t)(G * kHeadDim));
+                for (int i = lane; i < G * 16; i += 32) dst[i] = lds128(Qs + i * 16);
             }
         }
         if (hd.y & kNewTok) {  // fused append: put the new token in row n-1 of the tile and into the cache
@@ -498,7 +510,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
                     for (int nt = 0; nt < 16; ++nt) out[nt * 4 + tq] = pack_bf16x2(O[nt][0] * inv, O[nt][1] * inv);
                 }
             } else {
-                float* rec = p.partial + (size_t)((hd.y >> 3) + hid) * partial_stride(G);
+                float* rec = p.partial + (size_t)((hd.y >> kFlagBits) + hid) * partial_stride(G);
                 if (gq < G) {
 #pragma unroll
                     for (int nt = 0; nt < 16; ++nt)

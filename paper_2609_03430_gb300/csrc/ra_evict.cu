@@ -9,6 +9,8 @@
 //                   protected recency, block-contiguous draws), radix select of
 //                   the K smallest (score, ordinal) -- Eq. 1 -- and a
 //                   ballot-compacted, ascending list of the evicted ordinals.
+//                   Under the scored comparator the score is the max-pooled
+//                   window attention that ra_score.cu computed.
 //   compact_kernel  many CTAs per triggered head: order-preserving move of the
 //                   survivors (kept candidates, then the buffer rows) into
 //                   the head's spare region with coalesced 16-byte copies
@@ -111,6 +113,21 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         for (int j = tid; j < N; j += kSelThreads)
             keys[j] = philox4x32_10_w0((uint32_t)(pos[j] / p.block), (uint32_t)g, (uint32_t)p.layer, (uint32_t)head_id,
                                        k0, k1);
+    } else if (p.policy == RA_POLICY_SNAPKV) {
+        // scored comparator: the window score max-pooled over +-kScorePoolRadius candidates;
+        // larger scores must sort first, so the key is the order-reversed float
+        const float* sc = L.scores + (((size_t)p.layer * L.B + b) * L.KVH + h) * L.Cmax;
+        for (int j = tid; j < N; j += kSelThreads) {
+            float m = __ldcg(sc + j);
+#pragma unroll
+            for (int d = 1; d <= kScorePoolRadius; ++d) {
+                if (j - d >= 0) m = fmaxf(m, __ldcg(sc + j - d));
+                if (j + d < N) m = fmaxf(m, __ldcg(sc + j + d));
+            }
+            const uint32_t u = __float_as_uint(m);
+            const uint32_t asc = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // ascending with the float
+            keys[j] = ~asc;
+        }
     } else {  // random: an independent draw per KV head; shared: one draw for all heads of the sequence
         const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
         for (int j = tid; j < N; j += kSelThreads)
@@ -326,6 +343,45 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(const __grid_constant__ 
 }
 
 }  // namespace
+
+// Scored policy, warm start: the r latest queries of every (seq, query head), oldest first,
+// into the window slots of their steps.
+struct RestoreQParams {
+    DevLayout lay;
+    int layer;
+    const uint16_t* q;  // [B][H][r][128]
+    int32_t g[RA_MAX_BATCH];
+};
+
+__global__ void __launch_bounds__(256) restore_queries_kernel(const __grid_constant__ RestoreQParams p)
+{
+    const DevLayout& L = p.lay;
+    const int b = blockIdx.x / L.H, qh = blockIdx.x - b * L.H;
+    const int h = qh / L.G, gq = qh - h * L.G;
+    const int r = L.r;
+    uint16_t* win = L.qring + (((size_t)p.layer * L.B + b) * L.KVH + h) * (size_t)r * L.G * kHeadDim;
+    const uint16_t* src = p.q + ((size_t)b * L.H + qh) * (size_t)r * kHeadDim;
+    for (int i = threadIdx.x; i < r * 16; i += blockDim.x) {
+        const int u = i >> 4, c = i & 15;
+        const int step = p.g[b] - r + 1 + u;  // 1-based decode step of row u
+        if (step < 1) continue;
+        const int slot = (step - 1) % r;
+        reinterpret_cast<uint4*>(win + ((size_t)slot * L.G + gq) * kHeadDim)[c] =
+            reinterpret_cast<const uint4*>(src + (size_t)u * kHeadDim)[c];
+    }
+}
+
+cudaError_t launch_restore_queries(const DevLayout& lay, int layer, const uint16_t* q, const int32_t* g_host,
+                                   cudaStream_t s)
+{
+    RestoreQParams p{};
+    p.lay = lay;
+    p.layer = layer;
+    p.q = q;
+    for (int b = 0; b < lay.B; ++b) p.g[b] = g_host[b];
+    restore_queries_kernel<<<lay.B * lay.H, 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s)
 {

@@ -37,6 +37,11 @@ struct DevLayout {
     int32_t* arrive;       // [B*KVH] split-piece arrival counters
     unsigned long long* ticket;  // attention chunk-stealing counter
     int32_t* err;          // device error word
+    // scored policy (null when the context was bound without its buffers)
+    uint16_t* qring;       // [L][B][KVH][r][G][128] bf16: query of step s in slot (s - 1) mod r
+    float* scores;         // [L][B][KVH][Cmax] raw window score of each candidate of the latest round
+    float* stats;          // [B*KVH][stats_chunks][Mpad][2] pass-1 softmax statistics (max, sum) per chunk
+    int stats_chunks;      // chunks per head the stats buffer holds
     long long prompt_rows_per_layer;
     long long gen_row0;    // first row of the generated regions
     int L, B, KVH, H, G, Cmax, K, r;
@@ -64,7 +69,14 @@ struct EvictParams {
     int32_t trig_c[RA_MAX_BATCH];  // rows in the cache (a pending new token is not among them)
     int32_t trig_n[RA_MAX_BATCH];  // candidates (all rows but the newest r, counting a pending token)
     int32_t trig_g[RA_MAX_BATCH];  // step of the draw: generated tokens including this step's
+    // scored policy: tiles (of kScoreTile rows) per CTA of each pass, CTAs per head of each pass
+    int ch1, ch2, nch1, nch2;
+    float qk_scale_log2;
 };
+
+constexpr int kScoreTile = 64;      // key rows per scoring tile
+constexpr int kScoreMaxRows = 512;  // r * G window rows the scoring kernels hold
+constexpr int kScorePoolRadius = 3; // max-pool width 7 over neighbouring candidates
 
 // Attention work is counted in tiles of TILE rows: a head has ceil(lp / TILE) prompt tiles and
 // ceil(gen / TILE) tiles of generated rows (gen includes a fused new token, its last row).
@@ -89,7 +101,9 @@ struct AttnParams {
     uint32_t active[RA_MAX_BATCH / 32];
     int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of tiles per head over active sequences
     int32_t seq_gen[RA_MAX_BATCH];       // generated rows attended per head (incl. a fused new token)
-    int32_t seq_g[RA_MAX_BATCH];         // fused append: tokens generated before this one
+    int32_t seq_g[RA_MAX_BATCH];         // tokens generated before this step's (fused) / up to it (separate)
+    uint16_t* qring;                     // record each head's query rows in the scored policy's window (or null)
+    int ring_off;                        // window slot of sequence b = (seq_g[b] + ring_off) mod r
 };
 
 struct CopyRowsParams {
@@ -108,6 +122,14 @@ cudaError_t launch_select(const EvictParams& p, cudaStream_t s);
 cudaError_t launch_compact(const EvictParams& p, cudaStream_t s);
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s);
 cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s);
+cudaError_t launch_restore_queries(const DevLayout& lay, int layer, const uint16_t* q, const int32_t* g_dev,
+                                   cudaStream_t s);
+
+// Scored policy: pass 1 (softmax statistics) or pass 2 (per-candidate sums) of the window attention.
+// The tensor map covers kpool as [total_rows][128] bf16 with boxes of kScoreTile rows x 64 channels.
+cudaError_t launch_score(const EvictParams& p, int pass, const CUtensorMap* tmap_k, cudaStream_t s);
+cudaError_t score_prepare();
+int score_row_tiles_per_warp(int M);  // 16-row tiles of the M window rows per warp (1..4)
 
 // Attention: the tensor maps cover kpool / vpool as [total_rows][128] bf16.
 int attn_warps_per_cta(int G);

@@ -12,10 +12,38 @@ import synth
 
 MAX_ABS = 2e-2     # attention tolerance (bf16 inputs, fp32 accumulation, bf16 output)
 MEAN_REL = 5e-3    # sum |o - o*| / sum |o*|
+# Window scores of the scored comparator (sums of softmax weights, fp32 logits and exp2 on the GPU):
+# each weight carries a relative error of order 1e-5 (fp32 dot products of bf16 rows, the merged
+# softmax statistics, exp2); 1e-3 relative leaves two orders of margin.
+SCORE_RTOL = 1e-3
+SCORE_ATOL = 1e-7
 
 
 def bf16_to_f64(x):
     return synth.bf16_bits_to_f32(np.asarray(x).view(np.uint16)).astype(np.float64)
+
+
+def check_scores(got, ref, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    assert got.shape == ref.shape, (what, got.shape, ref.shape)
+    err = np.abs(got - ref)
+    bad = err > SCORE_RTOL * np.abs(ref) + SCORE_ATOL
+    assert not bad.any(), f"{what}: {int(bad.sum())} scores off, worst {float((err / (np.abs(ref) + 1e-30)).max()):.3g}"
+
+
+def check_scored_decision(got, ref, K, what=""):
+    """The kernel decides with its fp32 scores; where the fp64 scores decide differently, the
+    candidates concerned must sit at the threshold (their pooled fp64 score within tolerance of
+    the K-th largest)."""
+    if K == 0 or got.size == 0:
+        return 0
+    pg = oracle.max_pool(np.asarray(got, dtype=np.float64))
+    pr = oracle.max_pool(ref)
+    kg, kr = set(oracle.select_top(pg, K).tolist()), set(oracle.select_top(pr, K).tolist())
+    thr = np.sort(pr)[::-1][K - 1]
+    for j in kg ^ kr:
+        assert abs(pr[j] - thr) <= SCORE_RTOL * thr + SCORE_ATOL, f"{what}: candidate {j} far from the threshold"
+    return len(kg ^ kr)
 
 
 def check_attention(got_bits, ref, what=""):
@@ -43,11 +71,13 @@ class Runner:
         self.B = len(self.lp)
         self.K, self.r, self.eseed, self.dseed = K, r, eseed, dseed
         self.key_scale = key_scale  # fp32 [L][KVH][D] or None
-        self.cache = ra.RandomAttentionCache(L, H, KVH, D, self.lp, K, r, eseed)
+        self.cache = ra.RandomAttentionCache(L, H, KVH, D, self.lp, K, r, eseed, policy=policy, block=block)
         self.ctx = self.cache.ctx
         self.orc = oracle.OracleCache(L, KVH, self.lp, K, r, eseed, policy=policy, block=block)
-        if policy:
-            ra.ra_set_policy(self.ctx, policy, block)
+        self.policy = policy
+        self.qsteps = [[] for _ in range(self.B)]  # step index of each of a sequence's decode steps
+        self.scored_rounds = 0
+        self.near_ties = 0
         self.dev = torch.device("cuda")
         self.step_idx = 0
         self.fused = fused  # True: one ra_decode_layer call per layer instead of append/evict/attend
@@ -83,6 +113,10 @@ class Runner:
         """One decode step over all layers; returns {layer: n_fired} and checks attention where asked."""
         fired = {}
         outs = {}
+        for b in range(self.B):
+            if self.active[b]:
+                self.qsteps[b].append(self.step_idx)
+        scored = self.policy == oracle.POLICY_SNAPKV
         for l in range(self.L):
             k = np.zeros((self.B, self.KVH, self.D), np.uint16)
             v = np.zeros_like(k)
@@ -98,7 +132,8 @@ class Runner:
                           for b in range(self.B)])
             out = self.torch.zeros((self.B, self.H, self.D), dtype=self.torch.int16, device=self.dev)
             tq = self.up(q)
-            nf = sum(1 for b in range(self.B) if self.active[b] and self.orc.evict(b, l))
+            if not scored:
+                nf = sum(1 for b in range(self.B) if self.active[b] and self.orc.evict(b, l))
             if self.fused:
                 before = [self.ra.ra_get_counters(self.ctx, b, l)[2] for b in range(self.B)]
                 self.ra.ra_decode_layer(self.ctx, l, tq.data_ptr(), tk.data_ptr(), tv.data_ptr(), out.data_ptr(), scale)
@@ -107,6 +142,8 @@ class Runner:
                 self.ra.ra_append_kv(self.ctx, l, tk.data_ptr(), tv.data_ptr())
                 n = self.ra.ra_evict(self.ctx, l)
                 self.ra.ra_decode_attn(self.ctx, l, tq.data_ptr(), out.data_ptr(), scale)
+            if scored:  # the oracle's round needs the kernel's scores of this step
+                nf = sum(1 for b in range(self.B) if self.active[b] and self.orc.evict(b, l, scorer=self.scorer))
             assert n == nf, (l, n, nf)
             fired[l] = n
             if l in check_attn_layers:
@@ -115,6 +152,27 @@ class Runner:
             self.check_layer_attention(l, q, out.cpu().numpy(), scale)
         self.step_idx += 1
         return fired
+
+    def window(self, l, b, h, g):
+        """Query rows [r][G][D] and positions of the window at an eviction after token g."""
+        steps = range(g - self.r, g)  # 1-based decode steps of the window
+        heads = np.arange(h * self.G, (h + 1) * self.G)
+        q = np.stack([synth.q_rows(self.dseed, l, b, heads, self.qsteps[b][s - 1], self.D) for s in steps])
+        return q, np.array([self.lp[b] + s - 1 for s in steps], dtype=np.int32)
+
+    def scorer(self, b, l, h, cur):
+        """Oracle scorer of the scored policy: the fp64 window scores must match the kernel's within
+        tolerance; the round then follows the kernel's fp32 scores (see check_scored_decision)."""
+        g, n = int(self.orc.g[b, l]), cur.size - self.r
+        q, qpos = self.window(l, b, h, g)
+        kpos = self.orc.positions(b, l, h)
+        ref = oracle.window_scores(q, qpos, self.krows(l, b, h, kpos), kpos)[self.lp[b]:self.lp[b] + n]
+        got = self.ra.ra_get_scores(self.ctx, l, b, h, self.K + 2 * self.r)
+        what = f"scores l{l} b{b} h{h} g{g}"
+        check_scores(got, ref, what)
+        self.near_ties += check_scored_decision(got, ref, self.K, what)
+        self.scored_rounds += 1
+        return got.astype(np.float64)
 
     def check_layer_attention(self, l, q, got, scale=0.0):
         for b in range(self.B):

@@ -74,6 +74,35 @@ def test_device_bytes_cover_the_caches(ra):
     ra.ra_destroy(ctx)
 
 
+def test_scored_policy_sizes_its_buffers_before_bind(ra):
+    """The scored policy adds the query window (L*B*KVH*r*G rows), the scores (L*B*KVH*(K+2r) fp32)
+    and the pass-1 statistics to the arena; it must be chosen before binding; r*G is capped at 512."""
+    L, B, H, KVH, K, r = 4, 3, 32, 8, 256, 64
+    ctx = ra.ra_create_batched(L, H, KVH, 128, [100, 0, 700], K, r, 0)
+    base = ra.ra_device_bytes(ctx)
+    ra.ra_set_policy(ctx, ra.RA_POLICY_SNAPKV)
+    grown = ra.ra_device_bytes(ctx)
+    window = L * B * KVH * r * (H // KVH) * 256
+    scores = L * B * KVH * (K + 2 * r) * 4
+    assert grown >= base + window + scores
+    assert grown < base + window + scores + (64 << 20)
+    ra.ra_set_policy(ctx, ra.RA_POLICY_RANDOM)  # the buffers stay: switching back is allowed
+    assert ra.ra_device_bytes(ctx) == grown
+    with pytest.raises(ra.RAError) as e:
+        ra.ra_set_policy(ctx, 5)
+    assert e.value.code == ra.RA_ERR_INVALID_ARG
+    ra.ra_destroy(ctx)
+    big = ra.ra_create_batched(1, 64, 8, 128, [10], 64, 128, 0)  # r * G = 1024
+    with pytest.raises(ra.RAError) as e:
+        ra.ra_set_policy(big, ra.RA_POLICY_SNAPKV)
+    assert e.value.code == ra.RA_ERR_UNSUPPORTED
+    lib = ra.lib()
+    assert lib.ra_restore_queries(big, 0, None, None) == ra.RA_ERR_STATE  # unbound
+    n = ctypes.c_int(0)
+    assert lib.ra_get_scores(big, 0, 0, 0, None, 0, ctypes.byref(n), None) == ra.RA_ERR_STATE
+    ra.ra_destroy(big)
+
+
 def test_no_cpu_fallback_in_product_package():
     """The product package never imports the oracle (test infrastructure)."""
     pkg = os.path.join(ROOT, "paper_2609_03430_gb300")
