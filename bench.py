@@ -58,6 +58,9 @@ def _workloads():
 
 WORKLOADS = _workloads()
 DEFAULT_CONFIG = 2
+COMPARATOR_CONFIGS = (5,)  # workloads that also time the scored comparator on the same caches
+POLICY_SNAPKV = 4
+WINDOW_STEP0 = 1 << 20     # synthetic step index of the first restored window query (row u: WINDOW_STEP0 + u)
 
 
 def steady_state(w, rank=0):
@@ -92,7 +95,7 @@ def describe(w):
 class Workload:
     """Device-side setup of one workload through the public API."""
 
-    def __init__(self, cfg, rank=0, ring=4):
+    def __init__(self, cfg, rank=0, ring=4, policy=0):
         import torch
 
         import paper_2609_03430_gb300 as ra
@@ -108,13 +111,17 @@ class Workload:
         self.eseed = w["eseed"] + (rank << 32)
         self.dev = torch.device("cuda", torch.cuda.current_device())
         self.stream = torch.cuda.current_stream()
-        self.cache = ra.RandomAttentionCache(self.L, self.H, self.KVH, D, self.lp, self.K, self.r, self.eseed)
+        self.policy = policy
+        self.cache = ra.RandomAttentionCache(self.L, self.H, self.KVH, D, self.lp, self.K, self.r, self.eseed,
+                                             policy=policy)
         self.ctx = self.cache.ctx
         self.key_scale = None
         if w["key_scale"]:
             self.key_scale = torch.from_numpy(synth.key_channel_scale(self.dseed, self.L, self.KVH, D)).to(self.dev)
         self.g0, self.c0 = steady_state(w, rank)
         self._fill()
+        if policy == POLICY_SNAPKV:
+            self._fill_window()
         self.ring = ring
         self._make_inputs(ring)
 
@@ -149,6 +156,23 @@ class Workload:
                 self.ra.ra_restore(self.ctx, l, self.g0, self.c0, gpos.data_ptr(), kg.data_ptr(), vg.data_ptr(), maxc)
         torch.cuda.synchronize()
         del kp, vp, kg, vg
+
+    def _fill_window(self):
+        """Scored policy: the window of the r steps before the start, synthetic queries (row u of every
+        (seq, query head) is the generator's query for step index WINDOW_STEP0 + u)."""
+        torch = self.torch
+        B, H, r = self.B, self.H, self.r
+        pos = (WINDOW_STEP0 + torch.arange(r, dtype=torch.int32)).repeat(B, H, 1).contiguous().to(self.dev)
+        qw = torch.empty((B, H, r, D), dtype=torch.int16, device=self.dev)
+        for l in range(self.L):
+            self.sg.fill_rows(qw, pos, self.dseed, 2, l, 0)
+            self.ra.ra_restore_queries(self.ctx, l, qw.data_ptr())
+        torch.cuda.synchronize()
+        del qw
+
+    def evictions(self):
+        """Eviction rounds so far, summed over (sequence, layer)."""
+        return sum(self.ra.ra_get_counters(self.ctx, b, l)[2] for b in range(self.B) for l in range(self.L))
 
     def _make_inputs(self, ring):
         """Device-resident inputs of `ring` distinct steps (cycled): q [L][B][H][d], k/v [L][B][KVH][d]."""
@@ -359,6 +383,86 @@ def config_dict(w, args):
 
 
 # --------------------------------------------------------------------------- GPU run
+def timed_steps(wl, steps, t_next, barrier):
+    """Device time per step of `steps` whole-stack decode steps: CUDA events on the stream only at
+    its ends (no per-kernel events, which would break the overlap of consecutive launches)."""
+    import torch
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    wall0 = time.time()
+    e0.record(wl.stream)
+    for t in range(t_next, t_next + steps):
+        wl.step(t)
+    e1.record(wl.stream)
+    barrier()
+    wall1 = time.time()
+    return e0.elapsed_time(e1) / steps, t_next + steps, wall0, wall1
+
+
+def evented_steps(wl, steps, t_next):
+    """The same number of steps again with CUDA events around every launch (on the launching
+    stream): per-kernel durations and algorithmic bytes, and the eviction rounds they covered."""
+    import torch
+
+    ra = wl.ra
+    rounds0 = wl.evictions()
+    ra.ra_profile_reset(wl.ctx)
+    ra.ra_profile_enable(wl.ctx, True)
+    for t in range(t_next, t_next + steps):
+        wl.step(t)
+    torch.cuda.synchronize()
+    ra.ra_profile_enable(wl.ctx, False)
+    kern = {}
+    for kind, name in enumerate(ra.KERNEL_NAMES):
+        kms, n, by = ra.ra_profile_read(wl.ctx, kind)
+        if n:
+            kern[name] = {"launches": n, "ms_total": kms, "us_per_launch": 1000.0 * kms / n,
+                          "bytes_per_launch": by / n,
+                          "algorithmic_GBps": (by / (kms * 1e-3) / 1e9) if kms > 0 else None}
+    ra.ra_check_device(wl.ctx)
+    return kern, wl.evictions() - rounds0, t_next + steps
+
+
+def _eviction_us_per_round(kern, names, rounds):
+    if not rounds:
+        return None
+    return 1000.0 * sum(kern[n]["ms_total"] for n in names if n in kern) / rounds
+
+
+def run_comparator(args, rank, world, barrier, peaks, random_ms, random_kern, random_rounds):
+    """The scored comparator (SnapKV-style window top-K, prompt pinned) on the same caches: the
+    workload rebuilt from the same seeds with the scored policy and a restored query window,
+    timed like the main run; per-round cost of its eviction kernels next to the random policy's."""
+    wl = Workload(args.config, rank=rank, policy=POLICY_SNAPKV)
+    for t in range(args.warmup):
+        wl.step(t)
+    wl.ra.ra_check_device(wl.ctx)
+    ms, t_next, _, _ = timed_steps(wl, args.steps, args.warmup, barrier)
+    kern, rounds, _ = evented_steps(wl, args.steps, t_next)
+    ms_step, units = reduce_over_ranks(ms, float(wl.B), world)
+    M = wl.r * wl.G
+    score = {}
+    for name in ("score_stats", "score_sum"):
+        k = kern.get(name)
+        if k and k["ms_total"] > 0:
+            # algorithmic bytes of these kinds are the key rows read; each costs 2 * M * 128 flops
+            tflops = k["bytes_per_launch"] * M / (k["us_per_launch"] * 1e-6) / 1e12
+            score[name] = dict(k, tensor_TFLOPs=tflops, bound="tensor",
+                               frac_of_bf16_peak=tflops / peaks["bf16_tflops"])
+    wl.cache.close()
+    return {"policy": "snapkv-style window top-K: window = the last r queries, scores summed over the "
+                      "query heads of the group, max-pool width 7, prompt pinned, r-token buffer unscored",
+            "value": units / (ms_step * 1e-3), "unit": UNIT, "ms_per_step": ms_step,
+            "step_time_vs_random": ms_step / random_ms,
+            "rounds_in_evented_pass": {"random": random_rounds, "snapkv": rounds},
+            "eviction_us_per_round": {
+                "random": _eviction_us_per_round(random_kern, ("select", "compact"), random_rounds),
+                "snapkv": _eviction_us_per_round(kern, ("score_stats", "score_sum", "select", "compact"), rounds),
+                "what": "evented kernel time of a step's eviction launches / (sequence, layer) rounds they ran"},
+            "score_kernels": score, "kernels": kern}
+
+
 def run_ours(args, w):
     import torch
 
@@ -388,46 +492,19 @@ def run_ours(args, w):
     ra.ra_check_device(ctx)
     attn_bytes_before = wl.bytes_per_step()
 
-    # Timed region: K whole-stack decode steps, CUDA events on the stream only at its ends
-    # (no per-kernel events, which would break the overlap of consecutive launches).
+    # Timed region: K whole-stack decode steps.
     ra.ra_profile_reset(ctx)
     clocks = ClockSampler(torch.cuda.current_device())
     clocks.start()
     time.sleep(0.3)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    barrier()
-    wall0 = time.time()
-    e0.record(stream)
-    t_next = args.warmup
-    for t in range(t_next, t_next + args.steps):
-        wl.step(t)
-    e1.record(stream)
-    barrier()
-    wall1 = time.time()
+    ms, t_next, wall0, wall1 = timed_steps(wl, args.steps, args.warmup, barrier)
     clocks.stop()
-    t_next += args.steps
-    ms_total = e0.elapsed_time(e1)
     launches = sum(ra.ra_profile_read(ctx, kind)[1] for kind in range(len(ra.KERNEL_NAMES)))
 
-    # Kernel durations: the same number of steps again with CUDA events around every launch
-    # (on the launching stream), for the per-kernel achieved bandwidth.
-    ra.ra_profile_reset(ctx)
-    ra.ra_profile_enable(ctx, True)
-    for t in range(t_next, t_next + args.steps):
-        wl.step(t)
-    torch.cuda.synchronize()
-    t_next += args.steps
-    ra.ra_profile_enable(ctx, False)
-    kern = {}
-    for kind, name in enumerate(ra.KERNEL_NAMES):
-        kms, n, by = ra.ra_profile_read(ctx, kind)
-        if n:
-            kern[name] = {"launches": n, "ms_total": kms, "us_per_launch": 1000.0 * kms / n,
-                          "bytes_per_launch": by / n,
-                          "algorithmic_GBps": (by / (kms * 1e-3) / 1e9) if kms > 0 else None}
-    ra.ra_check_device(ctx)
+    # Kernel durations: the same number of steps again with CUDA events around every launch.
+    kern, rounds, t_next = evented_steps(wl, args.steps, t_next)
 
-    ms_step, units = reduce_over_ranks(ms_total / args.steps, float(wl.B), world)
+    ms_step, units = reduce_over_ranks(ms, float(wl.B), world)
     value = units / (ms_step * 1e-3)
 
     # e2e: the same steps with host buffers -- H2D of the step's inputs from pinned memory,
@@ -455,6 +532,9 @@ def run_ours(args, w):
         e2e = {"value": e2e_units / (e2e_ms * 1e-3), "unit": UNIT,
                "h2d_bytes_per_step": int(hq.numel() * 2 + hk.numel() * 2 + hv.numel() * 2),
                "d2h_bytes_per_step": int(ho.numel() * 2), "ms_per_step": e2e_ms}
+        del hq, hk, hv, ho, dq, dk, dv
+    wl.cache.close()
+    del wl
 
     peaks, peak_src = measured_peaks()
     a = kern.get("attn")
@@ -471,6 +551,9 @@ def run_ours(args, w):
                 "timing": "CUDA events around every attention launch on its stream, in a second pass of "
                           "the same number of steps (events between launches defeat their overlap, so "
                           "this duration is an upper bound)"}
+    comparator = None
+    if args.comparator == "on" or (args.comparator == "auto" and args.config in COMPARATOR_CONFIGS):
+        comparator = run_comparator(args, rank, world, barrier, peaks, ms_step, kern, rounds)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)
@@ -485,12 +568,13 @@ def run_ours(args, w):
                                    "frac": attn_bytes_before / (ms_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
                                    "what": "cache bytes streamed per step / device time per step "
                                            "(all kernels of the step, launches overlapped)"}}
+        if comparator is not None:
+            line["comparator"] = comparator
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
 
         dist.destroy_process_group()
-    wl.cache.close()
     return 0
 
 
@@ -506,6 +590,8 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--layers", type=int, default=None,
                     help="override the layer count (only to shrink profiler captures; not a benchmark workload)")
+    ap.add_argument("--comparator", choices=["auto", "on", "off"], default="auto",
+                    help="also time the scored comparator on the same caches (auto: the ragged workload)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per attention launch (from a committed profile), if current")
     args = ap.parse_args(argv)

@@ -262,6 +262,8 @@ int ra_check_device(ra_ctx* ctx, void* stream);
  * always counted; CUDA-event timing of every launch is recorded only while
  * enabled (ra_profile_enable).  ra_profile_read synchronises on the recorded
  * events and returns the totals of one ra_kernel_kind since the last reset.
+ * For the two scoring kinds the bytes are the key rows read (256 bytes each,
+ * every one contracted with the M = r * G window rows: flops = bytes * M).
  */
 int ra_profile_enable(ra_ctx* ctx, int on);
 int ra_profile_read(ra_ctx* ctx, int kind, double* total_ms, int64_t* launches, double* algorithmic_bytes);

@@ -319,10 +319,10 @@ void plan_scoring(ra_ctx* ctx, EvictParams* p, double* bytes1, double* bytes2)
     p->nch1 = (int)((max1 + ch1 - 1) / ch1);
     p->nch2 = (int)((max2 + ch2 - 1) / ch2);
     p->qk_scale_log2 = 1.4426950408889634f / sqrtf((float)kHeadDim);
-    // key rows read once and the window once per head; pass 2 also writes one score per candidate
-    const double win = (double)p->n_trig * ctx->KVH * M * kRowBytes;
-    *bytes1 = rows1 * kRowBytes + win;
-    *bytes2 = rows2 * (kRowBytes + 4) + win;
+    // counted as the key rows read (the window, read once per CTA, is L2-resident): every key
+    // row costs 2 * M * 128 flops, so flops = bytes * M
+    *bytes1 = rows1 * kRowBytes;
+    *bytes2 = rows2 * kRowBytes;
 }
 
 // One eviction round of the triggered sequences in p: [score passes,] select, compact.

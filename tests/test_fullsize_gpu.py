@@ -89,3 +89,87 @@ def test_workload_parity_sampled(cfg):
         ref = oracle.attend(qv, krow, vrow)
         check_attention(got_out[l, b, h * G:(h + 1) * G], ref, f"cfg {cfg} slice {(b, l, h)}")
     wl.cache.close()
+
+
+def test_scored_comparator_parity_full_size():
+    """The scored comparator at the ragged workload's full size (the configuration bench.py times it
+    in): query window restored, r + 2 steps so that every sequence scores once; sampled heads' raw
+    scores within tolerance of the fp64 oracle, keep-sets equal to the oracle's round on the kernel's
+    scores (fp64 disagreements only at the threshold), survivors and attention as for the method."""
+    import torch
+
+    import bench
+    import oracle
+    import paper_2609_03430_gb300 as ra
+    import synth
+    import synth.gpu as sg
+    from ra_testlib import check_scored_decision, check_scores
+
+    torch.cuda.set_device(0)
+    cfg = 5
+    wl = bench.Workload(cfg, ring=1, policy=bench.POLICY_SNAPKV)
+    w = wl.w
+    L, B, H, KVH, K, r, D = wl.L, wl.B, wl.H, wl.KVH, wl.K, wl.r, 128
+    G = H // KVH
+    heads, attn_heads = _samples(w, 10, 4, 77)
+    orc = oracle.OracleCache(L, KVH, wl.lp, K, r, wl.eseed, heads=heads, policy=oracle.POLICY_SNAPKV)
+    for (b, l, h) in heads:
+        c, g = wl.c0[b], wl.g0[b]
+        orc.gen[(b, l, h)] = np.arange(wl.lp[b] + g - c, wl.lp[b] + g, dtype=np.int32)
+        orc.g[b, l] = g
+
+    def step_index(b, s):  # generator step index of sequence b's 1-based decode step s
+        g0 = wl.g0[b]
+        return bench.WINDOW_STEP0 + s - (g0 - r + 1) if s <= g0 else s - g0 - 1
+
+    rounds = [0]
+
+    def scorer(b, l, h, cur):
+        g, n = int(orc.g[b, l]), cur.size - r
+        steps = range(g - r, g)
+        qh = np.arange(h * G, (h + 1) * G)
+        q = np.stack([synth.q_rows(wl.dseed, l, b, qh, step_index(b, s), D) for s in steps])
+        qpos = np.array([wl.lp[b] + s - 1 for s in steps], dtype=np.int32)
+        kpos = orc.positions(b, l, h)
+        krow = synth.kv_rows(wl.dseed, 0, l, b, h, kpos, D)
+        ref = oracle.window_scores(q, qpos, krow, kpos)[wl.lp[b]:wl.lp[b] + n]
+        got = ra.ra_get_scores(wl.ctx, l, b, h, K + 2 * r)
+        check_scores(got, ref, f"scores {(b, l, h)} g{g}")
+        check_scored_decision(got, ref, K, f"decision {(b, l, h)} g{g}")
+        rounds[0] += 1
+        return got.astype(np.float64)
+
+    dev = wl.dev
+    q = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((L, B, KVH, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    out = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    steps = r + 2
+    for t in range(steps):
+        qpos = torch.full((B, H, 1), t, dtype=torch.int32, device=dev)
+        npos = torch.tensor([[wl.lp[b] + wl.g0[b] + t] * KVH for b in range(B)], dtype=torch.int32,
+                            device=dev).reshape(B, KVH, 1)
+        for l in range(L):
+            sg.fill_rows(q[l].view(B, H, 1, D), qpos, wl.dseed, 2, l, 0)
+            sg.fill_rows(kn[l].view(B, KVH, 1, D), npos, wl.dseed, 0, l, 0)
+            sg.fill_rows(vn[l].view(B, KVH, 1, D), npos, wl.dseed, 1, l, 0)
+        ra.ra_decode_step(wl.ctx, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), out.data_ptr(), 0.0)
+        torch.cuda.synchronize()
+        for (b, l) in sorted({(b, l) for (b, l, _) in heads}):
+            orc.append(b, l)
+            orc.evict(b, l, scorer=scorer)
+    ra.ra_check_device(wl.ctx)
+    assert rounds[0] >= len(heads)  # every sampled head scored at least once
+    for (b, l, h) in heads:
+        got = ra.ra_get_positions(wl.ctx, l, b, h, K + 2 * r)
+        np.testing.assert_array_equal(got, orc.gen[(b, l, h)], err_msg=f"positions {(b, l, h)}")
+    got_out = out.cpu().numpy()
+    for (b, l, h) in attn_heads:
+        pos = orc.positions(b, l, h)
+        kk, vv = ra.ra_get_kv(wl.ctx, l, b, h, wl.lp[b] + K + 2 * r)
+        np.testing.assert_array_equal(kk, synth.kv_rows(wl.dseed, 0, l, b, h, pos, D), err_msg=f"K rows {(b, l, h)}")
+        np.testing.assert_array_equal(vv, synth.kv_rows(wl.dseed, 1, l, b, h, pos, D), err_msg=f"V rows {(b, l, h)}")
+        qv = synth.q_rows(wl.dseed, l, b, np.arange(h * G, (h + 1) * G), steps - 1, D)
+        ref = oracle.attend(qv, synth.kv_rows(wl.dseed, 0, l, b, h, pos, D), synth.kv_rows(wl.dseed, 1, l, b, h, pos, D))
+        check_attention(got_out[l, b, h * G:(h + 1) * G], ref, f"slice {(b, l, h)}")
+    wl.cache.close()
