@@ -379,7 +379,8 @@ def config_dict(w, args):
     return {"workload": describe(w), "config_index": args.config, "batch": w["B"], "layers": w["L"],
             "q_heads": w["H"], "kv_heads": w["KVH"], "head_dim": D, "K": w["K"], "r": w["r"],
             "prompt_mean": float(np.mean(w["lp"])), "start": "steady state (K + r cached generated per head)",
-            "l2": "inputs larger than L2 (every step streams the whole cache)", "parallelism": f"replicas x{args.gpus}"}
+            "l2": "inputs larger than L2 (every step streams the whole cache)", "parallelism": f"replicas x{args.gpus}",
+            "policy": getattr(args, "policy", "random")}
 
 
 # --------------------------------------------------------------------------- GPU run
@@ -476,7 +477,8 @@ def run_ours(args, w):
         dist.init_process_group("nccl")
     else:
         torch.cuda.set_device(0)
-    wl = Workload(args.config, rank=rank)
+    main_policy = POLICY_SNAPKV if args.policy == "snapkv" else 0
+    wl = Workload(args.config, rank=rank, policy=main_policy)
     stream = wl.stream
     ctx = wl.ctx
 
@@ -552,7 +554,8 @@ def run_ours(args, w):
                           "the same number of steps (events between launches defeat their overlap, so "
                           "this duration is an upper bound)"}
     comparator = None
-    if args.comparator == "on" or (args.comparator == "auto" and args.config in COMPARATOR_CONFIGS):
+    if main_policy == 0 and (args.comparator == "on" or
+                             (args.comparator == "auto" and args.config in COMPARATOR_CONFIGS)):
         comparator = run_comparator(args, rank, world, barrier, peaks, ms_step, kern, rounds)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -590,6 +593,8 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--layers", type=int, default=None,
                     help="override the layer count (only to shrink profiler captures; not a benchmark workload)")
+    ap.add_argument("--policy", choices=["random", "snapkv"], default="random",
+                    help="eviction policy of the timed run (random: the method; snapkv: the scored comparator)")
     ap.add_argument("--comparator", choices=["auto", "on", "off"], default="auto",
                     help="also time the scored comparator on the same caches (auto: the ragged workload)")
     ap.add_argument("--traffic", type=float, default=None,

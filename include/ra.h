@@ -69,8 +69,8 @@ enum ra_kernel_kind {
     RA_KERNEL_SELECT = 1,
     RA_KERNEL_COMPACT = 2,
     RA_KERNEL_ATTN = 3,
-    RA_KERNEL_SCORE_STATS = 4, /* scored comparator, pass 1: softmax statistics of the window queries */
-    RA_KERNEL_SCORE_SUM = 5,   /* scored comparator, pass 2: attention summed per candidate */
+    RA_KERNEL_SCORE_STATS = 4, /* scored comparator: normalisers of a restored query window */
+    RA_KERNEL_SCORE_SUM = 5,   /* scored comparator: window attention summed per candidate */
     RA_KERNEL_KINDS = 6
 };
 
@@ -134,15 +134,18 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
  *                      side (SnapKV as section 2 writes it, with the prompt
  *                      pinned and the buffer unscored as for the method); the
  *                      K best survive, ties to the earlier position.  Each
- *                      window query attends with scale 1/sqrt(head_dim) to the
- *                      keys at positions up to its own.
+ *                      window query's weights are those of its own decode
+ *                      step: the same scale, over the keys at positions up
+ *                      to its own (the cache only grows between rounds, so
+ *                      that is what it saw; the attention calls record each
+ *                      query's softmax normaliser for this).
  * Takes effect from the next eviction; `block` >= 1 is used by RA_POLICY_BLOCK.
  *
  * The scored policy needs a per-layer window of recent queries, which the
  * attention calls record: set it BEFORE ra_device_bytes / ra_bind (the arena
  * then also holds the window, the scores and their scratch, and the context
  * keeps recording the window under every policy); on a context bound without
- * them it fails with RA_ERR_STATE.  It requires r * G <= 512.
+ * them it fails with RA_ERR_STATE.  It requires r * G <= 512 and K + r <= 16384.
  */
 #define RA_POLICY_RANDOM 0
 #define RA_POLICY_SHARED 1
@@ -155,10 +158,13 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block);
  * Scored policy, warm start: load the query window of layer `layer` from q,
  * device [batch][q_heads][r][head_dim] bf16, where row u of (b, qh) is the
  * query of decode step g_b - r + 1 + u (g_b = the sequence's generated count,
- * so row r - 1 is the latest step).  Steps before the first are never read.
+ * so row r - 1 is the latest step), attended at `scale` (<= 0: 1/sqrt(d)).
+ * Call it after ra_prefill / ra_restore of the layer: it also recomputes each
+ * loaded query's softmax normaliser over the prompt and the cached rows at
+ * positions up to its own.  Steps before the first are never read.
  * RA_ERR_STATE unless the context was bound with the scored policy's buffers.
  */
-int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, void* stream);
+int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, float scale, void* stream);
 
 /*
  * Debug (scored policy): copy the raw window scores (before pooling) that the
@@ -262,8 +268,9 @@ int ra_check_device(ra_ctx* ctx, void* stream);
  * always counted; CUDA-event timing of every launch is recorded only while
  * enabled (ra_profile_enable).  ra_profile_read synchronises on the recorded
  * events and returns the totals of one ra_kernel_kind since the last reset.
- * For the two scoring kinds the bytes are the key rows read (256 bytes each,
- * every one contracted with the M = r * G window rows: flops = bytes * M).
+ * For the two scoring kinds (RA_KERNEL_SCORE_STATS runs only in
+ * ra_restore_queries) the bytes are the key rows read (256 bytes each, every
+ * one contracted with the M = r * G window rows: flops = bytes * M).
  */
 int ra_profile_enable(ra_ctx* ctx, int on);
 int ra_profile_read(ra_ctx* ctx, int kind, double* total_ms, int64_t* launches, double* algorithmic_bytes);

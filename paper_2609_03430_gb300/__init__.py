@@ -42,7 +42,7 @@ SIGNATURES = {
     "ra_prefill": (_i, [_vp, _i, _vp, _vp, _i, _vp]),
     "ra_restore": (_i, [_vp, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp]),
     "ra_set_policy": (_i, [_vp, _i, _i]),
-    "ra_restore_queries": (_i, [_vp, _i, _vp, _vp]),
+    "ra_restore_queries": (_i, [_vp, _i, _vp, ctypes.c_float, _vp]),
     "ra_get_scores": (_i, [_vp, _i, _i, _i, ctypes.POINTER(ctypes.c_float), _i, _ip, _vp]),
     "ra_set_active": (_i, [_vp, _i, _i]),
     "ra_append_kv": (_i, [_vp, _i, _vp, _vp, _vp]),
@@ -144,8 +144,8 @@ def ra_set_policy(ctx, policy, block=1):
     return _check(lib().ra_set_policy(ctx, int(policy), int(block)), ctx)
 
 
-def ra_restore_queries(ctx, layer, q_ptr, stream=None):
-    return _check(lib().ra_restore_queries(ctx, layer, q_ptr, _stream_ptr(stream)), ctx)
+def ra_restore_queries(ctx, layer, q_ptr, scale=0.0, stream=None):
+    return _check(lib().ra_restore_queries(ctx, layer, q_ptr, float(scale), _stream_ptr(stream)), ctx)
 
 
 def ra_get_scores(ctx, layer, seq, kv_head, capacity, stream=None):

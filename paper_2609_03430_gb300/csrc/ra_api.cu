@@ -28,10 +28,6 @@ namespace {
 thread_local std::string g_tls_error = "no error";
 
 constexpr int kMaxSMs = 256;       // partial-buffer sizing bound (the GB300 has 152)
-#ifndef RA_ATTN_CHUNKS_PER_WARP
-#define RA_ATTN_CHUNKS_PER_WARP 1
-#endif
-constexpr int kChunksPerWarp = RA_ATTN_CHUNKS_PER_WARP;  // chunks per warp on average: room for stealing
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -55,13 +51,12 @@ struct ra_ctx {
     long long gen_rows = 0;
     int regions = 0;
     size_t partial_records = 0;  // split-K partial records the arena holds
-    unsigned long long ticket_base = 0;  // first chunk ticket of the next attention launch
     // arena layout (byte offsets)
-    size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_poff, off_plan, off_partial, off_arrive, off_ticket,
+    size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_poff, off_plan, off_partial, off_arrive,
         off_err, bytes;
     // scored policy: query window, scores and pass-1 statistics after the base arena
     bool scoring = false;
-    size_t base_bytes = 0, off_qring = 0, off_scores = 0, off_stats = 0;
+    size_t base_bytes = 0, off_qring = 0, off_qstats = 0, off_scores = 0, off_stats = 0;
     int stats_chunks = 0;
     // binding
     bool bound = false;
@@ -71,6 +66,7 @@ struct ra_ctx {
     DevLayout lay{};
     CUtensorMap tmap_k{}, tmap_v{};
     CUtensorMap tmap_ks{};  // kpool in kScoreTile-row boxes (scoring kernels)
+    CUtensorMap tmap_q{};   // the query windows as [L*B*KVH*r*G][128] rows, same boxes
     // host mirror
     std::vector<int32_t> g, c, nev;  // [L][B]
     std::vector<uint8_t> active;     // [B]
@@ -188,7 +184,7 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-int make_tmap(ra_ctx* ctx, CUtensorMap* map, void* base, int box_rows)
+int make_tmap(ra_ctx* ctx, CUtensorMap* map, void* base, long long rows, int box_rows)
 {
     static EncodeTiledFn encode = nullptr;
     if (!encode) {
@@ -199,7 +195,7 @@ int make_tmap(ra_ctx* ctx, CUtensorMap* map, void* base, int box_rows)
             return fail(ctx, RA_ERR_CUDA, "cuTensorMapEncodeTiled entry point not available");
         encode = reinterpret_cast<EncodeTiledFn>(fn);
     }
-    const cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)ctx->total_rows};
+    const cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)kRowBytes};
     // boxes of 64 channels (128 bytes) x box_rows rows, stored with the 128-byte swizzle
     const cuuint32_t box[2] = {(cuuint32_t)(kHeadDim / 2), (cuuint32_t)box_rows};
@@ -220,7 +216,8 @@ void fill_active(const ra_ctx* ctx, uint32_t* mask)
 
 // Work split of one layer's attention from the host mirror, in tiles: a head has
 // ceil(lp / TILE) prompt tiles and ceil(gen / TILE) tiles of generated rows, where gen is
-// the cached generated rows plus one for a fused new token.  *slots = rows attended.
+// the cached generated rows plus one for a fused new token; the tiles are cut into one equal
+// chunk per warp.  *slots = rows attended.
 int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots)
 {
     fill_active(ctx, p->active);
@@ -244,28 +241,18 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     p->total = (int)acc;
     const int wpc = attn_warps_per_cta(ctx->G);
     const long long nwarps_max = (long long)ctx->sms * wpc;
-    long long W = (acc + kChunksPerWarp * nwarps_max - 1) / (kChunksPerWarp * nwarps_max);
-    if (W < 1) W = 1;
-    p->W = (int)W;
+    const long long W = std::max<long long>(1, (acc + nwarps_max - 1) / nwarps_max);
     const long long nchunks = (acc + W - 1) / W;
+    p->W = (int)W;
     p->nchunks = (int)nchunks;
     *ctas = (int)std::min<long long>(ctx->sms, (nchunks + wpc - 1) / wpc);
     p->nwarps = *ctas * wpc;
-    if (nchunks <= p->nwarps) p->ticket = nullptr;  // every chunk has a warp of its own: no stealing
     *n_active = na;
     *slots = (double)rows;
     // partial records are indexed chunk + head: both bounded by what the arena holds
-    if ((size_t)nchunks + (size_t)ctx->B * ctx->KVH > ctx->partial_records)
+    if ((size_t)p->nchunks + (size_t)ctx->B * ctx->KVH > ctx->partial_records)
         return fail(ctx, RA_ERR_STATE, "attention split needs more partial records than the arena holds");
     return RA_OK;
-}
-
-// Chunk tickets one launch takes: every stolen chunk, plus one failed take per warp that ran.
-unsigned long long tickets_taken(const AttnParams& p)
-{
-    if (!p.ticket) return 0;
-    const long long stolen = std::max(0, p.nchunks - p.nwarps);
-    return (unsigned long long)(stolen + std::min(p.nchunks, p.nwarps));
 }
 
 // Arena size with (or without) the scored policy's buffers after the base layout.
@@ -280,6 +267,8 @@ void layout_scoring(ra_ctx* ctx)
     size_t o = ctx->base_bytes;
     ctx->off_qring = o;
     o = align_up(o + (size_t)ctx->L * heads * M * kRowBytes, kAlign);
+    ctx->off_qstats = o;
+    o = align_up(o + (size_t)ctx->L * heads * M * sizeof(float2), kAlign);
     ctx->off_scores = o;
     o = align_up(o + (size_t)ctx->L * heads * ctx->Cmax * sizeof(float), kAlign);
     ctx->off_stats = o;
@@ -287,63 +276,50 @@ void layout_scoring(ra_ctx* ctx)
     ctx->bytes = o;
 }
 
-// Launch shape of the two scoring passes of one eviction round, from the host mirror:
-// about two waves of CTAs (one per SM when the window needs more than half the shared
-// memory), each taking a run of consecutive tiles of one head.
-void plan_scoring(ra_ctx* ctx, EvictParams* p, double* bytes1, double* bytes2)
+// Launch shape of a scoring pass over the heads of the sequences in p (pass 1: prompt + the
+// trig_n cached rows each; pass 2: the trig_n candidate rows each): about two waves of CTAs
+// (one per SM when the window needs more than half the shared memory), each taking a run of
+// consecutive tiles of one head.  Returns the algorithmic bytes: the key rows read (every
+// one is contracted with the M = r * G window rows, so flops = bytes * M).
+double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
 {
-    const int r = ctx->r, M = r * ctx->G;
+    const int M = ctx->r * ctx->G;
     const int per_sm = score_row_tiles_per_warp(M) <= 2 ? 2 : 1;
-    long long w1 = 0, w2 = 0;
-    int max1 = 1, max2 = 1;
-    double rows1 = 0, rows2 = 0;
+    long long work = 0;
+    int most = 1;
+    double rows = 0;
     for (int i = 0; i < p->n_trig; ++i) {
-        const int b = p->trig[i], N = p->trig_n[i], lp = ctx->lp[b];
-        const int t1 = (lp + kScoreTile - 1) / kScoreTile + (N + r - 1 + kScoreTile - 1) / kScoreTile;
-        const int t2 = (N + kScoreTile - 1) / kScoreTile;
-        w1 += (long long)ctx->KVH * t1;
-        w2 += (long long)ctx->KVH * t2;
-        max1 = std::max(max1, t1);
-        max2 = std::max(max2, t2);
-        rows1 += (double)ctx->KVH * (lp + N + r - 1);
-        rows2 += (double)ctx->KVH * N;
-        ctx->score_n[(size_t)p->layer * ctx->B + b] = N;
+        const int lp = pass == 1 ? ctx->lp[p->trig[i]] : 0, n = p->trig_n[i];
+        const int t = (lp + kScoreTile - 1) / kScoreTile + (n + kScoreTile - 1) / kScoreTile;
+        work += (long long)ctx->KVH * t;
+        most = std::max(most, t);
+        rows += (double)ctx->KVH * (lp + n);
     }
     const long long target = (long long)ctx->sms * per_sm;
-    long long ch1 = std::max<long long>((w1 + target - 1) / target, (max1 + ctx->stats_chunks - 1) / ctx->stats_chunks);
-    long long ch2 = (w2 + target - 1) / target;
-    ch1 = std::max<long long>(ch1, 1);
-    ch2 = std::max<long long>(ch2, 1);
-    p->ch1 = (int)ch1;
-    p->ch2 = (int)ch2;
-    p->nch1 = (int)((max1 + ch1 - 1) / ch1);
-    p->nch2 = (int)((max2 + ch2 - 1) / ch2);
-    p->qk_scale_log2 = 1.4426950408889634f / sqrtf((float)kHeadDim);
-    // counted as the key rows read (the window, read once per CTA, is L2-resident): every key
-    // row costs 2 * M * 128 flops, so flops = bytes * M
-    *bytes1 = rows1 * kRowBytes;
-    *bytes2 = rows2 * kRowBytes;
+    long long ch = std::max<long long>((work + target - 1) / target, 1);
+    if (pass == 1) ch = std::max<long long>(ch, (most + ctx->stats_chunks - 1) / ctx->stats_chunks);
+    const int nch = (int)((most + ch - 1) / ch);
+    if (pass == 1) {
+        p->ch1 = (int)ch;
+        p->nch1 = nch;
+    } else {
+        p->ch2 = (int)ch;
+        p->nch2 = nch;
+    }
+    return rows * kRowBytes;
 }
 
 // One eviction round of the triggered sequences in p: [score passes,] select, compact.
 int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s)
 {
     cudaError_t e;
-    if (p.policy == RA_POLICY_SNAPKV) {
-        double b1 = 0, b2 = 0;
-        plan_scoring(ctx, &p, &b1, &b2);
-        {
-            ProfScope ps(ctx, RA_KERNEL_SCORE_STATS, b1, s);
-            e = launch_score(p, 1, &ctx->tmap_ks, s);
-            ps.done();
-        }
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "score pass 1 launch");
-        {
-            ProfScope ps(ctx, RA_KERNEL_SCORE_SUM, b2, s);
-            e = launch_score(p, 2, &ctx->tmap_ks, s);
-            ps.done();
-        }
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "score pass 2 launch");
+    if (p.policy == RA_POLICY_SNAPKV) {  // window scores with the normalisers recorded at decode time
+        for (int i = 0; i < p.n_trig; ++i) ctx->score_n[(size_t)p.layer * ctx->B + p.trig[i]] = p.trig_n[i];
+        const double bytes = plan_scoring(ctx, &p, 2);
+        ProfScope ps(ctx, RA_KERNEL_SCORE_SUM, bytes, s);
+        e = launch_score(p, 2, &ctx->tmap_ks, &ctx->tmap_q, s);
+        ps.done();
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
     }
     {
         ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
@@ -434,12 +410,11 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_lp = take((size_t)batch * 4);
     ctx->off_poff = take((size_t)batch * 4);
     ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
-    // chunks of the attention split: about kChunksPerWarp per warp (at least one tile each)
-    const size_t max_chunks = (size_t)kChunksPerWarp * kMaxSMs * attn_warps_per_cta(ctx->G) + 1;
+    // chunks of the attention split: one per warp
+    const size_t max_chunks = (size_t)kMaxSMs * attn_warps_per_cta(ctx->G) + 1;
     ctx->partial_records = max_chunks + (size_t)batch * kv_heads;
     ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);
-    ctx->off_ticket = take(sizeof(unsigned long long));
     ctx->off_err = take(256);
     ctx->base_bytes = o;
     int maxlp = 0;
@@ -499,9 +474,9 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.plan = (int32_t*)(a + ctx->off_plan);
     Ly.partial = (float*)(a + ctx->off_partial);
     Ly.arrive = (int32_t*)(a + ctx->off_arrive);
-    Ly.ticket = (unsigned long long*)(a + ctx->off_ticket);
     Ly.err = (int32_t*)(a + ctx->off_err);
     Ly.qring = ctx->scoring ? (uint16_t*)(a + ctx->off_qring) : nullptr;
+    Ly.qstats = ctx->scoring ? (float2*)(a + ctx->off_qstats) : nullptr;
     Ly.scores = ctx->scoring ? (float*)(a + ctx->off_scores) : nullptr;
     Ly.stats = ctx->scoring ? (float*)(a + ctx->off_stats) : nullptr;
     Ly.stats_chunks = ctx->stats_chunks;
@@ -529,8 +504,7 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
         (e = cudaMemcpyAsync(Ly.seq_lp, ctx->lp.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.seq_poff, ctx->poff.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess ||
-        (e = cudaMemsetAsync(Ly.ticket, 0, sizeof(unsigned long long), s)) != cudaSuccess)
+        (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess)
         return cuda_fail(ctx, e, "table initialisation");
     // rows that were never written (past a head's cached slots) then read as zeros, never as stale NaNs
     if ((e = cudaMemsetAsync(a, 0, ctx->off_pos, s)) != cudaSuccess) return cuda_fail(ctx, e, "cache clear");
@@ -541,15 +515,16 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
 
     const int tile = attn_tile_rows(ctx->G);
     int rc;
-    if ((rc = make_tmap(ctx, &ctx->tmap_k, Ly.kpool, tile)) != RA_OK) return rc;
-    if ((rc = make_tmap(ctx, &ctx->tmap_v, Ly.vpool, tile)) != RA_OK) return rc;
+    if ((rc = make_tmap(ctx, &ctx->tmap_k, Ly.kpool, ctx->total_rows, tile)) != RA_OK) return rc;
+    if ((rc = make_tmap(ctx, &ctx->tmap_v, Ly.vpool, ctx->total_rows, tile)) != RA_OK) return rc;
     if ((e = attn_prepare(ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
     if (ctx->scoring) {
-        if ((rc = make_tmap(ctx, &ctx->tmap_ks, Ly.kpool, kScoreTile)) != RA_OK) return rc;
+        if ((rc = make_tmap(ctx, &ctx->tmap_ks, Ly.kpool, ctx->total_rows, kScoreTile)) != RA_OK) return rc;
+        const long long win_rows = (long long)ctx->L * ctx->B * ctx->KVH * ctx->r * ctx->G;
+        if ((rc = make_tmap(ctx, &ctx->tmap_q, Ly.qring, win_rows, kScoreTile)) != RA_OK) return rc;
         if ((e = score_prepare()) != cudaSuccess) return cuda_fail(ctx, e, "score kernel attributes");
     }
 
-    ctx->ticket_base = 0;
     ctx->arena = a;
     ctx->device = dev;
     ctx->sms = sms;
@@ -627,6 +602,8 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block)
         if (ctx->r * ctx->G > kScoreMaxRows)
             return fail(ctx, RA_ERR_UNSUPPORTED, "scored policy needs r * G <= %d (have %d)", kScoreMaxRows,
                         ctx->r * ctx->G);
+        if (ctx->K + ctx->r > kScoreMaxCandidates)
+            return fail(ctx, RA_ERR_UNSUPPORTED, "scored policy needs K + r <= %d", kScoreMaxCandidates);
         ctx->scoring = true;
         layout_scoring(ctx);
     }
@@ -643,15 +620,45 @@ int ra_set_active(ra_ctx* ctx, int seq, int active)
     return RA_OK;
 }
 
-int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, void* stream)
+int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, float scale, void* stream)
 {
     int rc;
     if ((rc = check_bound(ctx)) != RA_OK) return rc;
     if ((rc = check_layer(ctx, layer)) != RA_OK) return rc;
     if (!ctx->scoring) return fail(ctx, RA_ERR_STATE, "context bound without the scored policy's query window");
     if (!q || !aligned16(q)) return fail(ctx, RA_ERR_INVALID_ARG, "q must be non-NULL and 16-byte aligned");
-    cudaError_t e = launch_restore_queries(ctx->lay, layer, q, ctx->g.data() + (size_t)layer * ctx->B, (cudaStream_t)stream);
-    return e == cudaSuccess ? RA_OK : cuda_fail(ctx, e, "query window restore launch");
+    cudaStream_t s = (cudaStream_t)stream;
+    const size_t base = (size_t)layer * ctx->B;
+    cudaError_t e = launch_restore_queries(ctx->lay, layer, q, ctx->g.data() + base, s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "query window restore launch");
+    // The normalisers of the loaded queries: each over the prompt and the cached rows at
+    // positions up to its own (what it attended to at its step, as no eviction can come between).
+    EvictParams p{};
+    p.lay = ctx->lay;
+    p.layer = layer;
+    int n = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (ctx->g[base + b] < 1) continue;
+        p.trig[n] = (int16_t)b;
+        p.trig_c[n] = ctx->c[base + b];
+        p.trig_n[n] = ctx->c[base + b];
+        p.trig_g[n] = ctx->g[base + b];
+        ++n;
+    }
+    if (n == 0) return RA_OK;
+    p.n_trig = n;
+    AttnParams sp{};
+    set_scale(&sp, scale);
+    p.qk_scale_log2 = sp.qk_scale_log2;
+    const double bytes = plan_scoring(ctx, &p, 1);
+    {
+        ProfScope ps(ctx, RA_KERNEL_SCORE_STATS, bytes, s);
+        e = launch_score(p, 1, &ctx->tmap_ks, &ctx->tmap_q, s);
+        ps.done();
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "window normaliser launch");
+    if ((e = launch_score_merge(p, s)) != cudaSuccess) return cuda_fail(ctx, e, "window normaliser merge launch");
+    return RA_OK;
 }
 
 int ra_append_kv(ra_ctx* ctx, int layer, const uint16_t* k_new, const uint16_t* v_new, void* stream)
@@ -745,8 +752,6 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     p.out = out;
     p.partial = ctx->lay.partial;
     p.arrive = ctx->lay.arrive;
-    p.ticket = ctx->lay.ticket;
-    p.ticket_base = ctx->ticket_base;
     p.qring = ctx->lay.qring;
     p.ring_off = -1;  // the step's token is already appended: its query is step g
     int n_active = 0;
@@ -760,7 +765,6 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     cudaError_t e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
-    if (p.total > 0) ctx->ticket_base += tickets_taken(p);
     return RA_OK;
 }
 
@@ -819,8 +823,6 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     p.v_new = v_new;
     p.partial = ctx->lay.partial;
     p.arrive = ctx->lay.arrive;
-    p.ticket = ctx->lay.ticket;
-    p.ticket_base = ctx->ticket_base;
     p.qring = ctx->lay.qring;
     p.ring_off = 0;  // the query of step g + 1
     int n_active = 0, ctas = 0;
@@ -833,7 +835,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     // this step (else it is this layer's compaction) and more than one layer (else it is this
     // layer's previous step).  Kernels let successors start only after their own wait, so
     // everything older than the predecessor has completed.
-    p.early = (n == 0 && ctx->L >= 2 && p.ticket == nullptr) ? 1 : 0;
+    p.early = (n == 0 && ctx->L >= 2) ? 1 : 0;
     {
         // rows read (the new token's from the caller), its row written, q read, out written
         ProfScope ps(ctx, RA_KERNEL_ATTN,
@@ -844,7 +846,6 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
         ps.done();
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
-    if (p.total > 0) ctx->ticket_base += tickets_taken(p);
     for (int b = 0; b < ctx->B; ++b) {
         if (!ctx->active[b]) continue;
         ctx->c[base + b] += 1;
@@ -1082,8 +1083,8 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
-    // [chunk ticket][arrival counters, one int per (seq, KV head)][partial records, one per (chunk, head) piece]
-    const size_t counters = align_up(sizeof(unsigned long long) + (size_t)ctx->B * ctx->KVH * sizeof(int32_t), kAlign);
+    // [arrival counters, one int per (seq, KV head)][partial records, one per (chunk, head) piece]
+    const size_t counters = align_up((size_t)ctx->B * ctx->KVH * sizeof(int32_t), kAlign);
     const size_t need =
         counters + (size_t)(p.nchunks + (long long)ctx->B * ctx->KVH) * partial_stride(ctx->G) * sizeof(float);
     if (need > kNoAllocScratchBytes)
@@ -1092,11 +1093,9 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     float* scratch = nullptr;
     if ((rc = noalloc_scratch(ctx, ctx->device, &scratch)) != RA_OK) return rc;
     cudaStream_t s = (cudaStream_t)stream;
-    p.ticket = reinterpret_cast<unsigned long long*>(scratch);
-    p.ticket_base = 0;
-    p.arrive = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(scratch) + sizeof(unsigned long long));
+    p.arrive = reinterpret_cast<int32_t*>(scratch);
     p.partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(scratch) + counters);
-    // the ticket and the counters must start at zero; the array keeps whatever the previous call left
+    // the counters must start at zero; the array keeps whatever the previous call left
     cudaError_t e = cudaMemsetAsync(scratch, 0, counters, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "scratch counter clear");
     e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);

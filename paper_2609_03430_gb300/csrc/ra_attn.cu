@@ -12,8 +12,7 @@
 // Work split: every head is cut into tiles of TILE rows (its prompt rows, then
 // its generated rows); the tiles of all heads of the layer are laid end to end
 // (sequence-major, then KV head) and cut into equal chunks of W tiles, one per
-// warp, so every warp makes the same number of pipeline trips.  (A warp may
-// steal further chunks from an atomic ticket when chunks outnumber warps.)  A
+// warp, so every warp makes the same number of pipeline trips.  A
 // warp runs its own pipeline: lane 0 streams the tiles of K and V -- each as
 // two 64-channel boxes stored with the 128-byte swizzle -- plus, at the first
 // tile of each head piece, the G query rows, into a ring of SPW shared-memory
@@ -25,7 +24,9 @@
 // a piece of that head (an arrival counter per head) merges all of them.
 //
 // With the scored comparator's buffers bound, the warp that consumes a head's
-// first tile also copies the head's G query rows into the query window.
+// first tile also copies the head's G query rows into the query window, and
+// whoever finishes a head records each query's softmax normaliser beside it:
+// until the next eviction, the window score needs exactly these normalisers.
 //
 // Per-warp compute: the contraction of the G query rows with a tile of cache
 // rows runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
@@ -98,8 +99,7 @@ constexpr int kFirst = 1, kLast = 2, kNewTok = 4, kHead0 = 8, kFlagBits = 4;
 
 // Producer-side walk over the warp's chunks (chunks and cursors count tiles).
 struct TileIter {
-    int chunk;                       // current chunk (-1: none yet)
-    unsigned long long next_ticket;  // lane 0: ticket taken ahead for the chunk after this one
+    int chunk;                       // this warp's chunk (-1: not started)
     int f, end;                      // flattened tile cursor and end of the current chunk
     int b, h, k;                     // current sequence, KV head, tile within the head
     int nt, tp;                      // tiles in the head, prompt tiles among them
@@ -149,30 +149,19 @@ __device__ void iter_init(TileIter& it, const AttnParams& p, int R0, int R1)
     enter_head(it, p);
 }
 
-// Next chunk of this warp: its own index first, then stolen ones; false when none is left.
-// Called by all lanes together (lane 0 takes the tickets).
-__device__ bool iter_next_chunk(TileIter& it, const AttnParams& p, int warp_id, int lane)
+// The warp's chunk (its index): false once it is done.
+__device__ bool iter_next_chunk(TileIter& it, const AttnParams& p, int warp_id)
 {
-    int c;
-    if (it.chunk < 0) {
-        c = warp_id;
-    } else {
-        if (!p.ticket) return false;  // every chunk has a warp of its own: nothing to steal
-        const unsigned long long raw = __shfl_sync(0xffffffffu, it.next_ticket, 0);
-        c = p.nwarps + (int)(raw - p.ticket_base);
-    }
-    if (c >= p.nchunks) return false;
-    // Take the ticket for the chunk after this one now: its latency hides behind this chunk's loads.
-    if (lane == 0 && p.ticket) it.next_ticket = atomicAdd(p.ticket, 1ull);
-    it.chunk = c;
-    const int R0 = c * p.W;
+    if (it.chunk >= 0 || warp_id >= p.nchunks) return false;
+    it.chunk = warp_id;
+    const int R0 = warp_id * p.W;
     iter_init(it, p, R0, min(p.total, R0 + p.W));
     return true;
 }
 
-__device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int warp_id, int lane)
+__device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int warp_id)
 {
-    if (it.f >= it.end && !iter_next_chunk(it, p, warp_id, lane)) return false;
+    if (it.f >= it.end && !iter_next_chunk(it, p, warp_id)) return false;
     const int T = p.tile;
     d.flags = (it.piece_start ? kFirst : 0) | (it.k == 0 ? kHead0 : 0);
     if (it.k < it.tp) {
@@ -246,57 +235,86 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi)) << 16);
 }
 
-// Merge every piece of head `hid` (pieces are partial records c0 + q + hid, q < P)
-// into the bf16 output rows of its G query heads.  One warp; lanes split as
-// (query head g, sub-lane).  The sub-lanes of a head load the statistics of up
-// to LG pieces at once and the O loads of those pieces are all independent, so
-// each group of LG pieces costs about one round of L2 latency.  Partials come
-// from other SMs: read through L2.
+// The scored policy's window: the softmax normaliser of query head g of (b, KV head h) at this
+// step, as (scale * log2 e, log2 sum_i exp2(scale * log2 e * q.k_i)), beside its query rows.
+template <int G>
+__device__ __forceinline__ void record_stats(const AttnParams& p, int b, int h, int g, float lse2)
+{
+    const int r = p.lay.r;
+    int slot = (p.seq_g[b] + p.ring_off) % r;
+    if (slot < 0) slot += r;
+    p.lay.qstats[((((size_t)p.layer * p.lay.B + b) * p.lay.KVH + h) * r + slot) * G + g] =
+        make_float2(p.qk_scale_log2, lse2);
+}
+
+// Merge every piece of head `hid` (pieces are partial records c0 + q + hid, q < P) into the
+// bf16 output rows of its G query heads.  One warp, two rounds of L2 reads: first every lane
+// reads the statistics of its pieces (lane q: piece q, q + 32, ...) and the warp reduces them
+// to each query head's max M and normaliser L; then lanes split as (query head g, channel
+// group), and for every piece load its max (one address per head: a broadcast) and their
+// channels together, so the loads of all pieces are independent.  Partials come from other
+// SMs: read through L2.
 template <int G>
 __device__ void merge_head(const AttnParams& p, int hid, int c0, int P, int lane)
 {
     using C = Cfg<G>;
-    const int g = lane / C::LG, sub = lane % C::LG;
-    const int gg = g < G ? g : 0;  // lanes of padding heads shadow head 0 (results unused)
-    const int ch0 = sub * C::MCH;
     const size_t rs = (size_t)partial_stride(G);
     const float* base = p.partial + (size_t)(c0 + hid) * rs;
-    float M = -INFINITY;
-    for (int q = sub; q < P; q += C::LG) M = fmaxf(M, __ldcg(base + q * rs + G * kHeadDim + gg));
+    float M[G], Lh[G];
 #pragma unroll
-    for (int o = 1; o < C::LG; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float Lsum = 0.f;
+    for (int g = 0; g < G; ++g) {
+        M[g] = -INFINITY;
+        Lh[g] = 0.f;
+    }
+    for (int q = lane; q < P; q += 32)
+#pragma unroll
+        for (int g = 0; g < G; ++g) M[g] = fmaxf(M[g], __ldcg(base + q * rs + G * kHeadDim + g));
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) M[g] = fmaxf(M[g], __shfl_xor_sync(0xffffffffu, M[g], o));
+    for (int q = lane; q < P; q += 32)
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            const float* st = base + q * rs + G * kHeadDim;
+            Lh[g] = fmaf(exp2f(__ldcg(st + g) - M[g]), __ldcg(st + G + g), Lh[g]);
+        }
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) Lh[g] += __shfl_xor_sync(0xffffffffu, Lh[g], o);
+
+    const int g = lane / C::LG, sub = lane % C::LG;
+    const int gg = g < G ? g : 0;  // lanes of padding heads shadow head 0 (results unused)
+    float Mg = M[0], Lg = Lh[0];
+#pragma unroll
+    for (int k = 1; k < G; ++k)
+        if (gg == k) {
+            Mg = M[k];
+            Lg = Lh[k];
+        }
+    const int ch0 = sub * C::MCH;
     float4 acc[C::MCH / 4];
 #pragma unroll
     for (int j = 0; j < C::MCH / 4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int q0 = 0; q0 < P; q0 += C::LG) {
-        float a = 0.f;
-        if (q0 + sub < P) {
-            const float* rec = base + (q0 + sub) * rs;
-            a = exp2f(__ldcg(rec + G * kHeadDim + gg) - M);
-            Lsum = fmaf(a, __ldcg(rec + G * kHeadDim + G + gg), Lsum);
-        }
+#pragma unroll 4
+    for (int q = 0; q < P; ++q) {
+        const float* rec = base + q * rs;
+        const float a = exp2f(__ldcg(rec + G * kHeadDim + gg) - Mg);
+        const float4* o = reinterpret_cast<const float4*>(rec + gg * kHeadDim + ch0);
 #pragma unroll
-        for (int j = 0; j < C::LG; ++j) {
-            const float aj = __shfl_sync(0xffffffffu, a, g * C::LG + j);
-            if (q0 + j < P) {
-                const float4* o = reinterpret_cast<const float4*>(base + (q0 + j) * rs + gg * kHeadDim + ch0);
-#pragma unroll
-                for (int k = 0; k < C::MCH / 4; ++k) {
-                    const float4 v = __ldcg(o + k);
-                    acc[k].x = fmaf(aj, v.x, acc[k].x);
-                    acc[k].y = fmaf(aj, v.y, acc[k].y);
-                    acc[k].z = fmaf(aj, v.z, acc[k].z);
-                    acc[k].w = fmaf(aj, v.w, acc[k].w);
-                }
-            }
+        for (int k = 0; k < C::MCH / 4; ++k) {
+            const float4 v = __ldcg(o + k);
+            acc[k].x = fmaf(a, v.x, acc[k].x);
+            acc[k].y = fmaf(a, v.y, acc[k].y);
+            acc[k].z = fmaf(a, v.z, acc[k].z);
+            acc[k].w = fmaf(a, v.w, acc[k].w);
         }
     }
-#pragma unroll
-    for (int o = 1; o < C::LG; o <<= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
     if (g >= G) return;
-    const float inv = 1.f / Lsum;
+    const float inv = 1.f / Lg;
     const int b = hid / p.lay.KVH, h = hid - b * p.lay.KVH;
+    if (p.qring && sub == 0) record_stats<G>(p, b, h, g, Mg + log2f(Lg));
     uint16_t* out = p.out + ((size_t)b * p.lay.H + (size_t)h * G + g) * kHeadDim + ch0;
 #pragma unroll
     for (int k = 0; k < C::MCH / 4; ++k) {
@@ -320,7 +338,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)C::NSTAGE * C::STAGE_BYTES + C::NSTAGE * 16) + warp * C::SPW;
 
     const int gw = blockIdx.x * C::WARPS + warp;
-    if (gw >= p.nchunks) {  // no chunk for this warp (it takes no ticket either)
+    if (gw >= p.nchunks) {  // no chunk for this warp
         pdl_wait();
         pdl_launch_dependents();
         return;
@@ -341,7 +359,6 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
 
     TileIter it;
     it.chunk = -1;
-    it.next_ticket = 0;
     it.f = it.end = 0;
     int issued = 0;
     // The caller's rows of a stage: the query rows (first tile of a piece), the new token's row.
@@ -360,7 +377,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
     };
     auto issue = [&](int t, bool inputs) -> bool {
         TileDesc d;
-        if (!iter_next(it, p, d, gw, lane)) return false;
+        if (!iter_next(it, p, d, gw)) return false;
         const int s = t % C::SPW;
         if (lane == 0) {
             uint8_t* st = wstage + (size_t)s * C::STAGE_BYTES;
@@ -504,6 +521,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             const int w0 = (int)(A / p.W), w1 = (int)((A + nth - 1) / p.W);
             if (w0 == w1) {  // the whole head was this warp's: normalise and write the output
                 if (gq < G) {
+                    if (p.qring && tq == 0) record_stats<G>(p, b, h, gq, m_run + log2f(l));
                     const float inv = 1.f / l;
                     uint32_t* out = reinterpret_cast<uint32_t*>(p.out + ((size_t)b * p.lay.H + (size_t)h * G + gq) * kHeadDim);
 #pragma unroll
@@ -538,7 +556,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
         }
 
         __syncwarp();
-        if (more) {  // refill the stage just consumed with the tile SPW ahead
+        if (more) {
             if (lane == 0) fence_proxy_async_smem();
             more = issue(t + C::SPW, true);
             if (more) ++issued;

@@ -80,8 +80,8 @@ constexpr int kSelThreads = 256;
 __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ EvictParams p)
 {
     extern __shared__ uint32_t sm[];
-    __shared__ uint32_t hist[256];
-    __shared__ uint32_t s_bin, s_before, s_total;
+    __shared__ uint32_t hist[3][256];
+    __shared__ uint32_t s_total;
     pdl_wait();
     pdl_launch_dependents();
     const DevLayout& L = p.lay;
@@ -105,6 +105,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     uint32_t* keys = sm;                 // [N]
     uint32_t* evbits = sm + nwords * 32; // [nwords]
 
+    if (tid < 256) hist[0][tid] = 0;  // the first digit's histogram (the fill's barrier publishes it)
     const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
     if (p.policy == RA_POLICY_RECENCY) {  // protected recency: the K newest candidates score lowest
         for (int j = tid; j < N; j += kSelThreads) keys[j] = (uint32_t)(N - 1 - j);
@@ -117,12 +118,16 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         // scored comparator: the window score max-pooled over +-kScorePoolRadius candidates;
         // larger scores must sort first, so the key is the order-reversed float
         const float* sc = L.scores + (((size_t)p.layer * L.B + b) * L.KVH + h) * L.Cmax;
+        float* raw = reinterpret_cast<float*>(evbits + nwords);  // [N], staged once
+#pragma unroll 4
+        for (int j = tid; j < N; j += kSelThreads) raw[j] = __ldcg(sc + j);
+        __syncthreads();
         for (int j = tid; j < N; j += kSelThreads) {
-            float m = __ldcg(sc + j);
+            float m = raw[j];
 #pragma unroll
             for (int d = 1; d <= kScorePoolRadius; ++d) {
-                if (j - d >= 0) m = fmaxf(m, __ldcg(sc + j - d));
-                if (j + d < N) m = fmaxf(m, __ldcg(sc + j + d));
+                if (j - d >= 0) m = fmaxf(m, raw[j - d]);
+                if (j + d < N) m = fmaxf(m, raw[j + d]);
             }
             const uint32_t u = __float_as_uint(m);
             const uint32_t asc = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // ascending with the float
@@ -138,46 +143,65 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     // Radix select of the element at rank K (0-based) of the (key, ordinal) order:
     // 8 bits at a time from the top.  Afterwards T is its key and `rank` is its
     // rank among the keys equal to T, i.e. the number of ties that are kept.
+    // One barrier per digit: every warp scans the histogram itself, and the
+    // histograms rotate over three buffers -- the one a pass fills was last read
+    // two passes earlier, before the previous barrier, so it is cleared
+    // (during the pass before) without a barrier of its own.
     uint32_t prefix = 0, mask = 0;
     uint32_t rank = (uint32_t)K;
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        hist[tid] = 0;
-        __syncthreads();
-        for (int j = tid; j < N; j += kSelThreads) {
-            const uint32_t kk = keys[j];
-            if ((kk & mask) == prefix) atomicAdd(&hist[(kk >> shift) & 255u], 1u);
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        uint32_t* H = hist[pass % 3];
+        if (tid < 256) hist[(pass + 1) % 3][tid] = 0;
+        // A warp whose in-prefix keys all share one bin (the common case for the scored
+        // policy's first digits, and once few keys remain) adds once; otherwise each lane adds.
+        for (int j0 = warp * 32; j0 < N; j0 += kSelThreads) {
+            const int j = j0 + lane;
+            const uint32_t kk = j < N ? keys[j] : 0u;
+            const bool in = j < N && (kk & mask) == prefix;
+            const uint32_t bin = (kk >> shift) & 255u;
+            const uint32_t inb = __ballot_sync(0xffffffffu, in);
+            if (inb == 0u) continue;
+            const int leader = __ffs(inb) - 1;
+            const uint32_t b0 = __shfl_sync(0xffffffffu, bin, leader);
+            if (__all_sync(0xffffffffu, !in || bin == b0)) {
+                if (lane == leader) atomicAdd(&H[b0], (uint32_t)__popc(inb));
+            } else if (in) {
+                atomicAdd(&H[bin], 1u);
+            }
         }
         __syncthreads();
-        if (warp == 0) {
-            uint32_t loc[8], sum = 0;
+        uint32_t loc[8], sum = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            loc[q] = H[lane * 8 + q];
+            sum += loc[q];
+        }
+        uint32_t incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += t;
+        }
+        const uint32_t excl = incl - sum;
+        uint32_t bin = 0, before = 0;
+        if (excl <= rank && rank < incl) {
+            uint32_t cum = excl;
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
-                loc[q] = hist[lane * 8 + q];
-                sum += loc[q];
-            }
-            uint32_t incl = sum;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += t;
-            }
-            const uint32_t excl = incl - sum;
-            if (excl <= rank && rank < incl) {
-                uint32_t cum = excl;
-#pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    if (rank < cum + loc[q]) {
-                        s_bin = (uint32_t)(lane * 8 + q);
-                        s_before = cum;
-                        break;
-                    }
-                    cum += loc[q];
+                if (rank < cum + loc[q]) {
+                    bin = (uint32_t)(lane * 8 + q);
+                    before = cum;
+                    break;
                 }
+                cum += loc[q];
             }
         }
-        __syncthreads();
-        rank -= s_before;
-        prefix |= s_bin << shift;
+        const int src = __ffs(__ballot_sync(0xffffffffu, excl <= rank && rank < incl)) - 1;
+        bin = __shfl_sync(0xffffffffu, bin, src);
+        before = __shfl_sync(0xffffffffu, before, src);
+        rank -= before;
+        prefix |= bin << shift;
         mask |= 255u << shift;
     }
     const uint32_t T = prefix;
@@ -388,12 +412,17 @@ cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s)
     return launch_pdl(append_kernel, dim3(B), dim3(p.lay.KVH * 32), 0, s, p);
 }
 
-static size_t select_smem(int N) { return ((size_t)((N + 31) / 32) * 32 + (N + 31) / 32) * sizeof(uint32_t); }
+// keys [N rounded to 32], the evicted bitmap, and under the scored policy the raw scores [N]
+static size_t select_smem(int N, bool scored)
+{
+    const size_t words = (size_t)(N + 31) / 32;
+    return (words * 32 + words + (scored ? words * 32 : 0)) * sizeof(uint32_t);
+}
 
 cudaError_t launch_select(const EvictParams& p, cudaStream_t s)
 {
     const int N = p.lay.K + p.lay.r;  // candidates at a firing step never exceed K + r
-    const size_t smem = select_smem(N);
+    const size_t smem = select_smem(N, p.policy == RA_POLICY_SNAPKV);
     static size_t configured = 0;
     if (smem > 48 * 1024 && smem > configured) {
         cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

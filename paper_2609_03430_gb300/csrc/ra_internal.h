@@ -35,12 +35,12 @@ struct DevLayout {
     int32_t* plan;         // [B*KVH][kPlanHeader + r] eviction plan of the current layer
     float* partial;        // attention split partials
     int32_t* arrive;       // [B*KVH] split-piece arrival counters
-    unsigned long long* ticket;  // attention chunk-stealing counter
     int32_t* err;          // device error word
     // scored policy (null when the context was bound without its buffers)
     uint16_t* qring;       // [L][B][KVH][r][G][128] bf16: query of step s in slot (s - 1) mod r
     float* scores;         // [L][B][KVH][Cmax] raw window score of each candidate of the latest round
-    float* stats;          // [B*KVH][stats_chunks][Mpad][2] pass-1 softmax statistics (max, sum) per chunk
+    float2* qstats;        // [L][B][KVH][r][G] per window query: (its scale * log2 e, log2 of its softmax sum)
+    float* stats;          // [B*KVH][stats_chunks][M][2] restore pass: softmax statistics (max, sum) per chunk
     int stats_chunks;      // chunks per head the stats buffer holds
     long long prompt_rows_per_layer;
     long long gen_row0;    // first row of the generated regions
@@ -71,12 +71,13 @@ struct EvictParams {
     int32_t trig_g[RA_MAX_BATCH];  // step of the draw: generated tokens including this step's
     // scored policy: tiles (of kScoreTile rows) per CTA of each pass, CTAs per head of each pass
     int ch1, ch2, nch1, nch2;
-    float qk_scale_log2;
+    float qk_scale_log2;  // restore pass: the scale * log2 e the restored queries are taken at
 };
 
 constexpr int kScoreTile = 64;      // key rows per scoring tile
 constexpr int kScoreMaxRows = 512;  // r * G window rows the scoring kernels hold
 constexpr int kScorePoolRadius = 3; // max-pool width 7 over neighbouring candidates
+constexpr int kScoreMaxCandidates = 16384;  // K + r bound of the scored policy (select stages the scores too)
 
 // Attention work is counted in tiles of TILE rows: a head has ceil(lp / TILE) prompt tiles and
 // ceil(gen / TILE) tiles of generated rows (gen includes a fused new token, its last row).
@@ -90,12 +91,10 @@ struct AttnParams {
     const uint16_t* v_new;
     float* partial;         // split-K partial records (arena or the no-alloc array)
     int32_t* arrive;        // [B*KVH] pieces merged so far per head; zero between launches
-    int W;                  // tiles per chunk of the split (a warp's first chunk is its index, later ones are stolen)
+    int W;                  // tiles per chunk of the split: warp w takes tiles [w W, (w + 1) W)
     int total;              // total tiles of the layer
     int nchunks;            // ceil(total / W)
     int nwarps;             // warps launched
-    unsigned long long* ticket;  // chunk-stealing counter (never reset: this launch's tickets start at ticket_base)
-    unsigned long long ticket_base;
     float qk_scale_log2;    // scale * log2(e)
     int early;              // 1: the first tiles' K/V may be loaded before the predecessor kernel finishes
     uint32_t active[RA_MAX_BATCH / 32];
@@ -125,9 +124,13 @@ cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s);
 cudaError_t launch_restore_queries(const DevLayout& lay, int layer, const uint16_t* q, const int32_t* g_dev,
                                    cudaStream_t s);
 
-// Scored policy: pass 1 (softmax statistics) or pass 2 (per-candidate sums) of the window attention.
-// The tensor map covers kpool as [total_rows][128] bf16 with boxes of kScoreTile rows x 64 channels.
-cudaError_t launch_score(const EvictParams& p, int pass, const CUtensorMap* tmap_k, cudaStream_t s);
+// Scored policy: pass 1 (restore: softmax statistics of a loaded window, then launch_score_merge)
+// or pass 2 (eviction: per-candidate sums with the recorded normalisers).
+// The tensor maps cover kpool as [total_rows][128] bf16 and the query windows as
+// [L*B*KVH*r*G][128] bf16, both with boxes of kScoreTile rows x 64 channels.
+cudaError_t launch_score(const EvictParams& p, int pass, const CUtensorMap* tmap_k, const CUtensorMap* tmap_q,
+                         cudaStream_t s);
+cudaError_t launch_score_merge(const EvictParams& p, cudaStream_t s);
 cudaError_t score_prepare();
 int score_row_tiles_per_warp(int M);  // 16-row tiles of the M window rows per warp (1..4)
 

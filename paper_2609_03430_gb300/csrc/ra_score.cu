@@ -4,27 +4,31 @@
 // section 2 ("Baselines as choices of s"): the attention that the window of
 // the last r decode queries gives each candidate, summed over the window and
 // over the G query heads of the KV group (max-pooling and top-K happen in the
-// select kernel).  A window query of step s attends, like the decode step it
-// came from, to the keys at positions up to its own: the prompt, every
-// candidate, and the first u buffer rows, u = its rank in the window.
+// select kernel).  A window query attends, as at its own decode step, to the
+// keys at positions up to its own: the prompt, every candidate, and the first
+// u buffer rows, u = its rank in the window.
 //
-// Per triggered (sequence, KV head) the window is M = r * G query rows.  The
-// contraction of those rows with every key row is a dense GEMM (M x keys x 128),
-// so it runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
-//   pass 1 (score_kernel<1, MT>)  per row, the running max and sum of exp of
-//       the scaled logits over the keys it sees, over one chunk of key tiles;
-//       one (max, sum) pair per row and chunk goes to the statistics buffer.
-//   pass 2 (score_kernel<2, MT>)  merges a head's chunk statistics, recomputes
-//       the logits of the candidate tiles, normalises them and sums the weights
-//       over all M rows: one fp32 score per candidate.  Each CTA holds all M
-//       rows, so every column sum is complete inside it -- no atomics, and the
-//       result does not depend on the launch shape.
-// CTA layout: 8 warps; warp w owns the 16-row M tiles w, w + 8, ... (MT of
-// them).  The M rows sit in shared memory with a 16-byte-chunk xor swizzle and
-// are read as A fragments with ldmatrix; key tiles of 64 rows x 128 channels
-// arrive by 2-D TMA (two 64-channel boxes, 128-byte swizzle) into a two-stage
-// ring on mbarriers, and are read as B fragments with ldmatrix.  Logits are in
-// base 2 with the scale folded into one multiply.
+// Between two eviction rounds the cache only grows, so each window query saw
+// at its own step exactly the keys it sees now, and the decode attention
+// kernel records its softmax normaliser beside it.  The eviction therefore
+// needs one pass over the candidate rows only:
+//   summation pass (score_kernel<2, MT>)  per triggered (sequence, KV head),
+//       the logits of the M = r * G window rows against the candidate tiles,
+//       normalised by the recorded normalisers and summed over all M rows:
+//       one fp32 score per candidate.  Each CTA holds all M rows, so every
+//       column sum is complete inside it -- no atomics, and the result does
+//       not depend on the launch shape.
+//   restore pass (score_kernel<1, MT> + score_merge_kernel)  only when a
+//       window is loaded from outside (ra_restore_queries): the normalisers,
+//       recomputed over the prompt and the cached rows each query sees (by
+//       position), split over chunks of key tiles and merged.
+// The contraction of the window rows with the key rows is a dense GEMM
+// (M x keys x 128), so it runs on the tensor cores (mma.sync m16n8k16, bf16
+// in, fp32 accumulate).  CTA layout: 8 warps; warp w owns the 16-row M tiles
+// w, w + 8, ... (MT of them).  The M rows arrive by 2-D TMA (64-row x
+// 64-channel boxes, 128-byte swizzle) with the first key tile and are read as
+// A fragments with ldmatrix; key tiles of 64 rows x 128 channels arrive the
+// same way into a two-stage ring on mbarriers and are read as B fragments.  Logits are in base 2 with the scale folded in.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -48,18 +52,23 @@ static_assert(kHalfBytes % 1024 == 0, "128-byte-swizzled TMA boxes start 1024-by
 template <int MT>
 struct SCfg {
     static constexpr int ROWS = 16 * kWarps * MT;                 // window rows held (M padded)
+    static constexpr int Q_HALF = ROWS * 128;                     // one 64-channel half of the window
     static constexpr int Q_OFF = kStages * kTileBytes;            // after the key stages
     static constexpr int STAT_OFF = Q_OFF + ROWS * kRowBytes;     // pass 2: row max and 1/sum
     static constexpr int RED_OFF = STAT_OFF + 2 * ROWS * 4;       // pass 2: column sums per warp
     static constexpr int BAR_OFF = RED_OFF + kWarps * kScoreTile * 4;
     static constexpr size_t SMEM = 1024 + (size_t)BAR_OFF + kStages * 8;
     static_assert(ROWS <= kScoreMaxRows || MT == 1, "window rows");
+    static_assert(ROWS % kScoreTile == 0 && Q_HALF % 1024 == 0, "whole TMA boxes, 1024-byte aligned");
     static_assert(SMEM <= 232448, "fits the 227 KB opt-in shared memory");
 };
 
-// Byte offset of (window row R, 16-byte chunk c) of the M x 128 query block:
-// chunks are xored with R mod 8 within each 128-byte half of a row.
-__device__ __forceinline__ uint32_t qswz(int R, int c) { return (uint32_t)(R * kRowBytes + ((c & 8) | ((c ^ R) & 7)) * 16); }
+// Byte offset of (window row R, 16-byte chunk c) of the window block: two 64-channel halves of
+// `half` bytes each, rows of 128 bytes, chunks xored with R mod 8 (the TMA 128-byte swizzle).
+__device__ __forceinline__ uint32_t qswz(int R, int c, int half)
+{
+    return (uint32_t)((c >> 3) * half + R * 128 + (((c & 7) ^ (R & 7)) << 4));
+}
 
 // Byte offset of (key row j, 16-byte chunk c) inside a 128-byte-swizzled key tile.
 __device__ __forceinline__ uint32_t kswz(int j, int c)
@@ -84,28 +93,44 @@ __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], 
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-// Tiles of one head in pass 1: its prompt rows, then its generated rows up to the
-// newest any window query sees (ordinal N + r - 2); in pass 2: the candidate rows.
-__device__ __forceinline__ int head_tiles(int pass, int lp, int N, int r, int* tp)
+// Tiles of one head: restore pass -- its prompt rows, then its c cached generated rows;
+// summation pass -- its N candidate rows.
+__device__ __forceinline__ int head_tiles(int pass, int lp, int n_gen, int* tp)
 {
-    if (pass == 2) {
-        *tp = 0;
-        return (N + kScoreTile - 1) / kScoreTile;
-    }
-    *tp = (lp + kScoreTile - 1) / kScoreTile;
-    return *tp + (N + r - 1 + kScoreTile - 1) / kScoreTile;
+    *tp = pass == 1 ? (lp + kScoreTile - 1) / kScoreTile : 0;
+    return *tp + (n_gen + kScoreTile - 1) / kScoreTile;
 }
 
+// Restore pass: the decode step whose query sits in window slot `slot` when g tokens have been
+// generated (the r latest steps fill the r slots), and how many of the head's c cached generated
+// rows (positions pos[0..c), increasing) that query sees: those at positions up to its own.
+__device__ __forceinline__ int visible_rows(const int32_t* pos, int c, int lp, int g, int r, int slot)
+{
+    const int d = ((g - 1 - slot) % r + r) % r;
+    const int step = g - d;
+    if (step < 1) return 0;  // no such step yet: the slot is never read before a real query fills it
+    const int qpos = lp + step - 1;
+    int lo = 0, hi = c;      // first ordinal whose position is after qpos
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldcg(pos + mid) <= qpos) lo = mid + 1; else hi = mid;
+    }
+    return lo;
+}
+
+// PASS 1 (restore): per window row, (max, sum of exp2) over one chunk of the keys it sees.
+// PASS 2 (eviction): per candidate, the sum over window rows of exp2(logit - log2 normaliser).
 template <int PASS, int MT>
 __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const __grid_constant__ EvictParams p,
-                                                            const __grid_constant__ CUtensorMap tk)
+                                                                        const __grid_constant__ CUtensorMap tk,
+                                                                        const __grid_constant__ CUtensorMap tw)
 {
     using C = SCfg<MT>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::BAR_OFF);
-    float* s_m = reinterpret_cast<float*>(smem + C::STAT_OFF);
-    float* s_il = s_m + C::ROWS;
+    float* s_sl = reinterpret_cast<float*>(smem + C::STAT_OFF);  // pass 2: each row's scale * log2 e
+    float* s_lse = s_sl + C::ROWS;                               // pass 2: each row's log2 normaliser
     float* red = reinterpret_cast<float*>(smem + C::RED_OFF);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -118,24 +143,27 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
     const int N = p.trig_n[t], r = L.r, G = L.G, M = r * G;
     const int lp = L.seq_lp[b];
     int tp;
-    const int nt_head = head_tiles(PASS, lp, N, r, &tp);
+    const int nt_head = head_tiles(PASS, lp, N, &tp);
     const int ch = PASS == 1 ? p.ch1 : p.ch2;
     const int t0 = blockIdx.x * ch;
     if (t0 >= nt_head) return;
     const int ntile = min(ch, nt_head - t0);
     const long long prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[b] + (long long)h * lp;
-    const int reg = L.region[((size_t)p.layer * L.B + b) * L.KVH + h];
+    const size_t lbh = ((size_t)p.layer * L.B + b) * L.KVH + h;
+    const int reg = L.region[lbh];
     const long long grow = L.gen_row0 + (long long)reg * L.Cmax;
     const int hid = b * L.KVH + h;
 
     auto tile_row = [&](int k) -> long long {  // first cache row of the head's tile k
         return k < tp ? prow + (long long)k * kScoreTile : grow + (long long)(k - tp) * kScoreTile;
     };
-    auto issue = [&](int i) {  // thread 0: tile t0 + i into stage i % 2
+    // thread 0: tile t0 + i into stage i % 2 (one arrival per phase: `extra` bytes of other copies
+    // completing on the same barrier are expected together with the tile)
+    auto issue = [&](int i, uint32_t extra) {
         const int s = i % kStages;
         uint8_t* st = smem + (size_t)s * kTileBytes;
         const int row = (int)tile_row(t0 + i);
-        mbar_arrive_expect_tx(&bars[s], (uint32_t)kTileBytes);
+        mbar_arrive_expect_tx(&bars[s], (uint32_t)kTileBytes + extra);
         tma_load_2d(st, &tk, 0, row, &bars[s]);
         tma_load_2d(st + kHalfBytes, &tk, 64, row, &bars[s]);
     };
@@ -143,34 +171,24 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
         for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
         fence_mbar_init();
         prefetch_tensormap(&tk);
-        for (int i = 0; i < kStages && i < ntile; ++i) issue(i);
+        prefetch_tensormap(&tw);
+        // The window rows (row R = slot * G + g) complete on stage 0's barrier with the first
+        // key tile.  Rows past M belong to the next head's window (or lie past the end and
+        // read as zero): finite, and given no weight.
+        issue(0, (uint32_t)(C::ROWS * kRowBytes));
+        const int row0 = (int)(lbh * (size_t)M);
+        for (int rb = 0; rb < C::ROWS; rb += kScoreTile) {
+            tma_load_2d(smem + C::Q_OFF + rb * 128, &tw, 0, row0 + rb, &bars[0]);
+            tma_load_2d(smem + C::Q_OFF + C::Q_HALF + rb * 128, &tw, 64, row0 + rb, &bars[0]);
+        }
+        for (int i = 1; i < kStages && i < ntile; ++i) issue(i, 0u);
     }
-
-    // The window rows (row R = slot * G + g), zero past M.
-    const uint16_t* win = L.qring + (((size_t)p.layer * L.B + b) * L.KVH + h) * (size_t)M * kHeadDim;
-    for (int i = tid; i < C::ROWS * 16; i += kThreads) {
-        const int R = i >> 4, c = i & 15;
-        const uint4 v = R < M ? __ldcg(reinterpret_cast<const uint4*>(win) + i) : make_uint4(0u, 0u, 0u, 0u);
-        *reinterpret_cast<uint4*>(smem + C::Q_OFF + qswz(R, c)) = v;
-    }
-    float* stats = L.stats + (size_t)hid * L.stats_chunks * M * 2;
-    if (PASS == 2) {  // merge the chunk statistics of pass 1 into each row's max and 1/sum
-        int tp1;
-        const int nch = (head_tiles(1, lp, N, r, &tp1) + p.ch1 - 1) / p.ch1;
+    if (PASS == 2) {  // the normaliser each window query had at its decode step
+        const float2* qst = L.qstats + lbh * (size_t)M;
         for (int R = tid; R < C::ROWS; R += kThreads) {
-            float mx = 0.f, il = 0.f;
-            if (R < M) {
-                mx = -INFINITY;
-                for (int k = 0; k < nch; ++k) mx = fmaxf(mx, __ldcg(stats + ((size_t)k * M + R) * 2));
-                float sum = 0.f;
-                for (int k = 0; k < nch; ++k) {
-                    const float mk = __ldcg(stats + ((size_t)k * M + R) * 2);
-                    if (mk != -INFINITY) sum += __ldcg(stats + ((size_t)k * M + R) * 2 + 1) * exp2f(mk - mx);
-                }
-                il = 1.f / sum;
-            }
-            s_m[R] = mx;
-            s_il[R] = il;
+            const float2 f = R < M ? __ldcg(qst + R) : make_float2(0.f, INFINITY);  // padding rows weigh 0
+            s_sl[R] = f.x;
+            s_lse[R] = f.y;
         }
     }
     __syncthreads();
@@ -178,26 +196,27 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
     // This lane's rows: R = 16 * (warp + 8 i) + (lane / 4) + 8 hf; its columns: 8 nt + 2 (lane % 4) + e.
     const int tq = lane & 3;
     const int mi = lane >> 3, ri = lane & 7;
-    const float sl = p.qk_scale_log2;
-    int lim[MT][2];  // pass 1: generated ordinals this row sees (N + its rank in the window)
-    // pass 1: running max and (per-lane partial) sum of exp2; pass 2: the row's max and 1/sum
+    int lim[MT][2];  // pass 1: generated rows the row sees
+    // pass 1: running max and (per-lane partial) sum of exp2; pass 2: the row's scale and normaliser
     float mrow[MT][2], lrow[MT][2];
 #pragma unroll
     for (int i = 0; i < MT; ++i)
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
             const int R = 16 * (warp + kWarps * i) + (lane >> 2) + 8 * hf;
-            lim[i][hf] = N + ((R / G) + 1) % r;
             if (PASS == 1) {
+                lim[i][hf] = R < M ? visible_rows(L.pos + (size_t)reg * L.Cmax, N, lp, p.trig_g[t], r, R / G) : 0;
                 mrow[i][hf] = -INFINITY;
                 lrow[i][hf] = 0.f;
             } else {
-                mrow[i][hf] = s_m[R];
-                lrow[i][hf] = s_il[R];
+                lim[i][hf] = 0;
+                mrow[i][hf] = s_sl[R];
+                lrow[i][hf] = s_lse[R];
             }
         }
+    const float sl = p.qk_scale_log2;  // pass 1: the scale the restored queries are taken at
     const uint32_t qs = smem_u32(smem + C::Q_OFF);
-    float* scores = L.scores + (((size_t)p.layer * L.B + b) * L.KVH + h) * L.Cmax;
+    float* scores = L.scores + lbh * L.Cmax;
 
     for (int i = 0; i < ntile; ++i) {
         const int s = i % kStages;
@@ -220,7 +239,8 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
         for (int kk = 0; kk < 8; ++kk) {
             uint32_t af[MT][4];
 #pragma unroll
-            for (int a = 0; a < MT; ++a) ldsm_x4(af[a], qs + qswz(16 * (warp + kWarps * a) + (lane & 15), 2 * kk + (lane >> 4)));
+            for (int a = 0; a < MT; ++a)
+                ldsm_x4(af[a], qs + qswz(16 * (warp + kWarps * a) + (lane & 15), 2 * kk + (lane >> 4), C::Q_HALF));
 #pragma unroll
             for (int np = 0; np < 4; ++np) {
                 uint32_t bf[4];
@@ -276,7 +296,7 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
                     for (int n = 0; n < 8; ++n)
 #pragma unroll
                         for (int e = 0; e < 2; ++e)
-                            cs[n][e] += exp2f(acc[a][n][2 * hf + e] * sl - mrow[a][hf]) * lrow[a][hf];
+                            cs[n][e] += exp2f(fmaf(acc[a][n][2 * hf + e], mrow[a][hf], -lrow[a][hf]));
 #pragma unroll
             for (int n = 0; n < 8; ++n)
 #pragma unroll
@@ -299,12 +319,12 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
         __syncthreads();  // stage s (and the column-sum buffer) free again
         if (tid == 0 && i + kStages < ntile) {
             fence_proxy_async_smem();
-            issue(i + kStages);
+            issue(i + kStages, 0u);
         }
     }
 
     if (PASS == 1) {  // this chunk's statistics of every real row
-        float* out = stats + (size_t)blockIdx.x * M * 2;
+        float* out = L.stats + ((size_t)hid * L.stats_chunks + blockIdx.x) * M * 2;
 #pragma unroll
         for (int a = 0; a < MT; ++a)
 #pragma unroll
@@ -318,11 +338,37 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
     }
 }
 
+// Restore pass, last step: merge each window row's chunk statistics into its normaliser.
+__global__ void __launch_bounds__(256) score_merge_kernel(const __grid_constant__ EvictParams p)
+{
+    pdl_wait();
+    pdl_launch_dependents();
+    const DevLayout& L = p.lay;
+    const int t = blockIdx.x / L.KVH, h = blockIdx.x - t * L.KVH;
+    const int b = p.trig[t];
+    const int M = L.r * L.G;
+    int tp;
+    const int nch = (head_tiles(1, L.seq_lp[b], p.trig_n[t], &tp) + p.ch1 - 1) / p.ch1;
+    const float* st = L.stats + (size_t)(b * L.KVH + h) * L.stats_chunks * M * 2;
+    float2* qst = L.qstats + (((size_t)p.layer * L.B + b) * L.KVH + h) * (size_t)M;
+    for (int R = threadIdx.x; R < M; R += blockDim.x) {
+        float mx = -INFINITY;
+        for (int k = 0; k < nch; ++k) mx = fmaxf(mx, st[((size_t)k * M + R) * 2]);
+        float sum = 0.f;
+        if (mx != -INFINITY)
+            for (int k = 0; k < nch; ++k) {
+                const float mk = st[((size_t)k * M + R) * 2];
+                if (mk != -INFINITY) sum += st[((size_t)k * M + R) * 2 + 1] * exp2f(mk - mx);
+            }
+        qst[R] = make_float2(p.qk_scale_log2, mx + log2f(sum));
+    }
+}
+
 template <int PASS, int MT>
-cudaError_t launch_mt(const EvictParams& p, const CUtensorMap* tk, cudaStream_t s)
+cudaError_t launch_mt(const EvictParams& p, const CUtensorMap* tk, const CUtensorMap* tq, cudaStream_t s)
 {
     const dim3 grid(PASS == 1 ? p.nch1 : p.nch2, p.n_trig * p.lay.KVH);
-    return launch_pdl(score_kernel<PASS, MT>, grid, dim3(kThreads), SCfg<MT>::SMEM, s, p, *tk);
+    return launch_pdl(score_kernel<PASS, MT>, grid, dim3(kThreads), SCfg<MT>::SMEM, s, p, *tk, *tq);
 }
 
 template <int MT>
@@ -346,22 +392,27 @@ cudaError_t score_prepare()
     return prepare_mt<4>();
 }
 
-cudaError_t launch_score(const EvictParams& p, int pass, const CUtensorMap* tk, cudaStream_t s)
+cudaError_t launch_score_merge(const EvictParams& p, cudaStream_t s)
+{
+    return launch_pdl(score_merge_kernel, dim3(p.n_trig * p.lay.KVH), dim3(256), 0, s, p);
+}
+
+cudaError_t launch_score(const EvictParams& p, int pass, const CUtensorMap* tk, const CUtensorMap* tq, cudaStream_t s)
 {
     const int MT = score_row_tiles_per_warp(p.lay.r * p.lay.G);
     if (pass == 1) {
         switch (MT) {
-            case 1: return launch_mt<1, 1>(p, tk, s);
-            case 2: return launch_mt<1, 2>(p, tk, s);
-            case 3: return launch_mt<1, 3>(p, tk, s);
-            case 4: return launch_mt<1, 4>(p, tk, s);
+            case 1: return launch_mt<1, 1>(p, tk, tq, s);
+            case 2: return launch_mt<1, 2>(p, tk, tq, s);
+            case 3: return launch_mt<1, 3>(p, tk, tq, s);
+            case 4: return launch_mt<1, 4>(p, tk, tq, s);
         }
     } else {
         switch (MT) {
-            case 1: return launch_mt<2, 1>(p, tk, s);
-            case 2: return launch_mt<2, 2>(p, tk, s);
-            case 3: return launch_mt<2, 3>(p, tk, s);
-            case 4: return launch_mt<2, 4>(p, tk, s);
+            case 1: return launch_mt<2, 1>(p, tk, tq, s);
+            case 2: return launch_mt<2, 2>(p, tk, tq, s);
+            case 3: return launch_mt<2, 3>(p, tk, tq, s);
+            case 4: return launch_mt<2, 4>(p, tk, tq, s);
         }
     }
     return cudaErrorInvalidValue;

@@ -76,6 +76,7 @@ class Runner:
         self.orc = oracle.OracleCache(L, KVH, self.lp, K, r, eseed, policy=policy, block=block)
         self.policy = policy
         self.qsteps = [[] for _ in range(self.B)]  # step index of each of a sequence's decode steps
+        self.step_scale = []  # attention scale of every step (the window's weights use it)
         self.scored_rounds = 0
         self.near_ties = 0
         self.dev = torch.device("cuda")
@@ -116,6 +117,7 @@ class Runner:
         for b in range(self.B):
             if self.active[b]:
                 self.qsteps[b].append(self.step_idx)
+        self.step_scale.append(scale)
         scored = self.policy == oracle.POLICY_SNAPKV
         for l in range(self.L):
             k = np.zeros((self.B, self.KVH, self.D), np.uint16)
@@ -166,7 +168,9 @@ class Runner:
         g, n = int(self.orc.g[b, l]), cur.size - self.r
         q, qpos = self.window(l, b, h, g)
         kpos = self.orc.positions(b, l, h)
-        ref = oracle.window_scores(q, qpos, self.krows(l, b, h, kpos), kpos)[self.lp[b]:self.lp[b] + n]
+        scales = {self.step_scale[self.qsteps[b][s - 1]] for s in range(g - self.r, g)}
+        assert len(scales) == 1, "one attention scale per window"
+        ref = oracle.window_scores(q, qpos, self.krows(l, b, h, kpos), kpos, scales.pop())[self.lp[b]:self.lp[b] + n]
         got = self.ra.ra_get_scores(self.ctx, l, b, h, self.K + 2 * self.r)
         what = f"scores l{l} b{b} h{h} g{g}"
         check_scores(got, ref, what)

@@ -97,7 +97,7 @@ def test_scored_policy_sizes_its_buffers_before_bind(ra):
         ra.ra_set_policy(big, ra.RA_POLICY_SNAPKV)
     assert e.value.code == ra.RA_ERR_UNSUPPORTED
     lib = ra.lib()
-    assert lib.ra_restore_queries(big, 0, None, None) == ra.RA_ERR_STATE  # unbound
+    assert lib.ra_restore_queries(big, 0, None, ctypes.c_float(0), None) == ra.RA_ERR_STATE  # unbound
     n = ctypes.c_int(0)
     assert lib.ra_get_scores(big, 0, 0, 0, None, 0, ctypes.byref(n), None) == ra.RA_ERR_STATE
     ra.ra_destroy(big)
