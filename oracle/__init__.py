@@ -15,6 +15,8 @@ Paper sections followed (Random Attention, arXiv 2609.03430):
     K+r; keep-sets sorted chronologically; GQA query groups share their KV
     head's keep-set; keys stored post-RoPE (so attention applies no rotation);
   * section 2 "Notation" -- o_t = sum_i softmax_i(q.k_i/sqrt(d)) v_i;
+  * Appendix G (a keep-set is a random permutation of slot indices) -- the
+    order-free hole-filling compaction, keys drawn per position;
   * section 2 "Baselines as choices of s" -- the SnapKV window score of the
     scored comparator (window attention, max-pooled, top-K, prompt pinned).
 
@@ -78,6 +80,14 @@ def _load():
                                               ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, i32p]
         lib.ora_evict_head_policy.restype = ctypes.c_int
         lib.ora_attend.restype = None
+        lib.ora_position_key.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_uint32,
+                                         ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int32,
+                                         ctypes.c_int32]
+        lib.ora_position_key.restype = ctypes.c_uint32
+        lib.ora_evict_head_holefill.argtypes = [i32p, ctypes.POINTER(ctypes.c_int), ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, i32p]
+        lib.ora_evict_head_holefill.restype = ctypes.c_int
         lib.ora_window_scores.argtypes = [u16p, i32p, ctypes.c_int, ctypes.c_int, u16p, i32p, ctypes.c_int,
                                           ctypes.c_int, ctypes.c_double, f64p]
         lib.ora_window_scores.restype = None
@@ -177,6 +187,28 @@ def attend(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float = 0.0) -> n
     return out
 
 
+COMPACT_ORDERED, COMPACT_HOLEFILL = 0, 1
+
+
+def position_key(policy, seed, layer, seq, kv_heads, h, step, position, block=1) -> int:
+    """Policy score of the candidate at `position` when slots carry no order."""
+    return int(_load().ora_position_key(policy, seed, layer, seq, kv_heads, h, step, position, block))
+
+
+def evict_head_holefill(gen, g, K, r, seed, layer, seq, kv_heads, h, policy=POLICY_RANDOM, block=1):
+    """One eviction round with hole-filling compaction; returns (new_gen, evicted_ordinals)."""
+    buf = np.ascontiguousarray(gen, dtype=np.int32).copy()
+    c = ctypes.c_int(int(buf.size))
+    ev = np.zeros(max(int(buf.size), 1), dtype=np.int32)
+    if buf.size == 0:
+        return buf, ev[:0]
+    m = _load().ora_evict_head_holefill(_ptr(buf, ctypes.c_int32), ctypes.byref(c), g, K, r, seed, layer, seq,
+                                        kv_heads, h, policy, block, _ptr(ev, ctypes.c_int32))
+    if m < 0:
+        raise RuntimeError("ora_evict_head_holefill failed")
+    return buf[: c.value].copy(), ev[:m].copy()
+
+
 def window_scores(q: np.ndarray, q_pos, k: np.ndarray, k_pos, scale: float = 0.0) -> np.ndarray:
     """SnapKV window score of every key (section 2): attention from the window queries
     q [n_q][G][d] (bf16 bits) at positions q_pos, summed over queries and heads, each
@@ -248,7 +280,7 @@ class OracleCache:
     fix the order within a step).
     """
 
-    def __init__(self, layers, kv_heads, prompt_lens, K, r, seed, heads=None, policy=0, block=1):
+    def __init__(self, layers, kv_heads, prompt_lens, K, r, seed, heads=None, policy=0, block=1, compaction=0):
         self.L = layers
         self.KVH = kv_heads
         self.prompt_lens = [int(x) for x in prompt_lens]
@@ -256,7 +288,7 @@ class OracleCache:
         self.K = K
         self.r = r
         self.seed = seed
-        self.policy, self.block = policy, block
+        self.policy, self.block, self.compaction = policy, block, compaction
         self.g = np.zeros((self.B, layers), dtype=np.int64)
         # heads: iterable of (seq, layer, kv_head) to track; None = all
         if heads is None:
@@ -301,7 +333,10 @@ class OracleCache:
             cur = self.gen[key]
             if not should_evict(g, int(cur.size), self.K, self.r):
                 continue
-            if self.policy == POLICY_RANDOM:
+            if self.compaction == COMPACT_HOLEFILL:
+                new, ev = evict_head_holefill(cur, g, self.K, self.r, self.seed, layer, seq, self.KVH, h,
+                                              self.policy, self.block)
+            elif self.policy == POLICY_RANDOM:
                 new, ev = evict_head(cur, g, self.K, self.r, self.seed, layer, seq * self.KVH + h)
             elif self.policy == POLICY_SNAPKV:
                 new, ev = evict_head_scored(cur, g, self.K, self.r, scorer(seq, layer, h, cur))

@@ -24,6 +24,9 @@
  *   - Decode attention o = sum_i softmax_i(q.k_i / sqrt(d)) v_i in fp64
  *     (section 2 "Notation"), grouped-query: a KV head's keep-set serves
  *     every query head of its group (Appendix F).
+ *   - Order-free (hole-filling) compaction: keys drawn per position, the
+ *     evicted slots refilled from the newest ones (attention is a sum over
+ *     the cached set, so slot order carries nothing).
  *   - The scored comparator (section 2, "Baselines as choices of s"): the
  *     SnapKV score -- attention received from the last w queries, summed
  *     over the query heads of the group, max-pooled over neighbouring
@@ -143,8 +146,8 @@ static int ora_cmp_i32(const void* a, const void* b)
 
 /*
  * Keep the K candidates with the smallest (key, ordinal), returned in
- * ascending ordinal order ("keep-sets are sorted chronologically before
- * compaction", Appendix F).  The plain definition: sort all, take K.
+ * ascending ordinal order (Appendix F orders each keep-set by time before the
+ * cache is compacted).  The plain definition: sort all, take K.
  * Returns 0, or -1 on bad arguments / allocation failure.
  */
 int ora_select_keep(const uint32_t* keys, int n, int K, int32_t* keep_out)
@@ -165,9 +168,9 @@ int ora_select_keep(const uint32_t* keys, int n, int K, int32_t* keep_out)
 }
 
 /*
- * The periodic trigger (section 2: "the buffer fills every r steps and
- * triggers an eviction"; Appendix F: "every r=64 decode steps, once the
- * cache exceeds K+r").  `c` counts the cached generated tokens, `g` the
+ * The periodic trigger (section 2: an eviction runs each time the r-token
+ * buffer has filled; Appendix F: every r = 64 decode steps once the cache
+ * holds more than K + r).  `c` counts the cached generated tokens, `g` the
  * generated tokens appended so far; the check runs after the step's append.
  * Fires iff g is a multiple of r and the candidates (everything but the
  * newest r) outnumber the budget.
@@ -181,7 +184,7 @@ int ora_should_evict(int g, int c, int K, int r)
  * One eviction round for one (sequence, layer, KV head).
  *   gen[0..*c)  positions of the cached generated tokens, in slot order
  *               (ascending position); the prompt is not in this list -- it is
- *               never a candidate (section 3, "Protect the question").
+ *               never a candidate (section 3: the prompt is protected).
  * If the trigger fires: candidates are gen[0 .. c-r) (everything outside the
  * recent buffer), each gets its Philox score, the K smallest survive, and
  * gen becomes kept-candidates ++ the r buffer positions, in order.
@@ -439,5 +442,81 @@ int ora_evict_head_scored(int32_t* gen, int* c, int g, int K, int r, const doubl
     memcpy(gen, next, sizeof(int32_t) * (size_t)(K + r));
     *c = K + r;
     free(pooled); free(keep); free(next);
+    return m;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Order-free compaction.  Attention is a sum over the cached set (section 2, */
+/* "Notation"), so the slots need no chronological order; the keep-set is a   */
+/* random subset of positions -- in Appendix G's terms, a random permutation  */
+/* of slot indices.  Keys are drawn per position, so the kept set does not    */
+/* depend on the slot layout.                                                 */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * Policy score of the candidate at `position` when slots carry no order:
+ *   0 random  -- Philox word 0 of counter (position, step, layer, seq * kv_heads + h);
+ *   1 shared  -- the same with head id seq * kv_heads for every head;
+ *   2 recency -- the newest positions score lowest: 0xFFFFFFFF - position;
+ *   3 block   -- as ordered: counter word 0 = position / block.
+ */
+uint32_t ora_position_key(int policy, uint64_t seed, uint32_t layer, uint32_t seq, uint32_t kv_heads, uint32_t h,
+                          uint32_t step, int32_t position, int32_t block)
+{
+    switch (policy) {
+        case 1:
+            return ora_random_key(seed, layer, seq * kv_heads, step, (uint32_t)position);
+        case 2:
+            return 0xFFFFFFFFu - (uint32_t)position;
+        case 3:
+            return ora_random_key(seed, layer, seq * kv_heads + h, step, (uint32_t)(position / block));
+        default:
+            return ora_random_key(seed, layer, seq * kv_heads + h, step, (uint32_t)position);
+    }
+}
+
+/*
+ * One eviction round with hole-filling compaction.  Same trigger and the same
+ * top-K (the K smallest (key, ordinal) among the n = c - r candidates, keys
+ * by position).  The m = n - K evicted slots e_0 < ... < e_{m-1} are refilled
+ * from the m newest slots: slot e_i takes the row of slot c - m + i; the cache
+ * shrinks to c - m slots.  Every other slot keeps its row.  Defined for
+ * c <= K + 2r (the cache's capacity), where m <= r and the m newest slots are
+ * all buffer slots.  Returns m (0 when the trigger does not fire) and the
+ * evicted ordinals, -1 on error.
+ */
+int ora_evict_head_holefill(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int layer, int seq,
+                            int kv_heads, int h, int policy, int block, int32_t* evicted_out)
+{
+    const int cc = *c;
+    if (!ora_should_evict(g, cc, K, r)) return 0;
+    if (policy == 3 && block < 1) return -1;
+    const int n = cc - r;
+    if (n - K > r) return -1; /* the newest m slots must all be buffer slots: c <= K + 2r */
+    uint32_t* keys = (uint32_t*)malloc(sizeof(uint32_t) * (size_t)n);
+    int32_t* keep = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
+    int32_t* ev = (int32_t*)malloc(sizeof(int32_t) * (size_t)n);
+    if (!keys || !keep || !ev) {
+        free(keys); free(keep); free(ev);
+        return -1;
+    }
+    for (int j = 0; j < n; ++j)
+        keys[j] = ora_position_key(policy, seed, (uint32_t)layer, (uint32_t)seq, (uint32_t)kv_heads, (uint32_t)h,
+                                   (uint32_t)g, gen[j], block);
+    if (ora_select_keep(keys, n, K, keep) != 0) {
+        free(keys); free(keep); free(ev);
+        return -1;
+    }
+    int m = 0, ki = 0;
+    for (int j = 0; j < n; ++j) {
+        if (ki < K && keep[ki] == j) ++ki;
+        else ev[m++] = j;
+    }
+    for (int i = 0; i < m; ++i) {
+        gen[ev[i]] = gen[cc - m + i];
+        if (evicted_out) evicted_out[i] = ev[i];
+    }
+    *c = cc - m;
+    free(keys); free(keep); free(ev);
     return m;
 }

@@ -14,8 +14,8 @@
 //   compact_kernel  many CTAs per triggered head: order-preserving move of the
 //                   survivors (kept candidates, then the buffer rows) into
 //                   the head's spare region with coalesced 16-byte copies
-//                   ("keep-sets sorted chronologically ... compacted with a
-//                   gather", Appendix F).  Out of place, so CTAs never wait on
+//                   (Appendix F keeps each keep-set in time order and gathers
+//                   the cache into it).  Out of place, so CTAs never wait on
 //                   each other; the old region becomes the spare.
 #include <cuda_runtime.h>
 #include <stdint.h>
