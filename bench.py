@@ -60,6 +60,7 @@ WORKLOADS = _workloads()
 DEFAULT_CONFIG = 2
 COMPARATOR_CONFIGS = (5,)  # workloads that also time the scored comparator on the same caches
 POLICY_SNAPKV = 4
+COMPACTIONS = {"ordered": 0, "holefill": 1}  # order-preserving (the method's engine) / order-free in place
 WINDOW_STEP0 = 1 << 20     # synthetic step index of the first restored window query (row u: WINDOW_STEP0 + u)
 
 
@@ -95,7 +96,7 @@ def describe(w):
 class Workload:
     """Device-side setup of one workload through the public API."""
 
-    def __init__(self, cfg, rank=0, ring=4, policy=0):
+    def __init__(self, cfg, rank=0, ring=4, policy=0, compaction=0):
         import torch
 
         import paper_2609_03430_gb300 as ra
@@ -113,7 +114,7 @@ class Workload:
         self.stream = torch.cuda.current_stream()
         self.policy = policy
         self.cache = ra.RandomAttentionCache(self.L, self.H, self.KVH, D, self.lp, self.K, self.r, self.eseed,
-                                             policy=policy)
+                                             policy=policy, compaction=compaction)
         self.ctx = self.cache.ctx
         self.key_scale = None
         if w["key_scale"]:
@@ -380,7 +381,7 @@ def config_dict(w, args):
             "q_heads": w["H"], "kv_heads": w["KVH"], "head_dim": D, "K": w["K"], "r": w["r"],
             "prompt_mean": float(np.mean(w["lp"])), "start": "steady state (K + r cached generated per head)",
             "l2": "inputs larger than L2 (every step streams the whole cache)", "parallelism": f"replicas x{args.gpus}",
-            "policy": getattr(args, "policy", "random")}
+            "policy": getattr(args, "policy", "random"), "compaction": getattr(args, "compaction", "ordered")}
 
 
 # --------------------------------------------------------------------------- GPU run
@@ -464,6 +465,30 @@ def run_comparator(args, rank, world, barrier, peaks, random_ms, random_kern, ra
             "score_kernels": score, "kernels": kern}
 
 
+def run_holefill_variant(args, rank, world, barrier, peaks, ordered_ms, ordered_kern, ordered_rounds):
+    """Order-free (hole-filling) compaction on the same caches: the workload rebuilt from the same
+    seeds with the evicted slots refilled in place, timed like the main run."""
+    wl = Workload(args.config, rank=rank, compaction=COMPACTIONS["holefill"])
+    for t in range(args.warmup):
+        wl.step(t)
+    wl.ra.ra_check_device(wl.ctx)
+    cache_bytes = wl.bytes_per_step()
+    ms, t_next, _, _ = timed_steps(wl, args.steps, args.warmup, barrier)
+    kern, rounds, _ = evented_steps(wl, args.steps, t_next)
+    ms_step, units = reduce_over_ranks(ms, float(wl.B), world)
+    wl.cache.close()
+    return {"compaction": "order-free: keys per position, evicted slots refilled in place from the newest "
+                          "ones by the select kernel (no compaction launch)",
+            "value": units / (ms_step * 1e-3), "unit": UNIT, "ms_per_step": ms_step,
+            "step_time_vs_ordered": ms_step / ordered_ms,
+            "step_effective_frac": cache_bytes / (ms_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "eviction_us_per_round": {
+                "ordered": _eviction_us_per_round(ordered_kern, ("select", "compact"), ordered_rounds),
+                "holefill": _eviction_us_per_round(kern, ("select", "compact"), rounds),
+                "what": "evented kernel time of a step's eviction launches / (sequence, layer) rounds they ran"},
+            "kernels": kern}
+
+
 def run_ours(args, w):
     import torch
 
@@ -478,7 +503,7 @@ def run_ours(args, w):
     else:
         torch.cuda.set_device(0)
     main_policy = POLICY_SNAPKV if args.policy == "snapkv" else 0
-    wl = Workload(args.config, rank=rank, policy=main_policy)
+    wl = Workload(args.config, rank=rank, policy=main_policy, compaction=COMPACTIONS[args.compaction])
     stream = wl.stream
     ctx = wl.ctx
 
@@ -557,6 +582,9 @@ def run_ours(args, w):
     if main_policy == 0 and (args.comparator == "on" or
                              (args.comparator == "auto" and args.config in COMPARATOR_CONFIGS)):
         comparator = run_comparator(args, rank, world, barrier, peaks, ms_step, kern, rounds)
+    holefill = None
+    if main_policy == 0 and args.compaction == "ordered" and args.variants == "on":
+        holefill = run_holefill_variant(args, rank, world, barrier, peaks, ms_step, kern, rounds)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)
@@ -573,6 +601,8 @@ def run_ours(args, w):
                                            "(all kernels of the step, launches overlapped)"}}
         if comparator is not None:
             line["comparator"] = comparator
+        if holefill is not None:
+            line["holefill_variant"] = holefill
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
@@ -595,6 +625,10 @@ def main(argv=None):
                     help="override the layer count (only to shrink profiler captures; not a benchmark workload)")
     ap.add_argument("--policy", choices=["random", "snapkv"], default="random",
                     help="eviction policy of the timed run (random: the method; snapkv: the scored comparator)")
+    ap.add_argument("--compaction", choices=sorted(COMPACTIONS), default="ordered",
+                    help="eviction compaction of the timed run (holefill: order-free, in place)")
+    ap.add_argument("--variants", choices=["on", "off"], default="on",
+                    help="also time order-free (hole-filling) compaction on the same caches")
     ap.add_argument("--comparator", choices=["auto", "on", "off"], default="auto",
                     help="also time the scored comparator on the same caches (auto: the ragged workload)")
     ap.add_argument("--traffic", type=float, default=None,

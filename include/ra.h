@@ -155,6 +155,34 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
 int ra_set_policy(ra_ctx* ctx, int policy, int block);
 
 /*
+ * Compaction of an eviction round (default RA_COMPACT_ORDERED):
+ *   RA_COMPACT_ORDERED  the survivors stay in time order: kept candidates, then
+ *                       the buffer, moved into a fresh region (Appendix F keeps
+ *                       each keep-set in time order and gathers the cache into
+ *                       it).  Moves about K + r rows per head and round.
+ *   RA_COMPACT_HOLEFILL order-free: attention is a sum over the cached set
+ *                       (section 2), so slots need no order -- in Appendix G's
+ *                       terms a keep-set is a random permutation of slot
+ *                       indices.  Each candidate's key is drawn per position
+ *                       (counter word 0 = its position instead of its ordinal;
+ *                       recency keeps the largest positions), so the kept set
+ *                       does not depend on the layout.  The m evicted slots
+ *                       e_0 < ... < e_{m-1} are refilled in place from the m
+ *                       newest slots (slot e_i takes slot c - m + i): m <= r
+ *                       row moves per head and round, done by the selection
+ *                       kernel itself.  ra_get_positions then lists positions
+ *                       in slot order, which is no longer time order.  In
+ *                       ra_decode_layer the step's token, the newest slot, is
+ *                       written straight into the evicted slot it refills.
+ * Takes effect from the next eviction.  RA_COMPACT_HOLEFILL cannot be combined
+ * with RA_POLICY_SNAPKV (its pooling runs over neighbouring positions, which
+ * needs time order): that combination fails with RA_ERR_UNSUPPORTED.
+ */
+#define RA_COMPACT_ORDERED 0
+#define RA_COMPACT_HOLEFILL 1
+int ra_set_compaction(ra_ctx* ctx, int mode);
+
+/*
  * Scored policy, warm start: load the query window of layer `layer` from q,
  * device [batch][q_heads][r][head_dim] bf16, where row u of (b, qh) is the
  * query of decode step g_b - r + 1 + u (g_b = the sequence's generated count,

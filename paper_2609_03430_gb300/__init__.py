@@ -42,6 +42,7 @@ SIGNATURES = {
     "ra_prefill": (_i, [_vp, _i, _vp, _vp, _i, _vp]),
     "ra_restore": (_i, [_vp, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp]),
     "ra_set_policy": (_i, [_vp, _i, _i]),
+    "ra_set_compaction": (_i, [_vp, _i]),
     "ra_restore_queries": (_i, [_vp, _i, _vp, ctypes.c_float, _vp]),
     "ra_get_scores": (_i, [_vp, _i, _i, _i, ctypes.POINTER(ctypes.c_float), _i, _ip, _vp]),
     "ra_set_active": (_i, [_vp, _i, _i]),
@@ -142,6 +143,13 @@ RA_POLICY_RANDOM, RA_POLICY_SHARED, RA_POLICY_RECENCY, RA_POLICY_BLOCK, RA_POLIC
 
 def ra_set_policy(ctx, policy, block=1):
     return _check(lib().ra_set_policy(ctx, int(policy), int(block)), ctx)
+
+
+RA_COMPACT_ORDERED, RA_COMPACT_HOLEFILL = 0, 1
+
+
+def ra_set_compaction(ctx, mode):
+    return _check(lib().ra_set_compaction(ctx, int(mode)), ctx)
 
 
 def ra_restore_queries(ctx, layer, q_ptr, scale=0.0, stream=None):
@@ -247,7 +255,7 @@ class RandomAttentionCache:
     """Owns a context and its torch-allocated device arena (uint8 CUDA tensor)."""
 
     def __init__(self, layers, q_heads, kv_heads, head_dim, prompt_lens, K, r=64, seed=0, device=None, stream=None,
-                 policy=RA_POLICY_RANDOM, block=1):
+                 policy=RA_POLICY_RANDOM, block=1, compaction=RA_COMPACT_ORDERED):
         import torch
 
         if isinstance(prompt_lens, int):
@@ -256,6 +264,8 @@ class RandomAttentionCache:
         self.L, self.H, self.KVH, self.D = layers, q_heads, kv_heads, head_dim
         self.B, self.K, self.r, self.seed = len(self.prompt_lens), K, r, seed
         self.ctx = ra_create_batched(layers, q_heads, kv_heads, head_dim, self.prompt_lens, K, r, seed)
+        if compaction != RA_COMPACT_ORDERED:
+            ra_set_compaction(self.ctx, compaction)
         if policy != RA_POLICY_RANDOM:  # before sizing: the scored policy adds buffers to the arena
             ra_set_policy(self.ctx, policy, block)
         self.nbytes = ra_device_bytes(self.ctx)

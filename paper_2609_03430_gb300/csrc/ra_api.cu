@@ -72,6 +72,7 @@ struct ra_ctx {
     std::vector<uint8_t> active;     // [B]
     int policy = RA_POLICY_RANDOM;   // candidate scoring (ra_set_policy)
     int block = 1;
+    int compaction = RA_COMPACT_ORDERED;  // ra_set_compaction
     std::vector<int32_t> score_n;    // [L][B] candidates of the latest scored round
     // profiling
     bool prof = false;
@@ -218,18 +219,25 @@ void fill_active(const ra_ctx* ctx, uint32_t* mask)
 // ceil(lp / TILE) prompt tiles and ceil(gen / TILE) tiles of generated rows, where gen is
 // the cached generated rows plus one for a fused new token; the tiles are cut into one equal
 // chunk per warp.  *slots = rows attended.
-int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots)
+int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots,
+                   const std::vector<uint8_t>* appended = nullptr)
 {
     fill_active(ctx, p->active);
+    // fused: every active sequence's token is pending, except those an eviction already appended
+    for (int i = 0; i < RA_MAX_BATCH / 32; ++i) p->pending[i] = fused ? p->active[i] : 0u;
+    if (fused && appended)
+        for (int b = 0; b < ctx->B; ++b)
+            if ((*appended)[b]) p->pending[b >> 5] &= ~(1u << (b & 31));
     const int T = attn_tile_rows(ctx->G);
     p->tile = T;
     long long acc = 0, rows = 0;
     int na = 0;
     p->seq_base[0] = 0;
     for (int b = 0; b < ctx->B; ++b) {
-        const int gen = ctx->c[(size_t)layer * ctx->B + b] + fused;
+        const int gen = ctx->c[(size_t)layer * ctx->B + b] + (int)((p->pending[b >> 5] >> (b & 31)) & 1u);
         p->seq_gen[b] = gen;
-        p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b];
+        // generated tokens before this step's (a token an eviction already appended is not counted)
+        p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b] - (appended && (*appended)[b] ? 1 : 0);
         if (ctx->active[b]) {
             acc += (long long)ctx->KVH * ((ctx->lp[b] + T - 1) / T + (gen + T - 1) / T);
             rows += (long long)ctx->KVH * (ctx->lp[b] + gen);
@@ -322,11 +330,16 @@ int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s)
         if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
     }
     {
-        ProfScope ps(ctx, RA_KERNEL_SELECT, 0.0, s);
+        // with order-free compaction the select kernel also moves m rows per head (read and write)
+        double fill = 0;
+        if (p.holefill)
+            for (int i = 0; i < p.n_trig; ++i) fill += (double)(p.trig_n[i] - ctx->K) * ctx->KVH * 2.0 * (2 * kRowBytes + 4);
+        ProfScope ps(ctx, RA_KERNEL_SELECT, fill, s);
         e = launch_select(p, s);
         ps.done();
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
+    if (p.holefill) return RA_OK;  // the select kernel refilled the evicted slots in place
     {
         ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
         e = launch_compact(p, s);
@@ -596,6 +609,8 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block)
     if (policy < RA_POLICY_RANDOM || policy > RA_POLICY_SNAPKV)
         return fail(ctx, RA_ERR_INVALID_ARG, "unknown policy %d", policy);
     if (policy == RA_POLICY_BLOCK && block < 1) return fail(ctx, RA_ERR_INVALID_ARG, "block must be >= 1");
+    if (policy == RA_POLICY_SNAPKV && ctx->compaction == RA_COMPACT_HOLEFILL)
+        return fail(ctx, RA_ERR_UNSUPPORTED, "the scored policy needs ordered compaction");
     if (policy == RA_POLICY_SNAPKV && !ctx->scoring) {
         if (ctx->bound)
             return fail(ctx, RA_ERR_STATE, "the scored policy must be set before ra_device_bytes / ra_bind");
@@ -609,6 +624,17 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block)
     }
     ctx->policy = policy;
     ctx->block = policy == RA_POLICY_BLOCK ? block : 1;
+    return RA_OK;
+}
+
+int ra_set_compaction(ra_ctx* ctx, int mode)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (mode != RA_COMPACT_ORDERED && mode != RA_COMPACT_HOLEFILL)
+        return fail(ctx, RA_ERR_INVALID_ARG, "unknown compaction %d", mode);
+    if (mode == RA_COMPACT_HOLEFILL && ctx->policy == RA_POLICY_SNAPKV)
+        return fail(ctx, RA_ERR_UNSUPPORTED, "the scored policy needs ordered compaction");
+    ctx->compaction = mode;
     return RA_OK;
 }
 
@@ -711,6 +737,7 @@ int ra_evict(ra_ctx* ctx, int layer, int* n_fired, void* stream)
     p.layer = layer;
     p.policy = ctx->policy;
     p.block = ctx->block;
+    p.holefill = ctx->compaction == RA_COMPACT_HOLEFILL;
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
@@ -783,6 +810,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
                         ctx->Cmax);
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
+    std::vector<uint8_t> appended((size_t)ctx->B, 0);  // sequences whose token the eviction wrote
     // 1. Eviction first, with the step's token pending: it is the newest slot, so it is never a
     //    candidate, and evicting before writing it gives the same state as append-then-evict.
     EvictParams ep{};
@@ -790,6 +818,11 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     ep.layer = layer;
     ep.policy = ctx->policy;
     ep.block = ctx->block;
+    ep.holefill = ctx->compaction == RA_COMPACT_HOLEFILL;
+    if (ep.holefill) {  // the token refills an evicted slot: the select kernel writes it
+        ep.k_new = k_new;
+        ep.v_new = v_new;
+    }
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
@@ -809,8 +842,14 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
         if ((rc = run_eviction(ctx, ep, moved, s)) != RA_OK) return rc;
         for (int i = 0; i < n; ++i) {
             const int b = ep.trig[i];
-            ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written
             ctx->nev[base + b] += 1;
+            if (ep.holefill) {  // the token is in the cache already
+                ctx->c[base + b] = ctx->K + ctx->r;
+                ctx->g[base + b] += 1;
+                appended[b] = 1;
+            } else {
+                ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written
+            }
         }
     }
     // 2. Fused append + attention (+ merge of the split pieces).
@@ -827,7 +866,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     p.ring_off = 0;  // the query of step g + 1
     int n_active = 0, ctas = 0;
     double rows = 0;
-    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
+    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &appended)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
     // The kernel may request its first K/V tiles before its predecessor finishes when that
@@ -837,17 +876,19 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     // everything older than the predecessor has completed.
     p.early = (n == 0 && ctx->L >= 2) ? 1 : 0;
     {
-        // rows read (the new token's from the caller), its row written, q read, out written
+        // rows read (a new token's from the caller), a new token's row written, q read, out written
+        int n_pending = 0;
+        for (int b = 0; b < ctx->B; ++b) n_pending += (int)((p.pending[b >> 5] >> (b & 31)) & 1u);
         ProfScope ps(ctx, RA_KERNEL_ATTN,
                      rows * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes +
-                         (double)n_active * ctx->KVH * 2 * kRowBytes,
+                         (double)n_pending * ctx->KVH * 2 * kRowBytes,
                      s);
         e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
         ps.done();
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
     for (int b = 0; b < ctx->B; ++b) {
-        if (!ctx->active[b]) continue;
+        if (!ctx->active[b] || appended[b]) continue;
         ctx->c[base + b] += 1;
         ctx->g[base + b] += 1;
     }

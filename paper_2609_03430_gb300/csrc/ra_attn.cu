@@ -171,7 +171,8 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int wa
         const int kg = it.k - it.tp;
         d.row = it.grow + (long long)kg * T;
         d.n = min(T, it.gen - kg * T);
-        if (p.k_new && kg * T + d.n == it.gen) d.flags |= kNewTok;  // its last row is the step's new token
+        if (p.k_new && ((p.pending[it.b >> 5] >> (it.b & 31)) & 1u) && kg * T + d.n == it.gen)
+            d.flags |= kNewTok;  // its last row is the step's new token
     }
     if (it.k + 1 == it.nt || it.f + 1 == it.end) d.flags |= kLast;
     d.hid = it.b * p.lay.KVH + it.h;

@@ -10,7 +10,10 @@
 //                   the K smallest (score, ordinal) -- Eq. 1 -- and a
 //                   ballot-compacted, ascending list of the evicted ordinals.
 //                   Under the scored comparator the score is the max-pooled
-//                   window attention that ra_score.cu computed.
+//                   window attention that ra_score.cu computed; with order-free
+//                   slots every key follows the candidate's position.
+//                   With order-free slots the select CTA also refills the
+//                   evicted slots in place from the newest ones (no compact).
 //   compact_kernel  many CTAs per triggered head: order-preserving move of the
 //                   survivors (kept candidates, then the buffer rows) into
 //                   the head's spare region with coalesced 16-byte copies
@@ -107,10 +110,18 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
 
     if (tid < 256) hist[0][tid] = 0;  // the first digit's histogram (the fill's barrier publishes it)
     const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
-    if (p.policy == RA_POLICY_RECENCY) {  // protected recency: the K newest candidates score lowest
+    const int32_t* pos = L.pos + (size_t)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
+    if (p.holefill && p.policy != RA_POLICY_BLOCK) {  // order-free slots: every key follows the position
+        const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
+#pragma unroll 8
+        for (int j = tid; j < N; j += kSelThreads) {
+            const uint32_t pj = (uint32_t)__ldg(pos + j);
+            keys[j] = p.policy == RA_POLICY_RECENCY ? 0xFFFFFFFFu - pj
+                                                    : philox4x32_10_w0(pj, (uint32_t)g, (uint32_t)p.layer, id, k0, k1);
+        }
+    } else if (p.policy == RA_POLICY_RECENCY) {  // protected recency: the K newest candidates score lowest
         for (int j = tid; j < N; j += kSelThreads) keys[j] = (uint32_t)(N - 1 - j);
     } else if (p.policy == RA_POLICY_BLOCK) {  // one draw per block of consecutive positions
-        const int32_t* pos = L.pos + (size_t)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
         for (int j = tid; j < N; j += kSelThreads)
             keys[j] = philox4x32_10_w0((uint32_t)(pos[j] / p.block), (uint32_t)g, (uint32_t)p.layer, (uint32_t)head_id,
                                        k0, k1);
@@ -259,17 +270,57 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     __syncthreads();
     if (tid == 0) {
         const int32_t* regp = L.region + ((size_t)p.layer * L.B + b) * L.KVH + h;
-        const int src = *regp, dst = L.spare[b * L.KVH + h];
+        const int src = *regp, dst = p.holefill ? src : L.spare[b * L.KVH + h];  // hole-filling works in place
         const bool ok = (s_total == (uint32_t)m);
         plan[0] = src;
         plan[1] = dst;
         plan[2] = c;
         plan[3] = ok ? m : 0;
-        if (ok) {
+        if (ok && !p.holefill) {
             L.region[((size_t)p.layer * L.B + b) * L.KVH + h] = dst;
             L.spare[b * L.KVH + h] = src;
-        } else {
+        } else if (!ok) {
             atomicExch(L.err, kDeviceErrPlan);
+        }
+    }
+    if (!p.holefill) return;
+    // Order-free compaction, in place: evicted slot e_i takes the row of slot top - m + i, where
+    // top is the slot count including a pending token (the newest slot, taken from the caller's
+    // rows).  Those m <= r slots are all buffer slots, so sources and destinations never overlap.
+    __syncthreads();  // the evicted list (written by warp 0) and the header
+    if (s_total != (uint32_t)m) return;
+    const int top = p.k_new ? c + 1 : c;
+    const long long row0 = L.gen_row0 + (long long)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
+    int32_t* gpos = L.pos + (size_t)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
+    const int part = lane & 15;
+    uint16_t* pool = lane < 16 ? L.kpool : L.vpool;
+    constexpr int kWarpsSel = kSelThreads / 32, kBatch = 8;  // rows a warp has in flight
+    for (int i0 = warp; i0 < m; i0 += kWarpsSel * kBatch) {
+        uint4 v[kBatch];
+        int32_t pv[kBatch];
+        int to[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {  // every load of the batch first ...
+            const int i = i0 + u * kWarpsSel;
+            to[u] = -1;
+            if (i < m) {
+                const int from = top - m + i;
+                to[u] = plan[kPlanHeader + i];
+                if (from == c) {  // the step's pending token
+                    const uint16_t* src = (lane < 16 ? p.k_new : p.v_new) + ((size_t)b * L.KVH + h) * kHeadDim;
+                    v[u] = reinterpret_cast<const uint4*>(src)[part];
+                    pv[u] = L.seq_lp[b] + g - 1;
+                } else {
+                    v[u] = reinterpret_cast<const uint4*>(pool + (row0 + from) * kHeadDim)[part];
+                    pv[u] = gpos[from];
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {  // ... then the stores
+            if (to[u] < 0) continue;
+            reinterpret_cast<uint4*>(pool + (row0 + to[u]) * kHeadDim)[part] = v[u];
+            if (lane == 0) gpos[to[u]] = pv[u];
         }
     }
 }

@@ -62,8 +62,13 @@ struct AppendParams {
 struct EvictParams {
     DevLayout lay;
     int layer;
-    int policy;  // RA_POLICY_*: how candidates are scored
-    int block;   // RA_POLICY_BLOCK: positions per block
+    int policy;    // RA_POLICY_*: how candidates are scored
+    int block;     // RA_POLICY_BLOCK: positions per block
+    int holefill;  // RA_COMPACT_HOLEFILL: keys per position, evicted slots refilled in place by select
+    // Fused step under hole-filling: the step's new rows [B][KVH][128] (the token is the newest slot
+    // and always among those that refill the evicted ones); null when the token is already cached.
+    const uint16_t* k_new;
+    const uint16_t* v_new;
     int n_trig;
     int16_t trig[RA_MAX_BATCH];    // triggered sequence ids
     int32_t trig_c[RA_MAX_BATCH];  // rows in the cache (a pending new token is not among them)
@@ -101,6 +106,7 @@ struct AttnParams {
     int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of tiles per head over active sequences
     int32_t seq_gen[RA_MAX_BATCH];       // generated rows attended per head (incl. a fused new token)
     int32_t seq_g[RA_MAX_BATCH];         // tokens generated before this step's (fused) / up to it (separate)
+    uint32_t pending[RA_MAX_BATCH / 32]; // fused step: sequences whose new token this kernel appends
     uint16_t* qring;                     // record each head's query rows in the scored policy's window (or null)
     int ring_off;                        // window slot of sequence b = (seq_g[b] + ring_off) mod r
 };

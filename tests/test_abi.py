@@ -103,6 +103,23 @@ def test_scored_policy_sizes_its_buffers_before_bind(ra):
     ra.ra_destroy(big)
 
 
+def test_compaction_mode_validation(ra):
+    ctx = ra.ra_create_batched(2, 8, 2, 128, [10], 64, 16, 0)
+    ra.ra_set_compaction(ctx, ra.RA_COMPACT_HOLEFILL)
+    with pytest.raises(ra.RAError) as e:
+        ra.ra_set_policy(ctx, ra.RA_POLICY_SNAPKV)  # pooling needs time-ordered slots
+    assert e.value.code == ra.RA_ERR_UNSUPPORTED
+    ra.ra_set_compaction(ctx, ra.RA_COMPACT_ORDERED)
+    ra.ra_set_policy(ctx, ra.RA_POLICY_SNAPKV)
+    with pytest.raises(ra.RAError) as e:
+        ra.ra_set_compaction(ctx, ra.RA_COMPACT_HOLEFILL)
+    assert e.value.code == ra.RA_ERR_UNSUPPORTED
+    with pytest.raises(ra.RAError) as e:
+        ra.ra_set_compaction(ctx, 2)
+    assert e.value.code == ra.RA_ERR_INVALID_ARG
+    ra.ra_destroy(ctx)
+
+
 def test_no_cpu_fallback_in_product_package():
     """The product package never imports the oracle (test infrastructure)."""
     pkg = os.path.join(ROOT, "paper_2609_03430_gb300")

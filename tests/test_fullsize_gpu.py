@@ -27,8 +27,9 @@ def _samples(w, n_heads, n_attn, seed):
     return sorted(heads), attn
 
 
-@pytest.mark.parametrize("cfg", [2, 3, 4, 5])
-def test_workload_parity_sampled(cfg):
+@pytest.mark.parametrize("cfg,compaction", [(2, 0), (3, 0), (4, 0), (5, 0), (5, 1)],
+                         ids=["cfg2", "cfg3", "cfg4", "cfg5", "cfg5-holefill"])
+def test_workload_parity_sampled(cfg, compaction):
     import torch
 
     import bench
@@ -38,12 +39,12 @@ def test_workload_parity_sampled(cfg):
     import synth.gpu as sg
 
     torch.cuda.set_device(0)
-    wl = bench.Workload(cfg, ring=1)
+    wl = bench.Workload(cfg, ring=1, compaction=compaction)
     w = wl.w
     L, B, H, KVH, K, r, D = wl.L, wl.B, wl.H, wl.KVH, wl.K, wl.r, 128
     G = H // KVH
     heads, attn_heads = _samples(w, 64, 8, cfg)
-    orc = oracle.OracleCache(L, KVH, wl.lp, K, r, wl.eseed, heads=heads)
+    orc = oracle.OracleCache(L, KVH, wl.lp, K, r, wl.eseed, heads=heads, compaction=compaction)
     for (b, l, h) in heads:
         c, g = wl.c0[b], wl.g0[b]
         orc.gen[(b, l, h)] = np.arange(wl.lp[b] + g - c, wl.lp[b] + g, dtype=np.int32)
