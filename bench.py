@@ -60,7 +60,8 @@ WORKLOADS = _workloads()
 DEFAULT_CONFIG = 2
 COMPARATOR_CONFIGS = (5,)  # workloads that also time the scored comparator on the same caches
 POLICY_SNAPKV = 4
-COMPACTIONS = {"ordered": 0, "holefill": 1}  # order-preserving (the method's engine) / order-free in place
+# order-preserving (the method's engine) / order-free in place / order-preserving inside the attention pass
+COMPACTIONS = {"ordered": 0, "holefill": 1, "fused": 2}
 WINDOW_STEP0 = 1 << 20     # synthetic step index of the first restored window query (row u: WINDOW_STEP0 + u)
 
 

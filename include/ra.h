@@ -174,12 +174,23 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block);
  *                       in slot order, which is no longer time order.  In
  *                       ra_decode_layer the step's token, the newest slot, is
  *                       written straight into the evicted slot it refills.
+ *   RA_COMPACT_FUSED    the ordered layout, but in ra_decode_layer the attention
+ *                       pass itself does the compaction: it reads each evicting
+ *                       head's old region (as it must read every survivor
+ *                       anyway), gives the evicted rows no weight, and writes
+ *                       each survivor and the step's token to its slot in the
+ *                       new region -- one read of the old rows instead of two.
+ *                       Needs r <= 64; otherwise, and in ra_evict, the
+ *                       separate compaction runs.  Results are identical to
+ *                       RA_COMPACT_ORDERED (slower on the measured workloads:
+ *                       the copy is done by the attention warps).
  * Takes effect from the next eviction.  RA_COMPACT_HOLEFILL cannot be combined
  * with RA_POLICY_SNAPKV (its pooling runs over neighbouring positions, which
  * needs time order): that combination fails with RA_ERR_UNSUPPORTED.
  */
 #define RA_COMPACT_ORDERED 0
 #define RA_COMPACT_HOLEFILL 1
+#define RA_COMPACT_FUSED 2
 int ra_set_compaction(ra_ctx* ctx, int mode);
 
 /*

@@ -145,7 +145,7 @@ def ra_set_policy(ctx, policy, block=1):
     return _check(lib().ra_set_policy(ctx, int(policy), int(block)), ctx)
 
 
-RA_COMPACT_ORDERED, RA_COMPACT_HOLEFILL = 0, 1
+RA_COMPACT_ORDERED, RA_COMPACT_HOLEFILL, RA_COMPACT_FUSED = 0, 1, 2
 
 
 def ra_set_compaction(ctx, mode):

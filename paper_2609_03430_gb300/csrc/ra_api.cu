@@ -220,9 +220,14 @@ void fill_active(const ra_ctx* ctx, uint32_t* mask)
 // the cached generated rows plus one for a fused new token; the tiles are cut into one equal
 // chunk per warp.  *slots = rows attended.
 int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots,
-                   const std::vector<uint8_t>* appended = nullptr)
+                   const std::vector<uint8_t>* appended = nullptr, const std::vector<int32_t>* old_rows = nullptr)
 {
     fill_active(ctx, p->active);
+    // sequences whose compaction the launch does: their cached rows are the old region's
+    for (int i = 0; i < RA_MAX_BATCH / 32; ++i) p->compacting[i] = 0u;
+    if (old_rows)
+        for (int b = 0; b < ctx->B; ++b)
+            if ((*old_rows)[b] >= 0) p->compacting[b >> 5] |= 1u << (b & 31);
     // fused: every active sequence's token is pending, except those an eviction already appended
     for (int i = 0; i < RA_MAX_BATCH / 32; ++i) p->pending[i] = fused ? p->active[i] : 0u;
     if (fused && appended)
@@ -234,7 +239,8 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     int na = 0;
     p->seq_base[0] = 0;
     for (int b = 0; b < ctx->B; ++b) {
-        const int gen = ctx->c[(size_t)layer * ctx->B + b] + (int)((p->pending[b >> 5] >> (b & 31)) & 1u);
+        const int cached = (old_rows && (*old_rows)[b] >= 0) ? (*old_rows)[b] : ctx->c[(size_t)layer * ctx->B + b];
+        const int gen = cached + (int)((p->pending[b >> 5] >> (b & 31)) & 1u);
         p->seq_gen[b] = gen;
         // generated tokens before this step's (a token an eviction already appended is not counted)
         p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b] - (appended && (*appended)[b] ? 1 : 0);
@@ -317,8 +323,9 @@ double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
     return rows * kRowBytes;
 }
 
-// One eviction round of the triggered sequences in p: [score passes,] select, compact.
-int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s)
+// One eviction round of the triggered sequences in p: [score passes,] select, compact (unless
+// the caller's attention launch does the compaction).
+int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention = false)
 {
     cudaError_t e;
     if (p.policy == RA_POLICY_SNAPKV) {  // window scores with the normalisers recorded at decode time
@@ -339,7 +346,7 @@ int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s)
         ps.done();
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "select launch");
-    if (p.holefill) return RA_OK;  // the select kernel refilled the evicted slots in place
+    if (p.holefill || compact_in_attention) return RA_OK;  // done by select / by the attention launch
     {
         ProfScope ps(ctx, RA_KERNEL_COMPACT, moved * 2.0 * (2 * kRowBytes + 4), s);
         e = launch_compact(p, s);
@@ -630,7 +637,7 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block)
 int ra_set_compaction(ra_ctx* ctx, int mode)
 {
     if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
-    if (mode != RA_COMPACT_ORDERED && mode != RA_COMPACT_HOLEFILL)
+    if (mode != RA_COMPACT_ORDERED && mode != RA_COMPACT_HOLEFILL && mode != RA_COMPACT_FUSED)
         return fail(ctx, RA_ERR_INVALID_ARG, "unknown compaction %d", mode);
     if (mode == RA_COMPACT_HOLEFILL && ctx->policy == RA_POLICY_SNAPKV)
         return fail(ctx, RA_ERR_UNSUPPORTED, "the scored policy needs ordered compaction");
@@ -811,8 +818,13 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
     std::vector<uint8_t> appended((size_t)ctx->B, 0);  // sequences whose token the eviction wrote
+    std::vector<int32_t> old_rows((size_t)ctx->B, -1);  // sequences the attention launch compacts: rows before
+    // The attention pass compacts (time order kept) when each tile's evicted rows fit its 64-bit mask.
+    const bool fuse_compaction = ctx->compaction == RA_COMPACT_FUSED && ctx->r <= 64 && attn_tile_rows(ctx->G) == 64;
     // 1. Eviction first, with the step's token pending: it is the newest slot, so it is never a
     //    candidate, and evicting before writing it gives the same state as append-then-evict.
+    //    With ordered compaction only the selection runs here: the attention pass below reads
+    //    the old region anyway and writes the survivors to the new one as it goes.
     EvictParams ep{};
     ep.lay = ctx->lay;
     ep.layer = layer;
@@ -837,9 +849,10 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
             moved += (double)(ctx->K + ctx->r - 1) * ctx->KVH;
         }
     }
+    double compacted = 0;  // rows the attention launch writes as compaction
     if (n > 0) {
         ep.n_trig = n;
-        if ((rc = run_eviction(ctx, ep, moved, s)) != RA_OK) return rc;
+        if ((rc = run_eviction(ctx, ep, moved, s, fuse_compaction)) != RA_OK) return rc;
         for (int i = 0; i < n; ++i) {
             const int b = ep.trig[i];
             ctx->nev[base + b] += 1;
@@ -848,6 +861,10 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
                 ctx->g[base + b] += 1;
                 appended[b] = 1;
             } else {
+                if (fuse_compaction) {
+                    old_rows[b] = ep.trig_c[i];
+                    compacted += (double)(ctx->K + ctx->r) * ctx->KVH;
+                }
                 ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written
             }
         }
@@ -866,7 +883,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     p.ring_off = 0;  // the query of step g + 1
     int n_active = 0, ctas = 0;
     double rows = 0;
-    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &appended)) != RA_OK) return rc;
+    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &appended, &old_rows)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
     // The kernel may request its first K/V tiles before its predecessor finishes when that
@@ -879,9 +896,10 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
         // rows read (a new token's from the caller), a new token's row written, q read, out written
         int n_pending = 0;
         for (int b = 0; b < ctx->B; ++b) n_pending += (int)((p.pending[b >> 5] >> (b & 31)) & 1u);
+        // (a compacting head's survivors are written once more, with their positions)
         ProfScope ps(ctx, RA_KERNEL_ATTN,
                      rows * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes +
-                         (double)n_pending * ctx->KVH * 2 * kRowBytes,
+                         (double)n_pending * ctx->KVH * 2 * kRowBytes + compacted * (2 * kRowBytes + 8),
                      s);
         e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
         ps.done();

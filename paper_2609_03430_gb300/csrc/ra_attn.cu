@@ -44,6 +44,7 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <limits.h>
 #include <math.h>
 #include <stdint.h>
 
@@ -95,7 +96,7 @@ struct Cfg {
 };
 
 // Tile header flags; the chunk index sits above them (<< kFlagBits).
-constexpr int kFirst = 1, kLast = 2, kNewTok = 4, kHead0 = 8, kFlagBits = 4;
+constexpr int kFirst = 1, kLast = 2, kNewTok = 4, kHead0 = 8, kCompact = 16, kFlagBits = 5;
 
 // Producer-side walk over the warp's chunks (chunks and cursors count tiles).
 struct TileIter {
@@ -104,6 +105,7 @@ struct TileIter {
     int b, h, k;                     // current sequence, KV head, tile within the head
     int nt, tp;                      // tiles in the head, prompt tiles among them
     int lp, gen;                     // prompt rows, generated rows (incl. a fused new token)
+    bool comp;                       // the head compacts in this launch: its generated rows are the old region's
     long long prow, grow;            // first prompt row / first generated row of the head
     bool piece_start;
 };
@@ -118,6 +120,7 @@ __device__ __forceinline__ int seq_head_tiles(const AttnParams& p, int b)
     return (p.seq_base[b + 1] - p.seq_base[b]) / p.lay.KVH;
 }
 
+template <bool COMPACT>
 __device__ __forceinline__ void enter_head(TileIter& it, const AttnParams& p)
 {
     const DevLayout& L = p.lay;
@@ -125,11 +128,14 @@ __device__ __forceinline__ void enter_head(TileIter& it, const AttnParams& p)
     it.gen = p.seq_gen[it.b];
     it.tp = (it.lp + p.tile - 1) / p.tile;
     it.prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[it.b] + (long long)it.h * it.lp;
-    const int reg = L.region[((size_t)p.layer * L.B + it.b) * L.KVH + it.h];
+    it.comp = COMPACT && ((p.compacting[it.b >> 5] >> (it.b & 31)) & 1u);
+    const int reg = it.comp ? L.plan[(size_t)(it.b * L.KVH + it.h) * (kPlanHeader + L.r)]  // the old region
+                            : L.region[((size_t)p.layer * L.B + it.b) * L.KVH + it.h];
     it.grow = L.gen_row0 + (long long)reg * L.Cmax;
     it.piece_start = true;
 }
 
+template <bool COMPACT>
 __device__ void iter_init(TileIter& it, const AttnParams& p, int R0, int R1)
 {
     it.f = R0;
@@ -146,22 +152,24 @@ __device__ void iter_init(TileIter& it, const AttnParams& p, int R0, int R1)
     const int off = R0 - p.seq_base[b];
     it.h = off / it.nt;
     it.k = off - it.h * it.nt;
-    enter_head(it, p);
+    enter_head<COMPACT>(it, p);
 }
 
 // The warp's chunk (its index): false once it is done.
+template <bool COMPACT>
 __device__ bool iter_next_chunk(TileIter& it, const AttnParams& p, int warp_id)
 {
     if (it.chunk >= 0 || warp_id >= p.nchunks) return false;
     it.chunk = warp_id;
     const int R0 = warp_id * p.W;
-    iter_init(it, p, R0, min(p.total, R0 + p.W));
+    iter_init<COMPACT>(it, p, R0, min(p.total, R0 + p.W));
     return true;
 }
 
+template <bool COMPACT>
 __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int warp_id)
 {
-    if (it.f >= it.end && !iter_next_chunk(it, p, warp_id)) return false;
+    if (it.f >= it.end && !iter_next_chunk<COMPACT>(it, p, warp_id)) return false;
     const int T = p.tile;
     d.flags = (it.piece_start ? kFirst : 0) | (it.k == 0 ? kHead0 : 0);
     if (it.k < it.tp) {
@@ -173,6 +181,7 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int wa
         d.n = min(T, it.gen - kg * T);
         if (p.k_new && ((p.pending[it.b >> 5] >> (it.b & 31)) & 1u) && kg * T + d.n == it.gen)
             d.flags |= kNewTok;  // its last row is the step's new token
+        if (COMPACT && it.comp) d.flags |= kCompact;
     }
     if (it.k + 1 == it.nt || it.f + 1 == it.end) d.flags |= kLast;
     d.hid = it.b * p.lay.KVH + it.h;
@@ -189,7 +198,7 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int wa
             it.nt = seq_head_tiles(p, it.b);
         }
         it.k = 0;
-        enter_head(it, p);
+        enter_head<COMPACT>(it, p);
     }
     return true;
 }
@@ -324,7 +333,9 @@ __device__ void merge_head(const AttnParams& p, int hid, int c0, int P, int lane
     }
 }
 
-template <int G>
+// COMPACT: the launch also does the compaction of the heads in p.compacting (a separate
+// instantiation, so that launches without it run code free of its branches and registers).
+template <int G, bool COMPACT>
 __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
     attn_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tk,
                 const __grid_constant__ CUtensorMap tv)
@@ -378,7 +389,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
     };
     auto issue = [&](int t, bool inputs) -> bool {
         TileDesc d;
-        if (!iter_next(it, p, d, gw)) return false;
+        if (!iter_next<COMPACT>(it, p, d, gw)) return false;
         const int s = t % C::SPW;
         if (lane == 0) {
             uint8_t* st = wstage + (size_t)s * C::STAGE_BYTES;
@@ -447,14 +458,32 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
                 for (int i = lane; i < G * 16; i += 32) dst[i] = lds128(Qs + i * 16);
             }
         }
+        // A tile of a head that compacts in this launch: which of its rows were evicted (a 64-bit
+        // mask, from the ascending list of at most 64 evicted ordinals) and how many before it.
+        uint32_t ev_lo = 0u, ev_hi = 0u;
+        int ev_before = 0, j0 = 0;
+        if (COMPACT && (hd.y & kCompact)) {
+            const int32_t* plan = p.lay.plan + (size_t)hd.z * (kPlanHeader + p.lay.r);
+            const int m = plan[3];
+            j0 = (int)((long long)hd.w - p.lay.gen_row0 - (long long)plan[0] * p.lay.Cmax);
+            const int e0 = lane < m ? plan[kPlanHeader + lane] - j0 : INT_MAX;
+            const int e1 = lane + 32 < m ? plan[kPlanHeader + 32 + lane] - j0 : INT_MAX;
+            ev_before = __popc(__ballot_sync(0xffffffffu, e0 < 0)) + __popc(__ballot_sync(0xffffffffu, e1 < 0));
+            const uint32_t lo = ((e0 >= 0 && e0 < 32) ? 1u << e0 : 0u) | ((e1 >= 0 && e1 < 32) ? 1u << e1 : 0u);
+            const uint32_t hi = ((e0 >= 32 && e0 < 64) ? 1u << (e0 - 32) : 0u) | ((e1 >= 32 && e1 < 64) ? 1u << (e1 - 32) : 0u);
+            ev_lo = __reduce_or_sync(0xffffffffu, lo);
+            ev_hi = __reduce_or_sync(0xffffffffu, hi);
+        }
         if (hd.y & kNewTok) {  // fused append: put the new token in row n-1 of the tile and into the cache
             const int b = hd.z / p.lay.KVH;
             const int c = lane & 15;
             const uint4 v = lds128(Ks + C::NT_OFF + (lane >> 4) * kRowBytes + c * 16);
             *reinterpret_cast<uint4*>((lane < 16 ? Ks : Vs) + swz<G>(n - 1, c)) = v;
-            const long long row = (long long)hd.w + n - 1;
-            reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[c] = v;
-            if (lane == 0) p.lay.pos[row - p.lay.gen_row0] = p.lay.seq_lp[b] + p.seq_g[b];
+            if (!(COMPACT && (hd.y & kCompact))) {  // (a compacting head writes it with its survivors)
+                const long long row = (long long)hd.w + n - 1;
+                reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[c] = v;
+                if (lane == 0) p.lay.pos[row - p.lay.gen_row0] = p.lay.seq_lp[b] + p.seq_g[b];
+            }
             __syncwarp();
         }
         if (n < C::TILE) {  // rows past the valid ones hold stale data: zero V there so 0 * V stays 0
@@ -481,6 +510,12 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             const float sl = p.qk_scale_log2;
             float sc[4] = {r0 < n ? s0a * sl : -INFINITY, r0 + 1 < n ? s0b * sl : -INFINITY,
                            r0 + 8 < n ? s1a * sl : -INFINITY, r0 + 9 < n ? s1b * sl : -INFINITY};
+            if (COMPACT && (hd.y & kCompact)) {  // evicted rows get no weight
+                const int rr[4] = {r0, r0 + 1, r0 + 8, r0 + 9};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (((rr[e] < 32 ? ev_lo >> rr[e] : ev_hi >> (rr[e] - 32)) & 1u)) sc[e] = -INFINITY;
+            }
             float bm = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
             bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 1));
             bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 2));
@@ -498,7 +533,9 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             }
             float pr[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) pr[e] = exp2f(sc[e] - m_run);  // masked rows: exp2(-inf) = 0
+            // masked rows: exp2(-inf) = 0; a compacting head can have a whole batch evicted, with
+            // m_run still -inf (the difference would be NaN), so there a masked row weighs 0 outright
+            for (int e = 0; e < 4; ++e) pr[e] = (COMPACT && sc[e] == -INFINITY) ? 0.f : exp2f(sc[e] - m_run);
             l_run += (pr[0] + pr[1]) + (pr[2] + pr[3]);
             const uint32_t pa0 = pack_bf16x2(pr[0], pr[1]), pa2 = pack_bf16x2(pr[2], pr[3]);
             // O += P V: 16 n-tiles of 8 channels, k = the 16 rows
@@ -556,6 +593,36 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             for (int nt = 0; nt < 16; ++nt) O[nt][0] = O[nt][1] = 0.f;
         }
 
+        if (COMPACT && (hd.y & kCompact)) {
+            // Compaction fused into the pass: every surviving row of the tile (the new token
+            // included) goes from the staged tile to its slot in the new region, ordinal
+            // j - (evicted before j); positions follow.  One row per step, 16-byte lanes
+            // (0-15: K, 16-31: V).
+            const int32_t* plan = p.lay.plan + (size_t)hd.z * (kPlanHeader + p.lay.r);
+            const long long drow0 = p.lay.gen_row0 + (long long)plan[1] * p.lay.Cmax;
+            const int32_t* spos = p.lay.pos + (size_t)plan[0] * p.lay.Cmax;
+            int32_t* dpos = p.lay.pos + (size_t)plan[1] * p.lay.Cmax;
+            const int c = lane & 15;
+            uint16_t* pool = lane < 16 ? p.lay.kpool : p.lay.vpool;
+            const uint8_t* tile = lane < 16 ? Ks : Vs;
+            auto evicted = [&](int jj) { return ((jj < 32 ? ev_lo >> jj : ev_hi >> (jj - 32)) & 1u) != 0u; };
+            auto dest = [&](int jj) {
+                const int below = jj < 32 ? __popc(ev_lo & ((1u << jj) - 1u))
+                                          : __popc(ev_lo) + __popc(ev_hi & ((1u << (jj - 32)) - 1u));
+                return j0 + jj - ev_before - below;
+            };
+            for (int jj = 0; jj < n; ++jj) {
+                if (evicted(jj)) continue;
+                reinterpret_cast<uint4*>(pool + (drow0 + dest(jj)) * kHeadDim)[c] = lds128(tile + swz<G>(jj, c));
+            }
+            for (int jj = lane; jj < n; jj += 32) {
+                if (evicted(jj)) continue;
+                const int b = hd.z / p.lay.KVH;
+                const bool newtok = (hd.y & kNewTok) && jj == n - 1;
+                dpos[dest(jj)] = newtok ? p.lay.seq_lp[b] + p.seq_g[b] : __ldg(spos + j0 + jj);
+            }
+        }
+
         __syncwarp();
         if (more) {
             if (lane == 0) fence_proxy_async_smem();
@@ -582,13 +649,19 @@ template <int G>
 cudaError_t launch_attn_g(const AttnParams& p, const CUtensorMap* tk, const CUtensorMap* tv, int ctas, cudaStream_t s)
 {
     using C = Cfg<G>;
-    return launch_pdl(attn_kernel<G>, dim3(ctas), dim3(C::WARPS * 32), C::SMEM, s, p, *tk, *tv);
+    bool compact = false;
+    for (int i = 0; i < RA_MAX_BATCH / 32; ++i) compact |= p.compacting[i] != 0u;
+    if (compact) return launch_pdl(attn_kernel<G, true>, dim3(ctas), dim3(C::WARPS * 32), C::SMEM, s, p, *tk, *tv);
+    return launch_pdl(attn_kernel<G, false>, dim3(ctas), dim3(C::WARPS * 32), C::SMEM, s, p, *tk, *tv);
 }
 
 template <int G>
 cudaError_t prepare_g()
 {
-    return cudaFuncSetAttribute(attn_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<G>::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<G, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)Cfg<G>::SMEM);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(attn_kernel<G, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<G>::SMEM);
 }
 
 }  // namespace

@@ -107,6 +107,10 @@ struct AttnParams {
     int32_t seq_gen[RA_MAX_BATCH];       // generated rows attended per head (incl. a fused new token)
     int32_t seq_g[RA_MAX_BATCH];         // tokens generated before this step's (fused) / up to it (separate)
     uint32_t pending[RA_MAX_BATCH / 32]; // fused step: sequences whose new token this kernel appends
+    // fused step: sequences that evicted this step and whose compaction this kernel does -- it reads
+    // their old regions (plan header), masks the evicted rows and writes every survivor (and the new
+    // token) to its slot in the new region (time order kept)
+    uint32_t compacting[RA_MAX_BATCH / 32];
     uint16_t* qring;                     // record each head's query rows in the scored policy's window (or null)
     int ring_off;                        // window slot of sequence b = (seq_g[b] + ring_off) mod r
 };

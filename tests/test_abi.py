@@ -115,7 +115,7 @@ def test_compaction_mode_validation(ra):
         ra.ra_set_compaction(ctx, ra.RA_COMPACT_HOLEFILL)
     assert e.value.code == ra.RA_ERR_UNSUPPORTED
     with pytest.raises(ra.RAError) as e:
-        ra.ra_set_compaction(ctx, 2)
+        ra.ra_set_compaction(ctx, 3)
     assert e.value.code == ra.RA_ERR_INVALID_ARG
     ra.ra_destroy(ctx)
 
