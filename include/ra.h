@@ -214,6 +214,18 @@ int ra_restore_queries(ra_ctx* ctx, int layer, const uint16_t* q, float scale, v
 int ra_get_scores(ra_ctx* ctx, int layer, int seq, int kv_head, float* host_scores, int capacity, int* n,
                   void* stream);
 
+/*
+ * Tuning: the decode-attention kernel shape.  RA_ATTN_SHAPE_AUTO (default)
+ * picks per launch: layers attending fewer than 2^20 cache rows take the
+ * narrow shape (32-row tiles, 6 warps per SM: a finer split of a short layer),
+ * larger ones the wide shape (48-row tiles, 4 warps).  Outputs agree within
+ * fp32 rounding (the split, hence the summation order, differs).
+ */
+#define RA_ATTN_SHAPE_AUTO 0
+#define RA_ATTN_SHAPE_WIDE 1
+#define RA_ATTN_SHAPE_NARROW 2
+int ra_set_attention_shape(ra_ctx* ctx, int shape);
+
 /* Mark sequence `seq` active (1) or finished (0); finished ones are skipped by every call. */
 int ra_set_active(ra_ctx* ctx, int seq, int active);
 

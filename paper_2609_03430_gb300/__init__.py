@@ -43,6 +43,7 @@ SIGNATURES = {
     "ra_restore": (_i, [_vp, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp]),
     "ra_set_policy": (_i, [_vp, _i, _i]),
     "ra_set_compaction": (_i, [_vp, _i]),
+    "ra_set_attention_shape": (_i, [_vp, _i]),
     "ra_restore_queries": (_i, [_vp, _i, _vp, ctypes.c_float, _vp]),
     "ra_get_scores": (_i, [_vp, _i, _i, _i, ctypes.POINTER(ctypes.c_float), _i, _ip, _vp]),
     "ra_set_active": (_i, [_vp, _i, _i]),
@@ -146,6 +147,13 @@ def ra_set_policy(ctx, policy, block=1):
 
 
 RA_COMPACT_ORDERED, RA_COMPACT_HOLEFILL, RA_COMPACT_FUSED = 0, 1, 2
+
+
+RA_ATTN_SHAPE_AUTO, RA_ATTN_SHAPE_WIDE, RA_ATTN_SHAPE_NARROW = 0, 1, 2
+
+
+def ra_set_attention_shape(ctx, shape):
+    return _check(lib().ra_set_attention_shape(ctx, int(shape)), ctx)
 
 
 def ra_set_compaction(ctx, mode):

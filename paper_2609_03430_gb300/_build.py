@@ -15,6 +15,14 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libra.so")
 SOURCES = ["ra_api.cu", "ra_evict.cu", "ra_attn.cu", "ra_score.cu"]
+# (source, object, extra flags): the attention file is built twice, once per kernel shape.
+UNITS = [
+    ("ra_api.cu", "ra_api.o", []),
+    ("ra_evict.cu", "ra_evict.o", []),
+    ("ra_attn.cu", "ra_attn_wide.o", ["-DRA_ATTN_NS=attn_wide", "-DRA_ATTN_TILE=48", "-DRA_ATTN_WARPS=4"]),
+    ("ra_attn.cu", "ra_attn_narrow.o", ["-DRA_ATTN_NS=attn_narrow", "-DRA_ATTN_TILE=32", "-DRA_ATTN_WARPS=6"]),
+    ("ra_score.cu", "ra_score.o", []),
+]
 HEADERS = ["ra_internal.h", "ra_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include"), "-I" + CSRC]
@@ -34,12 +42,12 @@ def needs_build() -> bool:
 
 
 def compile_procs():
-    """Start one nvcc per translation unit; returns [(popen, object path)]."""
+    """Start one nvcc per translation unit; returns [(popen, object path, command)]."""
     os.makedirs(BUILD, exist_ok=True)
     procs = []
-    for s in SOURCES:
-        obj = os.path.join(BUILD, s.replace(".cu", ".o"))
-        cmd = ["nvcc", *ARCH, *FLAGS, *EXTRA, "-c", os.path.join(CSRC, s), "-o", obj]
+    for src, obj_name, unit_flags in UNITS:
+        obj = os.path.join(BUILD, obj_name)
+        cmd = ["nvcc", *ARCH, *FLAGS, *unit_flags, *EXTRA, "-c", os.path.join(CSRC, src), "-o", obj]
         procs.append((subprocess.Popen(cmd), obj, cmd))
     return procs
 

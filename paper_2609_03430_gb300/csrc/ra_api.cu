@@ -64,7 +64,7 @@ struct ra_ctx {
     int sms = 0;
     uint8_t* arena = nullptr;
     DevLayout lay{};
-    CUtensorMap tmap_k{}, tmap_v{};
+    CUtensorMap tmap_k[kAttnShapes]{}, tmap_v[kAttnShapes]{};  // per attention shape (tile rows)
     CUtensorMap tmap_ks{};  // kpool in kScoreTile-row boxes (scoring kernels)
     CUtensorMap tmap_q{};   // the query windows as [L*B*KVH*r*G][128] rows, same boxes
     // host mirror
@@ -73,6 +73,7 @@ struct ra_ctx {
     int policy = RA_POLICY_RANDOM;   // candidate scoring (ra_set_policy)
     int block = 1;
     int compaction = RA_COMPACT_ORDERED;  // ra_set_compaction
+    int attn_shape = RA_ATTN_SHAPE_AUTO;  // ra_set_attention_shape
     std::vector<int32_t> score_n;    // [L][B] candidates of the latest scored round
     // profiling
     bool prof = false;
@@ -220,7 +221,8 @@ void fill_active(const ra_ctx* ctx, uint32_t* mask)
 // the cached generated rows plus one for a fused new token; the tiles are cut into one equal
 // chunk per warp.  *slots = rows attended.
 int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots,
-                   const std::vector<uint8_t>* appended = nullptr, const std::vector<int32_t>* old_rows = nullptr)
+                   int* shape, const std::vector<uint8_t>* appended = nullptr,
+                   const std::vector<int32_t>* old_rows = nullptr)
 {
     fill_active(ctx, p->active);
     // sequences whose compaction the launch does: their cached rows are the old region's
@@ -233,11 +235,8 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     if (fused && appended)
         for (int b = 0; b < ctx->B; ++b)
             if ((*appended)[b]) p->pending[b >> 5] &= ~(1u << (b & 31));
-    const int T = attn_tile_rows(ctx->G);
-    p->tile = T;
     long long acc = 0, rows = 0;
     int na = 0;
-    p->seq_base[0] = 0;
     for (int b = 0; b < ctx->B; ++b) {
         const int cached = (old_rows && (*old_rows)[b] >= 0) ? (*old_rows)[b] : ctx->c[(size_t)layer * ctx->B + b];
         const int gen = cached + (int)((p->pending[b >> 5] >> (b & 31)) & 1u);
@@ -245,15 +244,24 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
         // generated tokens before this step's (a token an eviction already appended is not counted)
         p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b] - (appended && (*appended)[b] ? 1 : 0);
         if (ctx->active[b]) {
-            acc += (long long)ctx->KVH * ((ctx->lp[b] + T - 1) / T + (gen + T - 1) / T);
             rows += (long long)ctx->KVH * (ctx->lp[b] + gen);
             ++na;
         }
+    }
+    *shape = ctx->attn_shape == RA_ATTN_SHAPE_WIDE     ? kAttnWide
+             : ctx->attn_shape == RA_ATTN_SHAPE_NARROW ? kAttnNarrow
+             : rows < kNarrowRows                      ? kAttnNarrow
+                                                       : kAttnWide;
+    const int T = attn_tile_rows(*shape, ctx->G);
+    p->tile = T;
+    p->seq_base[0] = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        if (ctx->active[b]) acc += (long long)ctx->KVH * ((ctx->lp[b] + T - 1) / T + (p->seq_gen[b] + T - 1) / T);
         p->seq_base[b + 1] = (int32_t)acc;
     }
     if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 tiles");
     p->total = (int)acc;
-    const int wpc = attn_warps_per_cta(ctx->G);
+    const int wpc = attn_warps_per_cta(*shape, ctx->G);
     const long long nwarps_max = (long long)ctx->sms * wpc;
     const long long W = std::max<long long>(1, (acc + nwarps_max - 1) / nwarps_max);
     const long long nchunks = (acc + W - 1) / W;
@@ -431,7 +439,8 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_poff = take((size_t)batch * 4);
     ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
     // chunks of the attention split: one per warp
-    const size_t max_chunks = (size_t)kMaxSMs * attn_warps_per_cta(ctx->G) + 1;
+    const size_t max_chunks =
+        (size_t)kMaxSMs * std::max(attn_warps_per_cta(kAttnWide, ctx->G), attn_warps_per_cta(kAttnNarrow, ctx->G)) + 1;
     ctx->partial_records = max_chunks + (size_t)batch * kv_heads;
     ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);
@@ -533,11 +542,13 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
         return cuda_fail(ctx, e, "query window clear");
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(ctx, e, "table initialisation sync");
 
-    const int tile = attn_tile_rows(ctx->G);
     int rc;
-    if ((rc = make_tmap(ctx, &ctx->tmap_k, Ly.kpool, ctx->total_rows, tile)) != RA_OK) return rc;
-    if ((rc = make_tmap(ctx, &ctx->tmap_v, Ly.vpool, ctx->total_rows, tile)) != RA_OK) return rc;
-    if ((e = attn_prepare(ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
+    for (int sh = 0; sh < kAttnShapes; ++sh) {
+        const int tile = attn_tile_rows(sh, ctx->G);
+        if ((rc = make_tmap(ctx, &ctx->tmap_k[sh], Ly.kpool, ctx->total_rows, tile)) != RA_OK) return rc;
+        if ((rc = make_tmap(ctx, &ctx->tmap_v[sh], Ly.vpool, ctx->total_rows, tile)) != RA_OK) return rc;
+        if ((e = attn_prepare(sh, ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
+    }
     if (ctx->scoring) {
         if ((rc = make_tmap(ctx, &ctx->tmap_ks, Ly.kpool, ctx->total_rows, kScoreTile)) != RA_OK) return rc;
         const long long win_rows = (long long)ctx->L * ctx->B * ctx->KVH * ctx->r * ctx->G;
@@ -642,6 +653,15 @@ int ra_set_compaction(ra_ctx* ctx, int mode)
     if (mode == RA_COMPACT_HOLEFILL && ctx->policy == RA_POLICY_SNAPKV)
         return fail(ctx, RA_ERR_UNSUPPORTED, "the scored policy needs ordered compaction");
     ctx->compaction = mode;
+    return RA_OK;
+}
+
+int ra_set_attention_shape(ra_ctx* ctx, int shape)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (shape < RA_ATTN_SHAPE_AUTO || shape > RA_ATTN_SHAPE_NARROW)
+        return fail(ctx, RA_ERR_INVALID_ARG, "unknown attention shape %d", shape);
+    ctx->attn_shape = shape;
     return RA_OK;
 }
 
@@ -791,12 +811,13 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     int n_active = 0;
     int ctas = 0;
     double rows = 0;
-    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
+    int shape = kAttnWide;
+    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows, &shape)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
     cudaStream_t s = (cudaStream_t)stream;
     ProfScope ps(ctx, RA_KERNEL_ATTN, rows * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes, s);
-    cudaError_t e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+    cudaError_t e = launch_attention(shape, p, &ctx->tmap_k[shape], &ctx->tmap_v[shape], ctas, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
     return RA_OK;
@@ -820,7 +841,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     std::vector<uint8_t> appended((size_t)ctx->B, 0);  // sequences whose token the eviction wrote
     std::vector<int32_t> old_rows((size_t)ctx->B, -1);  // sequences the attention launch compacts: rows before
     // The attention pass compacts (time order kept) when each tile's evicted rows fit its 64-bit mask.
-    const bool fuse_compaction = ctx->compaction == RA_COMPACT_FUSED && ctx->r <= 64 && attn_tile_rows(ctx->G) == 64;
+    const bool fuse_compaction = ctx->compaction == RA_COMPACT_FUSED && ctx->r <= 64;  // tiles have <= 64 rows
     // 1. Eviction first, with the step's token pending: it is the newest slot, so it is never a
     //    candidate, and evicting before writing it gives the same state as append-then-evict.
     //    With ordered compaction only the selection runs here: the attention pass below reads
@@ -883,7 +904,9 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     p.ring_off = 0;  // the query of step g + 1
     int n_active = 0, ctas = 0;
     double rows = 0;
-    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &appended, &old_rows)) != RA_OK) return rc;
+    int shape = kAttnWide;
+    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &shape, &appended, &old_rows)) != RA_OK)
+        return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
     // The kernel may request its first K/V tiles before its predecessor finishes when that
@@ -901,7 +924,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
                      rows * 2 * kRowBytes + 2.0 * n_active * ctx->H * kRowBytes +
                          (double)n_pending * ctx->KVH * 2 * kRowBytes + compacted * (2 * kRowBytes + 8),
                      s);
-        e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+        e = launch_attention(shape, p, &ctx->tmap_k[shape], &ctx->tmap_v[shape], ctas, s);
         ps.done();
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
@@ -1139,7 +1162,8 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     p.ring_off = -1;
     int n_active = 0, ctas = 0;
     double rows = 0;
-    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows)) != RA_OK) return rc;
+    int shape = kAttnWide;
+    if ((rc = plan_attention(ctx, layer, 0, &p, &n_active, &ctas, &rows, &shape)) != RA_OK) return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
     // [arrival counters, one int per (seq, KV head)][partial records, one per (chunk, head) piece]
@@ -1157,7 +1181,7 @@ extern "C" int ra_decode_attn_noalloc(ra_ctx* ctx, int layer, const uint16_t* q,
     // the counters must start at zero; the array keeps whatever the previous call left
     cudaError_t e = cudaMemsetAsync(scratch, 0, counters, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "scratch counter clear");
-    e = launch_attention(p, &ctx->tmap_k, &ctx->tmap_v, ctas, s);
+    e = launch_attention(shape, p, &ctx->tmap_k[shape], &ctx->tmap_v[shape], ctas, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
     return RA_OK;
 }

@@ -60,15 +60,20 @@ constexpr int kSmemBudget = 220 * 1024;
 constexpr int kHalfCh = 64;                        // channels per swizzled TMA box (128 bytes)
 
 // Kernel shape: rows per stage (a multiple of 16), stages per warp, warps per CTA
-// (one CTA per SM; the warp count is capped by what fits in shared memory).
+// (one CTA per SM; the warp count is capped by what fits in shared memory).  The library
+// builds this file twice, into the namespaces attn_wide (48-row tiles, 4 warps: large
+// layers) and attn_narrow (32-row tiles, 6 warps: small layers, finer work split).
+#ifndef RA_ATTN_NS
+#define RA_ATTN_NS attn_wide
+#endif
 #ifndef RA_ATTN_TILE
-#define RA_ATTN_TILE 64
+#define RA_ATTN_TILE 48
 #endif
 #ifndef RA_ATTN_SPW
 #define RA_ATTN_SPW 2
 #endif
 #ifndef RA_ATTN_WARPS
-#define RA_ATTN_WARPS 3
+#define RA_ATTN_WARPS 4
 #endif
 
 template <int G>
@@ -666,6 +671,8 @@ cudaError_t prepare_g()
 
 }  // namespace
 
+namespace RA_ATTN_NS {
+
 int attn_warps_per_cta(int G)
 {
     switch (G) {
@@ -735,4 +742,5 @@ cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tk, const C
     return cudaErrorInvalidValue;
 }
 
+}  // namespace RA_ATTN_NS
 }  // namespace ra

@@ -144,12 +144,44 @@ cudaError_t launch_score_merge(const EvictParams& p, cudaStream_t s);
 cudaError_t score_prepare();
 int score_row_tiles_per_warp(int M);  // 16-row tiles of the M window rows per warp (1..4)
 
-// Attention: the tensor maps cover kpool / vpool as [total_rows][128] bf16.
-int attn_warps_per_cta(int G);
-int attn_tile_rows(int G);
-cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tmap_k, const CUtensorMap* tmap_v, int ctas,
-                             cudaStream_t s);
-cudaError_t attn_prepare(int G);  // one-time function attributes (dynamic smem)
+// Attention comes in two kernel shapes, one build of ra_attn.cu each: wide (48-row tiles, 4 warps
+// per CTA) for large layers and narrow (32-row tiles, 6 warps) for small ones, where a finer split
+// of a short layer across more warps shortens its tail.  The tensor maps cover kpool / vpool as
+// [total_rows][128] bf16 in boxes of the shape's tile rows.
+#define RA_ATTN_API                                                                                        \
+    int attn_warps_per_cta(int G);                                                                         \
+    int attn_tile_rows(int G);                                                                             \
+    cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tmap_k, const CUtensorMap* tmap_v, \
+                                 int ctas, cudaStream_t s);                                                \
+    cudaError_t attn_prepare(int G); /* one-time function attributes (dynamic smem) */
+namespace attn_wide { RA_ATTN_API }
+namespace attn_narrow { RA_ATTN_API }
+#undef RA_ATTN_API
+
+enum AttnShape { kAttnWide = 0, kAttnNarrow = 1, kAttnShapes = 2 };
+#ifndef RA_ATTN_NARROW_ROWS
+#define RA_ATTN_NARROW_ROWS (1 << 20)
+#endif
+constexpr long long kNarrowRows = RA_ATTN_NARROW_ROWS;  // layers attending fewer rows take the narrow shape
+
+inline int attn_warps_per_cta(int shape, int G)
+{
+    return shape == kAttnNarrow ? attn_narrow::attn_warps_per_cta(G) : attn_wide::attn_warps_per_cta(G);
+}
+inline int attn_tile_rows(int shape, int G)
+{
+    return shape == kAttnNarrow ? attn_narrow::attn_tile_rows(G) : attn_wide::attn_tile_rows(G);
+}
+inline cudaError_t launch_attention(int shape, const AttnParams& p, const CUtensorMap* tk, const CUtensorMap* tv,
+                                    int ctas, cudaStream_t s)
+{
+    return shape == kAttnNarrow ? attn_narrow::launch_attention(p, tk, tv, ctas, s)
+                                : attn_wide::launch_attention(p, tk, tv, ctas, s);
+}
+inline cudaError_t attn_prepare(int shape, int G)
+{
+    return shape == kAttnNarrow ? attn_narrow::attn_prepare(G) : attn_wide::attn_prepare(G);
+}
 
 // Launch with programmatic dependent launch: the kernel may be scheduled while its
 // predecessor on the stream finishes.  Every kernel waits (griddepcontrol.wait)

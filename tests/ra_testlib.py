@@ -59,7 +59,7 @@ class Runner:
     """A small workload run through the C ABI with an oracle mirror of every head."""
 
     def __init__(self, L, H, KVH, prompt_lens, K, r, eseed, dseed, key_scale=None, D=128, fused=False, policy=0,
-                 block=1, compaction=0):
+                 block=1, compaction=0, attn_shape=0):
         import torch
 
         import paper_2609_03430_gb300 as ra
@@ -74,6 +74,8 @@ class Runner:
         self.cache = ra.RandomAttentionCache(L, H, KVH, D, self.lp, K, r, eseed, policy=policy, block=block,
                                              compaction=compaction)
         self.ctx = self.cache.ctx
+        if attn_shape:
+            ra.ra_set_attention_shape(self.ctx, attn_shape)
         self.orc = oracle.OracleCache(L, KVH, self.lp, K, r, eseed, policy=policy, block=block, compaction=compaction)
         self.policy = policy
         self.qsteps = [[] for _ in range(self.B)]  # step index of each of a sequence's decode steps

@@ -45,9 +45,12 @@ def test_ragged_batch_layers_and_finishing(fused):
     run.close()
 
 
+@pytest.mark.parametrize("shape", [1, 2], ids=["wide", "narrow"])
 @pytest.mark.parametrize("G", [1, 2, 3, 4, 6, 7, 8])
-def test_group_sizes(G):
-    run = Runner(L=1, H=2 * G, KVH=2, prompt_lens=[70, 1], K=48, r=16, eseed=G, dseed=10 + G, fused=G % 2 == 0)
+def test_group_sizes(G, shape):
+    """Every group size through both attention kernel shapes (48-row tiles x 4 warps, 32 x 6)."""
+    run = Runner(L=1, H=2 * G, KVH=2, prompt_lens=[70, 1], K=48, r=16, eseed=G, dseed=10 + G, fused=G % 2 == 0,
+                 attn_shape=shape)
     for step in range(150):
         fired = run.step(check_attn_layers=(0,) if step % 25 == 0 or step in (95, 96, 97) else ())
         if any(fired.values()):
