@@ -391,6 +391,8 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     if (!prompt_lens) return fail(nullptr, RA_ERR_INVALID_ARG, "prompt_lens is NULL");
     if (K < 0 || r < 1) return fail(nullptr, RA_ERR_INVALID_ARG, "need K >= 0 and r >= 1");
     if ((long long)K + r > kMaxCandidates) return fail(nullptr, RA_ERR_UNSUPPORTED, "K + r must be <= %d", kMaxCandidates);
+    if (select_smem(K + r, r, false) > kSelectSmemLimit)
+        return fail(nullptr, RA_ERR_UNSUPPORTED, "K + 2r too large for the selection's shared memory");
 
     ra_ctx* ctx = new ra_ctx();
     ctx->L = layers;
@@ -852,6 +854,11 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     ep.policy = ctx->policy;
     ep.block = ctx->block;
     ep.holefill = ctx->compaction == RA_COMPACT_HOLEFILL;
+    // The selection reads nothing its predecessor (the previous layer's attention) writes: Philox
+    // needs no input, and positions were last written by this layer's previous step, which has
+    // completed (every kernel before the predecessor has).  The scored policy reads scores its
+    // predecessor computes, and with one layer the predecessor is this layer's previous step.
+    ep.early = (ctx->policy != RA_POLICY_SNAPKV && ctx->L >= 2) ? 1 : 0;
     if (ep.holefill) {  // the token refills an evicted slot: the select kernel writes it
         ep.k_new = k_new;
         ep.v_new = v_new;

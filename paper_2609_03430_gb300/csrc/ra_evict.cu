@@ -85,8 +85,13 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     extern __shared__ uint32_t sm[];
     __shared__ uint32_t hist[3][256];
     __shared__ uint32_t s_total;
-    pdl_wait();
-    pdl_launch_dependents();
+    // With p.early the keys, the radix select and the evicted list are computed before waiting for
+    // the previous kernel (their inputs come from kernels that completed earlier); everything this
+    // kernel writes to global memory comes after the wait.
+    if (!p.early) {
+        pdl_wait();
+        pdl_launch_dependents();
+    }
     const DevLayout& L = p.lay;
     const int b = p.trig[blockIdx.x], h = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -98,6 +103,10 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     const int head_id = b * L.KVH + h;
     int32_t* plan = L.plan + (size_t)head_id * (kPlanHeader + r);
     if (m <= 0 || m > r || N > kMaxCandidates || N > c) {  // the host mirror rules this out; never move data on a bad plan
+        if (p.early) {
+            pdl_wait();
+            pdl_launch_dependents();
+        }
         if (tid == 0) {
             atomicExch(L.err, kDeviceErrPlan);
             plan[3] = 0;
@@ -105,8 +114,10 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         return;
     }
     const int nwords = (N + 31) >> 5;
-    uint32_t* keys = sm;                 // [N]
-    uint32_t* evbits = sm + nwords * 32; // [nwords]
+    uint32_t* keys = sm;                       // [N]
+    uint32_t* evbits = sm + nwords * 32;       // [nwords]
+    int32_t* s_ev = reinterpret_cast<int32_t*>(evbits + nwords);  // [r] evicted ordinals, ascending
+    // (under the scored policy the raw scores follow s_ev)
 
     if (tid < 256) hist[0][tid] = 0;  // the first digit's histogram (the fill's barrier publishes it)
     const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
@@ -129,7 +140,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         // scored comparator: the window score max-pooled over +-kScorePoolRadius candidates;
         // larger scores must sort first, so the key is the order-reversed float
         const float* sc = L.scores + (((size_t)p.layer * L.B + b) * L.KVH + h) * L.Cmax;
-        float* raw = reinterpret_cast<float*>(evbits + nwords);  // [N], staged once
+        float* raw = reinterpret_cast<float*>(s_ev + r);  // [N], staged once
 #pragma unroll 4
         for (int j = tid; j < N; j += kSelThreads) raw[j] = __ldcg(sc + j);
         __syncthreads();
@@ -260,7 +271,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
             while (bits) {
                 const int bit = __ffs(bits) - 1;
                 bits &= bits - 1;
-                if (pos < (uint32_t)r) plan[kPlanHeader + pos] = w * 32 + bit;
+                if (pos < (uint32_t)r) s_ev[pos] = w * 32 + bit;
                 ++pos;
             }
             off += __shfl_sync(0xffffffffu, incl, 31);
@@ -268,6 +279,11 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         if (lane == 0) s_total = off;
     }
     __syncthreads();
+    if (p.early) {
+        pdl_wait();
+        pdl_launch_dependents();
+    }
+    for (int i = tid; i < min((int)s_total, r); i += kSelThreads) plan[kPlanHeader + i] = s_ev[i];
     if (tid == 0) {
         const int32_t* regp = L.region + ((size_t)p.layer * L.B + b) * L.KVH + h;
         const int src = *regp, dst = p.holefill ? src : L.spare[b * L.KVH + h];  // hole-filling works in place
@@ -287,7 +303,6 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     // Order-free compaction, in place: evicted slot e_i takes the row of slot top - m + i, where
     // top is the slot count including a pending token (the newest slot, taken from the caller's
     // rows).  Those m <= r slots are all buffer slots, so sources and destinations never overlap.
-    __syncthreads();  // the evicted list (written by warp 0) and the header
     if (s_total != (uint32_t)m) return;
     const int top = p.k_new ? c + 1 : c;
     const long long row0 = L.gen_row0 + (long long)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
@@ -305,7 +320,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
             to[u] = -1;
             if (i < m) {
                 const int from = top - m + i;
-                to[u] = plan[kPlanHeader + i];
+                to[u] = s_ev[i];
                 if (from == c) {  // the step's pending token
                     const uint16_t* src = (lane < 16 ? p.k_new : p.v_new) + ((size_t)b * L.KVH + h) * kHeadDim;
                     v[u] = reinterpret_cast<const uint4*>(src)[part];
@@ -463,17 +478,18 @@ cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s)
     return launch_pdl(append_kernel, dim3(B), dim3(p.lay.KVH * 32), 0, s, p);
 }
 
-// keys [N rounded to 32], the evicted bitmap, and under the scored policy the raw scores [N]
-static size_t select_smem(int N, bool scored)
+// keys [N rounded to 32], the evicted bitmap, the evicted list [r], and under the scored policy
+// the raw scores [N]
+size_t select_smem(int N, int r, bool scored)
 {
     const size_t words = (size_t)(N + 31) / 32;
-    return (words * 32 + words + (scored ? words * 32 : 0)) * sizeof(uint32_t);
+    return (words * 32 + words + (size_t)r + (scored ? words * 32 : 0)) * sizeof(uint32_t);
 }
 
 cudaError_t launch_select(const EvictParams& p, cudaStream_t s)
 {
     const int N = p.lay.K + p.lay.r;  // candidates at a firing step never exceed K + r
-    const size_t smem = select_smem(N, p.policy == RA_POLICY_SNAPKV);
+    const size_t smem = select_smem(N, p.lay.r, p.policy == RA_POLICY_SNAPKV);
     static size_t configured = 0;
     if (smem > 48 * 1024 && smem > configured) {
         cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -65,6 +65,7 @@ struct EvictParams {
     int policy;    // RA_POLICY_*: how candidates are scored
     int block;     // RA_POLICY_BLOCK: positions per block
     int holefill;  // RA_COMPACT_HOLEFILL: keys per position, evicted slots refilled in place by select
+    int early;     // select may compute before its predecessor finishes (it writes only after the wait)
     // Fused step under hole-filling: the step's new rows [B][KVH][128] (the token is the newest slot
     // and always among those that refill the evicted ones); null when the token is already cached.
     const uint16_t* k_new;
@@ -128,6 +129,8 @@ struct CopyRowsParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s);
 cudaError_t launch_select(const EvictParams& p, cudaStream_t s);
+size_t select_smem(int N, int r, bool scored);  // dynamic shared memory of one select CTA
+constexpr size_t kSelectSmemLimit = 220 * 1024;
 cudaError_t launch_compact(const EvictParams& p, cudaStream_t s);
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s);
 cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s);
