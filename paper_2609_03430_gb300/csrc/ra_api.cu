@@ -333,14 +333,18 @@ double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
 
 // One eviction round of the triggered sequences in p: [score passes,] select, compact (unless
 // the caller's attention launch does the compaction).
-int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention = false)
+int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention = false,
+                 int score_early = 0)
 {
     cudaError_t e;
     if (p.policy == RA_POLICY_SNAPKV) {  // window scores with the normalisers recorded at decode time
         for (int i = 0; i < p.n_trig; ++i) ctx->score_n[(size_t)p.layer * ctx->B + p.trig[i]] = p.trig_n[i];
         const double bytes = plan_scoring(ctx, &p, 2);
         ProfScope ps(ctx, RA_KERNEL_SCORE_SUM, bytes, s);
+        const int select_early = p.early;
+        p.early = score_early;  // the scoring pass's own flag; the selection after it waits first
         e = launch_score(p, 2, &ctx->tmap_ks, &ctx->tmap_q, s);
+        p.early = select_early;
         ps.done();
         if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
     }
@@ -859,6 +863,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     // completed (every kernel before the predecessor has).  The scored policy reads scores its
     // predecessor computes, and with one layer the predecessor is this layer's previous step.
     ep.early = (ctx->policy != RA_POLICY_SNAPKV && ctx->L >= 2) ? 1 : 0;
+    const int score_early = ctx->L >= 2 ? 1 : 0;  // the scoring pass reads only older kernels' output
     if (ep.holefill) {  // the token refills an evicted slot: the select kernel writes it
         ep.k_new = k_new;
         ep.v_new = v_new;
@@ -880,7 +885,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     double compacted = 0;  // rows the attention launch writes as compaction
     if (n > 0) {
         ep.n_trig = n;
-        if ((rc = run_eviction(ctx, ep, moved, s, fuse_compaction)) != RA_OK) return rc;
+        if ((rc = run_eviction(ctx, ep, moved, s, fuse_compaction, score_early)) != RA_OK) return rc;
         for (int i = 0; i < n; ++i) {
             const int b = ep.trig[i];
             ctx->nev[base + b] += 1;

@@ -134,8 +134,14 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
     float* red = reinterpret_cast<float*>(smem + C::RED_OFF);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-    pdl_wait();  // the window, the cache and the tables come from earlier kernels
-    pdl_launch_dependents();
+    // The window, the cache and the tables come from earlier kernels.  With p.early (pass 2 inside
+    // the fused step) they were all written by kernels that completed before the predecessor (the
+    // previous layer's attention) started, and the scores are read only by the successor: the pass
+    // computes before waiting, and lets its successor start only after the wait, at its end.
+    if (!(PASS == 2 && p.early)) {
+        pdl_wait();
+        pdl_launch_dependents();
+    }
 
     const DevLayout& L = p.lay;
     const int t = blockIdx.y / L.KVH, h = blockIdx.y - t * L.KVH;
@@ -146,7 +152,7 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
     const int nt_head = head_tiles(PASS, lp, N, &tp);
     const int ch = PASS == 1 ? p.ch1 : p.ch2;
     const int t0 = blockIdx.x * ch;
-    if (t0 >= nt_head) return;
+    if (t0 >= nt_head) return;  // (exiting counts as letting the successor start)
     const int ntile = min(ch, nt_head - t0);
     const long long prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[b] + (long long)h * lp;
     const size_t lbh = ((size_t)p.layer * L.B + b) * L.KVH + h;
@@ -227,6 +233,7 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
                 for (int j = i + 1; j < ntile && j < i + kStages; ++j)
                     (void)mbar_wait_bounded(&bars[j % kStages], (uint32_t)((j / kStages) & 1), kWaitLimitNs);
             }
+            if (PASS == 2 && p.early) pdl_wait();  // the successor still starts only after the predecessor
             return;
         }
         const uint32_t ks = smem_u32(smem + (size_t)s * kTileBytes);
@@ -323,6 +330,10 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_kernel(const 
         }
     }
 
+    if (PASS == 2 && p.early) {
+        pdl_wait();
+        pdl_launch_dependents();
+    }
     if (PASS == 1) {  // this chunk's statistics of every real row
         float* out = L.stats + ((size_t)hid * L.stats_chunks + blockIdx.x) * M * 2;
 #pragma unroll
