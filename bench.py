@@ -427,6 +427,35 @@ def evented_steps(wl, steps, t_next):
     return kern, wl.evictions() - rounds0, t_next + steps
 
 
+def attention_window(wl, steps, t_next):
+    """Attention launch duration as the timed region runs it: `steps` more whole-stack steps with
+    CUDA events only at the step boundaries (on the launching stream), so the launches inside a
+    step keep the overlap they have in the timed region.  A step in which no sequence evicts
+    launches nothing but the attention kernel of every layer; those steps give the duration
+    (their device time / their attention launches) and bytes (the library's algorithmic count)."""
+    import torch
+
+    ra = wl.ra
+    kind = ra.KERNEL_NAMES.index("attn")
+
+    def evictions_layer0():  # the host mirror's counts; every layer of a sequence evicts on the same step
+        return sum(ra.ra_get_counters(wl.ctx, b, 0)[2] for b in range(wl.B))
+
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    marks = []
+    evs[0].record(wl.stream)
+    for i, t in enumerate(range(t_next, t_next + steps)):
+        n0 = evictions_layer0()
+        _, l0, b0 = ra.ra_profile_read(wl.ctx, kind)
+        wl.step(t)
+        evs[i + 1].record(wl.stream)
+        _, l1, b1 = ra.ra_profile_read(wl.ctx, kind)
+        marks.append((evictions_layer0() != n0, l1 - l0, b1 - b0))
+    torch.cuda.synchronize()
+    clean = [(evs[i].elapsed_time(evs[i + 1]), n, by) for i, (fired, n, by) in enumerate(marks) if not fired and n > 0]
+    return clean, t_next + steps
+
+
 def _eviction_us_per_round(kern, names, rounds):
     if not rounds:
         return None
@@ -529,8 +558,10 @@ def run_ours(args, w):
     clocks.stop()
     launches = sum(ra.ra_profile_read(ctx, kind)[1] for kind in range(len(ra.KERNEL_NAMES)))
 
-    # Kernel durations: the same number of steps again with CUDA events around every launch.
+    # Kernel durations: the same number of steps again with CUDA events around every launch ...
     kern, rounds, t_next = evented_steps(wl, args.steps, t_next)
+    # ... and once more with events only at the step boundaries (attention launches overlapped).
+    clean, t_next = attention_window(wl, args.steps, t_next)
 
     ms_step, units = reduce_over_ranks(ms, float(wl.B), world)
     value = units / (ms_step * 1e-3)
@@ -568,17 +599,30 @@ def run_ours(args, w):
     a = kern.get("attn")
     roof = None
     if a:
-        by_launch = a["bytes_per_launch"]
-        achieved = a["algorithmic_GBps"]
+        serialized = {"us_per_launch": a["us_per_launch"], "achieved": a["algorithmic_GBps"],
+                      "frac": a["algorithmic_GBps"] / peaks["hbm_gbs"],
+                      "timing": "CUDA events around every attention launch on its stream, in a second pass "
+                                "of the same number of steps (the events between launches defeat their "
+                                "overlap, so this duration is an upper bound)"}
+        if clean:
+            win_ms = sum(c[0] for c in clean)
+            win_n = sum(c[1] for c in clean)
+            by_launch = sum(c[2] for c in clean) / win_n
+            us_launch = 1000.0 * win_ms / win_n
+            timing = (f"CUDA events at the step boundaries on the launching stream, over the {len(clean)} of "
+                      f"{args.steps} steps of a third pass in which no sequence evicts: such a step launches "
+                      f"only the {w['L']} layers' attention kernels, overlapped as in the timed region; "
+                      f"duration = their device time / {win_n} launches")
+        else:  # every step evicts somewhere (ragged phases): the per-launch events are all there is
+            by_launch, us_launch, timing = a["bytes_per_launch"], a["us_per_launch"], serialized["timing"]
+        achieved = by_launch / (us_launch * 1e-6) / 1e9
         roof = {"kernel": "attn_kernel (split-K decode attention)", "bound": "hbm", "achieved": achieved,
                 "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
                 "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
                 else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
-                "algorithmic_bytes_per_launch": by_launch, "us_per_launch": a["us_per_launch"],
+                "algorithmic_bytes_per_launch": by_launch, "us_per_launch": us_launch,
                 "traffic": args.traffic if args.traffic is not None else profiled_traffic(args.config),
-                "timing": "CUDA events around every attention launch on its stream, in a second pass of "
-                          "the same number of steps (events between launches defeat their overlap, so "
-                          "this duration is an upper bound)"}
+                "timing": timing, "serialized": serialized}
     comparator = None
     if main_policy == 0 and (args.comparator == "on" or
                              (args.comparator == "auto" and args.config in COMPARATOR_CONFIGS)):
