@@ -306,7 +306,9 @@ void layout_scoring(ra_ctx* ctx)
 double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
 {
     const int M = ctx->r * ctx->G;
-    const int per_sm = score_row_tiles_per_warp(M) <= 2 ? 2 : 1;
+    // pass 2 runs on tcgen05 with all of an SM's tensor memory: one CTA per SM, and runs of
+    // whole 128-row tiles (two scoring tiles)
+    const int per_sm = pass == 2 ? 1 : (score_row_tiles_per_warp(M) <= 2 ? 2 : 1);
     long long work = 0;
     int most = 1;
     double rows = 0;
@@ -320,6 +322,7 @@ double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
     const long long target = (long long)ctx->sms * per_sm;
     long long ch = std::max<long long>((work + target - 1) / target, 1);
     if (pass == 1) ch = std::max<long long>(ch, (most + ctx->stats_chunks - 1) / ctx->stats_chunks);
+    if (pass == 2) ch = (ch + 1) / 2 * 2;
     const int nch = (int)((most + ch - 1) / ch);
     if (pass == 1) {
         p->ch1 = (int)ch;
