@@ -174,3 +174,90 @@ def test_scored_comparator_parity_full_size():
         ref = oracle.attend(qv, synth.kv_rows(wl.dseed, 0, l, b, h, pos, D), synth.kv_rows(wl.dseed, 1, l, b, h, pos, D))
         check_attention(got_out[l, b, h * G:(h + 1) * G], ref, f"slice {(b, l, h)}")
     wl.cache.close()
+
+
+def test_config2_full_length_sampled():
+    """The Qwen3-4B-shape workload over its whole generation: the 32768 decode steps from an empty
+    generated cache (prompts only), through the growth phase (no eviction until K + 2r tokens) and
+    then an eviction round every r steps, about 480 rounds per (sequence, layer).  Step inputs come
+    from the seeded generator for their true positions.  The oracle replays sampled heads through
+    every round: survivor positions and cached K/V bytes bit-exact, and the last step's attention of
+    sampled slices within tolerance of the fp64 oracle."""
+    import torch
+
+    import bench
+    import oracle
+    import paper_2609_03430_gb300 as ra
+    import synth
+    import synth.gpu as sg
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    w = bench.WORKLOADS[2]
+    L, H, KVH, B, K, r, D = w["L"], w["H"], w["KVH"], w["B"], w["K"], w["r"], 128
+    G = H // KVH
+    lp, steps = w["lp"], w["gen"][0]
+    dseed, eseed = w["dseed"], w["eseed"]
+    cache = ra.RandomAttentionCache(L, H, KVH, D, lp, K, r, eseed)
+    ctx = cache.ctx
+    key_scale = torch.from_numpy(synth.key_channel_scale(dseed, L, KVH, D)).to(dev)
+    maxlp = max(lp)
+    ppos = torch.tensor([[list(range(lp[b])) + [-1] * (maxlp - lp[b])] * KVH for b in range(B)],
+                        dtype=torch.int32, device=dev)
+    kp = torch.empty((B, KVH, maxlp, D), dtype=torch.int16, device=dev)
+    vp = torch.empty_like(kp)
+    for l in range(L):
+        sg.fill_rows(kp, ppos, dseed, 0, l, 0, key_scale[l].contiguous())
+        sg.fill_rows(vp, ppos, dseed, 1, l, 0)
+        ra.ra_prefill(ctx, l, kp.data_ptr(), vp.data_ptr(), maxlp)
+    del kp, vp
+
+    heads, attn_heads = _samples(w, 8, 4, 202)
+    orc = oracle.OracleCache(L, KVH, lp, K, r, eseed, heads=heads)
+    pairs = sorted({(b, l) for (b, l, _) in heads})
+    CH = 64  # steps whose inputs are generated at once
+    qch = torch.empty((L, B, H, CH, D), dtype=torch.int16, device=dev)
+    kch = torch.empty((L, B, KVH, CH, D), dtype=torch.int16, device=dev)
+    vch = torch.empty_like(kch)
+    q = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((L, B, KVH, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    out = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    lp_t = torch.tensor(lp, dtype=torch.int32, device=dev).view(B, 1, 1)
+    for t0 in range(0, steps, CH):
+        ar = torch.arange(t0, t0 + CH, dtype=torch.int32, device=dev).view(1, 1, CH)
+        npos = (lp_t + ar).expand(B, KVH, CH).contiguous()
+        qpos = ar.expand(B, H, CH).contiguous()
+        for l in range(L):
+            sg.fill_rows(qch[l], qpos, dseed, 2, l, 0)
+            sg.fill_rows(kch[l], npos, dseed, 0, l, 0, key_scale[l].contiguous())
+            sg.fill_rows(vch[l], npos, dseed, 1, l, 0)
+        for i in range(min(CH, steps - t0)):
+            q.copy_(qch[:, :, :, i, :])
+            kn.copy_(kch[:, :, :, i, :])
+            vn.copy_(vch[:, :, :, i, :])
+            ra.ra_decode_step(ctx, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), out.data_ptr(), 0.0)
+            for (b, l) in pairs:
+                orc.append(b, l)
+                orc.evict(b, l)
+    torch.cuda.synchronize()
+    ra.ra_check_device(ctx)
+    rounds = (steps - (K + 2 * r)) // r + 1
+    for (b, l, h) in heads:
+        g, c, nev = ra.ra_get_counters(ctx, b, l)
+        assert g == steps == orc.g[b, l] and c == orc.gen[(b, l, h)].size
+        assert nev == orc.n_evictions[b, l] == rounds
+        got = ra.ra_get_positions(ctx, l, b, h, K + 2 * r)
+        np.testing.assert_array_equal(got, orc.gen[(b, l, h)], err_msg=f"positions {(b, l, h)}")
+    sc_np = key_scale.cpu().numpy()
+    got_out = out.cpu().numpy()
+    for (b, l, h) in attn_heads:
+        pos = orc.positions(b, l, h)
+        krow = synth.kv_rows(dseed, 0, l, b, h, pos, D, sc_np[l, h])
+        vrow = synth.kv_rows(dseed, 1, l, b, h, pos, D)
+        kk, vv = ra.ra_get_kv(ctx, l, b, h, lp[b] + K + 2 * r)
+        np.testing.assert_array_equal(kk, krow, err_msg=f"K rows {(b, l, h)}")
+        np.testing.assert_array_equal(vv, vrow, err_msg=f"V rows {(b, l, h)}")
+        qv = synth.q_rows(dseed, l, b, np.arange(h * G, (h + 1) * G), steps - 1, D)
+        check_attention(got_out[l, b, h * G:(h + 1) * G], oracle.attend(qv, krow, vrow), f"full length slice {(b, l, h)}")
+    cache.close()
