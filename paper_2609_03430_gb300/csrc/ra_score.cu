@@ -439,7 +439,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_sum_tc_kernel(const __grid_
         prefetch_tensormap(&tw);
         // The window rows (row R = slot * G + g) complete on full[0] with the first key tile;
         // rows past M are another head's (or read as zero): finite, and given no weight below.
-        issue_tile(0, (uint32_t)(ROWS * kRowBytes));  // (n_loaded counts tiles whose copies are issued)
+        issue_tile(0, (uint32_t)(ROWS * kRowBytes));
         const int row0 = (int)(lbh * (size_t)M);
         for (int rb = 0; rb < ROWS; rb += kScoreTile) {
             tma_load_2d(smem + C::Q_OFF + rb * 128, &tw, 0, row0 + rb, &full[0]);
@@ -447,7 +447,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_sum_tc_kernel(const __grid_
         }
         if (ntile > 1) issue_tile(1, 0u);
     }
-    int n_loaded = min(ntile, 2), n_mma = 0, done = 0;  // thread 0's counts: tiles loaded, multiplied, waited for
+    // thread 0's counts of tiles: copies issued, MMAs issued, MMAs waited for
+    int n_loaded = min(ntile, 2), n_mma = 0, done = 0;
     {  // the normaliser each window query had at its decode step
         const float2* qst = L.qstats + lbh * (size_t)M;
         for (int R = tid; R < ROWS; R += kThreads) {
