@@ -20,7 +20,8 @@ UNITS = [
     ("ra_api.cu", "ra_api.o", []),
     ("ra_evict.cu", "ra_evict.o", []),
     ("ra_attn.cu", "ra_attn_wide.o", ["-DRA_ATTN_NS=attn_wide", "-DRA_ATTN_TILE=48", "-DRA_ATTN_WARPS=4"]),
-    ("ra_attn.cu", "ra_attn_narrow.o", ["-DRA_ATTN_NS=attn_narrow", "-DRA_ATTN_TILE=32", "-DRA_ATTN_WARPS=6"]),
+    ("ra_attn.cu", "ra_attn_narrow.o",
+     ["-DRA_ATTN_NS=attn_narrow", "-DRA_ATTN_TILE=32", "-DRA_ATTN_WARPS=6", "-DRA_ATTN_TRANSPOSED=1"]),
     ("ra_score.cu", "ra_score.o", []),
 ]
 HEADERS = ["ra_internal.h", "ra_ptx.cuh"]
