@@ -246,6 +246,8 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr)
                  : "r"(addr));
 }
 
+#if !RA_ATTN_TRANSPOSED
+#pragma nv_diag_suppress 550  // d2, d3: the product's padding rows, discarded
 // D[16x8] += A[16x16] B[16x8], bf16 inputs, fp32 accumulators.  Only rows 0..7 of A
 // (the query heads) are nonzero, so only c0/c1 of the accumulator are kept.
 __device__ __forceinline__ void mma_rows8(float& c0, float& c1, uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1)
@@ -259,6 +261,8 @@ __device__ __forceinline__ void mma_rows8(float& c0, float& c1, uint32_t a0, uin
     (void)d2;  // rows 8..15 of the product: padding
     (void)d3;
 }
+#pragma nv_diag_default 550
+#endif
 
 #if RA_ATTN_TRANSPOSED
 // C[16x8] += A[16x16] B[16x8], bf16 inputs, fp32 accumulators (register-only: not volatile, so the
