@@ -456,6 +456,38 @@ def attention_window(wl, steps, t_next):
     return clean, t_next + steps
 
 
+def attention_roofline(a, clean, steps, layers, peaks, peak_src, traffic):
+    """The bench line's roofline of the attention kernel.  a: its per-launch-event totals (the
+    serialized measurement); clean: (device ms, launches, algorithmic bytes) of the eviction-free
+    steps of the step-boundary pass.  The duration is the windowed one when such steps exist, else
+    the serialized one; achieved = algorithmic bytes per launch / duration."""
+    if not a:
+        return None
+    serialized = {"us_per_launch": a["us_per_launch"], "achieved": a["algorithmic_GBps"],
+                  "frac": a["algorithmic_GBps"] / peaks["hbm_gbs"],
+                  "timing": "CUDA events around every attention launch on its stream, in a second pass "
+                            "of the same number of steps (the events between launches defeat their "
+                            "overlap, so this duration is an upper bound)"}
+    if clean:
+        win_ms = sum(c[0] for c in clean)
+        win_n = sum(c[1] for c in clean)
+        by_launch = sum(c[2] for c in clean) / win_n
+        us_launch = 1000.0 * win_ms / win_n
+        timing = (f"CUDA events at the step boundaries on the launching stream, over the {len(clean)} of "
+                  f"{steps} steps of a third pass in which no sequence evicts: such a step launches "
+                  f"only the {layers} layers' attention kernels, overlapped as in the timed region; "
+                  f"duration = their device time / {win_n} launches")
+    else:  # every step evicts somewhere (ragged phases): the per-launch events are all there is
+        by_launch, us_launch, timing = a["bytes_per_launch"], a["us_per_launch"], serialized["timing"]
+    achieved = by_launch / (us_launch * 1e-6) / 1e9
+    return {"kernel": "attn_kernel (split-K decode attention)", "bound": "hbm", "achieved": achieved,
+            "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+            "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+            else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
+            "algorithmic_bytes_per_launch": by_launch, "us_per_launch": us_launch,
+            "traffic": traffic, "timing": timing, "serialized": serialized}
+
+
 def _eviction_us_per_round(kern, names, rounds):
     if not rounds:
         return None
@@ -627,33 +659,8 @@ def run_ours(args, w):
     del wl
 
     peaks, peak_src = measured_peaks()
-    a = kern.get("attn")
-    roof = None
-    if a:
-        serialized = {"us_per_launch": a["us_per_launch"], "achieved": a["algorithmic_GBps"],
-                      "frac": a["algorithmic_GBps"] / peaks["hbm_gbs"],
-                      "timing": "CUDA events around every attention launch on its stream, in a second pass "
-                                "of the same number of steps (the events between launches defeat their "
-                                "overlap, so this duration is an upper bound)"}
-        if clean:
-            win_ms = sum(c[0] for c in clean)
-            win_n = sum(c[1] for c in clean)
-            by_launch = sum(c[2] for c in clean) / win_n
-            us_launch = 1000.0 * win_ms / win_n
-            timing = (f"CUDA events at the step boundaries on the launching stream, over the {len(clean)} of "
-                      f"{args.steps} steps of a third pass in which no sequence evicts: such a step launches "
-                      f"only the {w['L']} layers' attention kernels, overlapped as in the timed region; "
-                      f"duration = their device time / {win_n} launches")
-        else:  # every step evicts somewhere (ragged phases): the per-launch events are all there is
-            by_launch, us_launch, timing = a["bytes_per_launch"], a["us_per_launch"], serialized["timing"]
-        achieved = by_launch / (us_launch * 1e-6) / 1e9
-        roof = {"kernel": "attn_kernel (split-K decode attention)", "bound": "hbm", "achieved": achieved,
-                "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
-                "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
-                else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
-                "algorithmic_bytes_per_launch": by_launch, "us_per_launch": us_launch,
-                "traffic": args.traffic if args.traffic is not None else profiled_traffic(args.config),
-                "timing": timing, "serialized": serialized}
+    roof = attention_roofline(kern.get("attn"), clean, args.steps, w["L"], peaks, peak_src,
+                              args.traffic if args.traffic is not None else profiled_traffic(args.config))
     comparator = None
     if main_policy == 0 and (args.comparator == "on" or
                              (args.comparator == "auto" and args.config in COMPARATOR_CONFIGS)):

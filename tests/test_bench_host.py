@@ -83,3 +83,34 @@ def test_reference_arm_prints_one_json_line():
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
     assert d["metric"] == bench.METRIC
+
+
+def _attn_totals(us, by):
+    return {"us_per_launch": us, "bytes_per_launch": by, "algorithmic_GBps": by / (us * 1e-6) / 1e9}
+
+
+def test_roofline_takes_the_windowed_duration_of_the_eviction_free_steps():
+    peaks = {"hbm_gbs": 6000.0}
+    a = _attn_totals(40.0, 180e6)  # serialized: per-launch events
+    # two eviction-free steps of 36 launches each: 1.26 ms and 1.26 ms, 36 x 174 MB each
+    clean = [(1.26, 36, 36 * 174e6), (1.26, 36, 36 * 174e6)]
+    r = bench.attention_roofline(a, clean, 4, 36, peaks, "measured", 178e6)
+    assert r["us_per_launch"] == pytest.approx(1000.0 * 2.52 / 72)
+    assert r["algorithmic_bytes_per_launch"] == pytest.approx(174e6)
+    assert r["achieved"] == pytest.approx(174e6 / (35e-6) / 1e9)
+    assert r["frac"] == pytest.approx(r["achieved"] / 6000.0)
+    assert r["frac_of_nominal_8TBps"] == pytest.approx(r["achieved"] / 8000.0)
+    assert r["serialized"]["us_per_launch"] == 40.0
+    assert r["serialized"]["frac"] == pytest.approx(180e6 / 40e-6 / 1e9 / 6000.0)
+    assert r["traffic"] == 178e6 and r["bound"] == "hbm" and r["unit"] == "GB/s"
+    assert "2 of 4 steps" in r["timing"] and "36 layers" in r["timing"]
+
+
+def test_roofline_falls_back_to_the_per_launch_events_without_eviction_free_steps():
+    a = _attn_totals(240.0, 1.6e9)
+    r = bench.attention_roofline(a, [], 128, 40, {"hbm_gbs": 6691.0}, "fallback", None)
+    assert r["us_per_launch"] == 240.0 and r["algorithmic_bytes_per_launch"] == 1.6e9
+    assert r["achieved"] == pytest.approx(a["algorithmic_GBps"])
+    assert r["timing"] == r["serialized"]["timing"] and r["peak_source"].startswith("fallback")
+    assert r["traffic"] is None
+    assert bench.attention_roofline(None, [], 1, 1, {"hbm_gbs": 1.0}, "measured", None) is None
