@@ -57,7 +57,7 @@ def _workloads():
 
 
 WORKLOADS = _workloads()
-DEFAULT_CONFIG = 2
+DEFAULT_CONFIG = 4         # the largest workload that fits one GPU (Qwen3-32B shape, ~78 GB of cache)
 COMPARATOR_CONFIGS = (5,)  # workloads that also time the scored comparator on the same caches
 POLICY_SNAPKV = 4
 # order-preserving (the method's engine) / order-free in place / order-preserving inside the attention pass
@@ -66,8 +66,12 @@ WINDOW_STEP0 = 1 << 20     # synthetic step index of the first restored window q
 
 
 def steady_state(w, rank=0):
-    """Per-sequence (g0, c0): right after an eviction (c0 = K + r) for lock-step configs; with a
-    per-sequence phase in [0, r) for the ragged one.  Positions are the newest c0 generated ones."""
+    """Per-sequence (g0, c0) at steady state: phase = the steps since the sequence's last eviction,
+    c0 = K + r + phase, positions the newest c0 generated ones.  The ragged workload draws every
+    sequence's phase and progress; the equal-length ones spread the phases evenly over [0, r)
+    (sequence b at b r / B), as requests that joined a continuous batch at different times, so
+    that any window of steps holds eviction rounds in proportion to its length (about B / r
+    sequences evict per step) instead of all sequences on one step every r."""
     K, r, B = w["K"], w["r"], w["B"]
     if w["B"] == 1 and w["L"] == 1:  # the small config starts empty (full run from step 0)
         return [0] * B, [0] * B
@@ -79,8 +83,8 @@ def steady_state(w, rank=0):
             lo_epochs = -(-(K + 2 * r) // r)
             hi_epochs = max((w["gen"][b] - 2048) // r, lo_epochs)
             ep = int(synth.uniform_ints(2000 + b, 1, lo_epochs, hi_epochs)[0])
-        else:  # an eviction step at least K + 2r (the first one possible), mid-generation
-            phase, ep = 0, max(8192, -(-(K + 2 * r) // r) * r) // r
+        else:  # last eviction at a step of at least K + 2r (the first one possible), mid-generation
+            phase, ep = (b * r) // B, max(8192, -(-(K + 2 * r) // r) * r) // r
         ge = ep * r
         g0.append(ge + phase)
         c0.append(K + r + phase)
@@ -380,7 +384,9 @@ def run_reference(args, w):
 def config_dict(w, args):
     return {"workload": describe(w), "config_index": args.config, "batch": w["B"], "layers": w["L"],
             "q_heads": w["H"], "kv_heads": w["KVH"], "head_dim": D, "K": w["K"], "r": w["r"],
-            "prompt_mean": float(np.mean(w["lp"])), "start": "steady state (K + r cached generated per head)",
+            "prompt_mean": float(np.mean(w["lp"])), "start": "steady state: K + r + phase cached generated rows per head, phase = steps since the "
+                      "sequence's last eviction (spread evenly over [0, r) for equal-length batches, drawn "
+                      "for the ragged one)",
             "l2": "inputs larger than L2 (every step streams the whole cache)", "parallelism": f"replicas x{args.gpus}",
             "policy": getattr(args, "policy", "random"), "compaction": getattr(args, "compaction", "ordered")}
 
@@ -488,6 +494,55 @@ def attention_roofline(a, clean, steps, layers, peaks, peak_src, traffic):
             "traffic": traffic, "timing": timing, "serialized": serialized}
 
 
+EVICT_KINDS = ("score_stats", "score_sum", "select", "compact", "evict")
+
+
+def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None):
+    """The bench line's roofline of the eviction: its copy kernel (the fused select + compaction
+    kernel when the library ran it, else the compaction kernel) at its algorithmic bytes -- the
+    survivors' K, V and position read and written, 2 (2 d 2 + 4) bytes per row -- over its
+    per-launch CUDA-event duration, and the whole round (every eviction kernel's time per
+    (sequence, layer) round).  holefill: (kernels, rounds) of the order-free run, whose select
+    kernel moves the m refilled rows itself."""
+    name = "evict" if "evict" in kern else ("compact" if "compact" in kern else None)
+    if name is None or not rounds:
+        return None
+    k = kern[name]
+    if not k["ms_total"]:
+        return None
+    achieved = k["bytes_per_launch"] / (k["us_per_launch"] * 1e-6) / 1e9
+    round_ms = sum(kern[n]["ms_total"] for n in EVICT_KINDS if n in kern)
+    round_bytes = sum(kern[n]["bytes_per_launch"] * kern[n]["launches"] for n in EVICT_KINDS if n in kern)
+    out = {"kernel": ("evict_kernel (selection and order-preserving compaction, one cluster per head)"
+                      if name == "evict" else "compact_kernel (order-preserving compaction)"),
+           "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+           "frac": achieved / peaks["hbm_gbs"],
+           "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+           else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
+           "algorithmic_bytes_per_launch": k["bytes_per_launch"], "us_per_launch": k["us_per_launch"],
+           "launches": k["launches"], "traffic": traffic,
+           "timing": "CUDA events around every eviction launch on its stream, in a second pass of the same "
+                     "number of steps (events between launches defeat programmatic dependent launch, so "
+                     "the duration includes the launch's own start-up)",
+           "round": {"rounds": rounds, "us_per_round": 1000.0 * round_ms / rounds,
+                     "bytes_per_round": round_bytes / rounds,
+                     "frac": (round_bytes / (round_ms * 1e-3) / 1e9 / peaks["hbm_gbs"]) if round_ms else None,
+                     "what": "every eviction kernel's evented time and algorithmic bytes per (sequence, layer) "
+                             "round"}}
+    if holefill is not None:
+        hk, hr = holefill
+        sel = hk.get("select")
+        if sel and hr and sel["ms_total"]:
+            out["holefill_select"] = {
+                "us_per_launch": sel["us_per_launch"], "bytes_per_launch": sel["bytes_per_launch"],
+                "achieved": sel["bytes_per_launch"] / (sel["us_per_launch"] * 1e-6) / 1e9,
+                "frac": sel["bytes_per_launch"] / (sel["us_per_launch"] * 1e-6) / 1e9 / peaks["hbm_gbs"],
+                "us_per_round": 1000.0 * sel["ms_total"] / hr,
+                "what": "order-free compaction: the select kernel refills the m evicted slots in place, "
+                        "2 m (2 d 2 + 4) bytes per head"}
+    return out
+
+
 def _eviction_us_per_round(kern, names, rounds):
     if not rounds:
         return None
@@ -521,8 +576,8 @@ def run_comparator(args, rank, world, barrier, peaks, random_ms, random_kern, ra
             "step_time_vs_random": ms_step / random_ms,
             "rounds_in_evented_pass": {"random": random_rounds, "snapkv": rounds},
             "eviction_us_per_round": {
-                "random": _eviction_us_per_round(random_kern, ("select", "compact"), random_rounds),
-                "snapkv": _eviction_us_per_round(kern, ("score_stats", "score_sum", "select", "compact"), rounds),
+                "random": _eviction_us_per_round(random_kern, EVICT_KINDS, random_rounds),
+                "snapkv": _eviction_us_per_round(kern, EVICT_KINDS, rounds),
                 "what": "evented kernel time of a step's eviction launches / (sequence, layer) rounds they ran"},
             "score_kernels": score, "kernels": kern}
 
@@ -545,10 +600,10 @@ def run_holefill_variant(args, rank, world, barrier, peaks, ordered_ms, ordered_
             "step_time_vs_ordered": ms_step / ordered_ms,
             "step_effective_frac": cache_bytes / (ms_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
             "eviction_us_per_round": {
-                "ordered": _eviction_us_per_round(ordered_kern, ("select", "compact"), ordered_rounds),
-                "holefill": _eviction_us_per_round(kern, ("select", "compact"), rounds),
+                "ordered": _eviction_us_per_round(ordered_kern, EVICT_KINDS, ordered_rounds),
+                "holefill": _eviction_us_per_round(kern, EVICT_KINDS, rounds),
                 "what": "evented kernel time of a step's eviction launches / (sequence, layer) rounds they ran"},
-            "kernels": kern}
+            "rounds_in_evented_pass": rounds, "kernels": kern}
 
 
 def run_ours(args, w):
@@ -668,6 +723,8 @@ def run_ours(args, w):
     holefill = None
     if main_policy == 0 and args.compaction == "ordered" and args.variants == "on":
         holefill = run_holefill_variant(args, rank, world, barrier, peaks, ms_step, kern, rounds)
+    roof_evict = eviction_roofline(kern, rounds, peaks, peak_src, args.traffic_evict,
+                                   (holefill["kernels"], holefill["rounds_in_evented_pass"]) if holefill else None)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)
@@ -675,7 +732,7 @@ def run_ours(args, w):
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_dict(w, args),
-                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "roofline": roof, "roofline_evict": roof_evict, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                 "clocks": clocks.summary(wall0, wall1), "kernels": kern,
                 "attn_cache_bytes_per_step": attn_bytes_before,
                 "step_effective": {"GBps": attn_bytes_before / (ms_step * 1e-3) / 1e9,
@@ -716,6 +773,8 @@ def main(argv=None):
                     help="also time the scored comparator on the same caches (auto: the ragged workload)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per attention launch (from a committed profile), if current")
+    ap.add_argument("--traffic-evict", type=float, default=None,
+                    help="ncu dram bytes per eviction copy launch (from a committed profile), if current")
     args = ap.parse_args(argv)
     args.cpu_seconds_set = any(a.startswith("--cpu-seconds") for a in (argv if argv is not None else sys.argv[1:]))
     if args.warmup < 3:

@@ -310,8 +310,24 @@ int ra_get_positions(ra_ctx* ctx, int layer, int seq, int kv_head, int32_t* host
 int ra_get_kv(ra_ctx* ctx, int layer, int seq, int kv_head, uint16_t* host_k, uint16_t* host_v, int capacity_rows,
               int* n_rows, void* stream);
 
-/* Synchronise `stream` and report RA_ERR_DEVICE_TIMEOUT if any kernel flagged a bounded-wait timeout. */
+/*
+ * Synchronise `stream` and report what the kernels flagged in the context's device error word:
+ * RA_ERR_DEVICE_TIMEOUT if a kernel gave up a bounded wait (every mbarrier wait of the pipelines
+ * is bounded at 2 s; the kernel then lets its own copies land, releases what it holds and
+ * returns), RA_ERR_STATE if an eviction plan disagreed with the host counters.  The word is
+ * cleared once reported, so a later call reports only new events.
+ */
 int ra_check_device(ra_ctx* ctx, void* stream);
+
+/*
+ * Test hook of the device-timeout path: launch one CTA on `stream` that arms an mbarrier for 16
+ * bytes of transfer that nothing ever issues, waits on it with its wait bounded at limit_ns
+ * nanoseconds (1 000 .. 100 000 000), then flags the timeout in the device error word exactly as
+ * the pipeline kernels do, and returns.  It touches no memory but its own shared memory and the
+ * error word, so the context stays usable: ra_check_device then returns RA_ERR_DEVICE_TIMEOUT
+ * once.  (The paper has no counterpart: failure detection of this library.)
+ */
+int ra_debug_timeout_probe(ra_ctx* ctx, uint64_t limit_ns, void* stream);
 
 /*
  * Per-kernel accounting.  Launch counts and algorithmic bytes (the bytes each

@@ -57,6 +57,7 @@ SIGNATURES = {
     "ra_get_positions": (_i, [_vp, _i, _i, _i, _i32p, _i, _ip, _vp]),
     "ra_get_kv": (_i, [_vp, _i, _i, _i, _vp, _vp, _i, _ip, _vp]),
     "ra_check_device": (_i, [_vp, _vp]),
+    "ra_debug_timeout_probe": (_i, [_vp, _u64, _vp]),
     "ra_profile_enable": (_i, [_vp, _i]),
     "ra_profile_read": (_i, [_vp, _i, _dp, _i64p, _dp]),
     "ra_profile_reset": (_i, [_vp]),
@@ -234,6 +235,10 @@ def ra_get_kv(ctx, layer, seq, kv_head, capacity_rows, head_dim=128, stream=None
 
 def ra_check_device(ctx, stream=None):
     return _check(lib().ra_check_device(ctx, _stream_ptr(stream)), ctx)
+
+
+def ra_debug_timeout_probe(ctx, limit_ns, stream=None):
+    return _check(lib().ra_debug_timeout_probe(ctx, int(limit_ns), _stream_ptr(stream)), ctx)
 
 
 def ra_profile_enable(ctx, on=True):

@@ -1070,10 +1070,25 @@ int ra_check_device(ra_ctx* ctx, void* stream)
     if ((e = cudaStreamSynchronize((cudaStream_t)stream)) != cudaSuccess) return cuda_fail(ctx, e, "stream sync");
     int32_t w = 0;
     if ((e = cudaMemcpy(&w, ctx->lay.err, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(ctx, e, "err read");
+    if (w != 0) {  // reported once: clear it (the stream is idle, nothing else writes it now)
+        const int32_t zero = 0;
+        if ((e = cudaMemcpy(ctx->lay.err, &zero, 4, cudaMemcpyHostToDevice)) != cudaSuccess)
+            return cuda_fail(ctx, e, "err clear");
+    }
     if (w == kDeviceErrTimeout) return fail(ctx, RA_ERR_DEVICE_TIMEOUT, "a kernel gave up a bounded wait");
     if (w == kDeviceErrPlan) return fail(ctx, RA_ERR_STATE, "device eviction plan inconsistent with host counters");
     if (w != 0) return fail(ctx, RA_ERR_STATE, "device error word %d", w);
     return RA_OK;
+}
+
+int ra_debug_timeout_probe(ra_ctx* ctx, uint64_t limit_ns, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if (limit_ns < 1000ull || limit_ns > 100000000ull)
+        return fail(ctx, RA_ERR_INVALID_ARG, "limit_ns %llu outside [1e3, 1e8]", (unsigned long long)limit_ns);
+    cudaError_t e = launch_timeout_probe(ctx->lay.err, limit_ns, (cudaStream_t)stream);
+    return e == cudaSuccess ? RA_OK : cuda_fail(ctx, e, "timeout probe launch");
 }
 
 int ra_profile_enable(ra_ctx* ctx, int on)

@@ -406,6 +406,21 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
     }
 }
 
+// ----------------------------------------------------------------------------- timeout probe
+// The failure path of every bounded wait, run on purpose: one arrival with 16 bytes of
+// transfer expected, and no copy ever issued, so the barrier's phase cannot complete; the
+// bounded wait gives up after limit_ns and the error word is flagged as the pipelines do.
+__global__ void __launch_bounds__(32) timeout_probe_kernel(int32_t* err, uint64_t limit_ns)
+{
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x != 0) return;
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(&bar, 16u);
+    if (!mbar_wait_bounded(&bar, 0u, limit_ns)) atomicExch(err, kDeviceErrTimeout);
+    mbar_inval(&bar);
+}
+
 // ----------------------------------------------------------------------------- prefill / restore
 __global__ void __launch_bounds__(256) copy_rows_kernel(const __grid_constant__ CopyRowsParams p, int restore)
 {
@@ -505,6 +520,12 @@ cudaError_t launch_compact(const EvictParams& p, cudaStream_t s)
     const int chunks = (Cmax + kCompactChunk - 1) / kCompactChunk;
     return launch_pdl(compact_kernel, dim3(chunks, p.n_trig * p.lay.KVH), dim3(kCompactThreads),
                       p.lay.r * sizeof(int32_t), s, p);
+}
+
+cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s)
+{
+    timeout_probe_kernel<<<1, 32, 0, s>>>(err, limit_ns);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s)

@@ -132,6 +132,7 @@ cudaError_t launch_select(const EvictParams& p, cudaStream_t s);
 size_t select_smem(int N, int r, bool scored);  // dynamic shared memory of one select CTA
 constexpr size_t kSelectSmemLimit = 220 * 1024;
 cudaError_t launch_compact(const EvictParams& p, cudaStream_t s);
+cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s);
 cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s);
 cudaError_t launch_restore_queries(const DevLayout& lay, int layer, const uint16_t* q, const int32_t* g_dev,

@@ -60,6 +60,7 @@ def test_create_validation_is_host_only(ra):
     assert L.ra_append_kv(ctx, 0, None, None, None) == ra.RA_ERR_STATE
     assert L.ra_evict(ctx, 0, None, None) == ra.RA_ERR_STATE
     assert L.ra_decode_attn(ctx, 0, None, None, ctypes.c_float(0), None) == ra.RA_ERR_STATE
+    assert L.ra_debug_timeout_probe(ctx, ctypes.c_uint64(1000000), None) == ra.RA_ERR_STATE
     assert L.ra_bind(ctx, None, 0, None) == ra.RA_ERR_INVALID_ARG
     assert ra.ra_get_counters(ctx, 0, 1) == (0, 0, 0)
     ra.ra_destroy(ctx)

@@ -37,6 +37,22 @@ def test_steady_state_is_a_reachable_state(cfg):
         assert g + 2048 <= gen  # the sequence stays active through a benchmark window
 
 
+@pytest.mark.parametrize("cfg", [2, 3, 4])
+def test_equal_length_batches_spread_their_evictions_over_every_window(cfg):
+    """Sequence b of an equal-length batch evicts on the steps where its generated count reaches a
+    multiple of r; with the phases spread over [0, r), any window of W steps holds about W B / r
+    (sequence) rounds, so a short timed window still prices the eviction."""
+    w = bench.WORKLOADS[cfg]
+    g0, _ = bench.steady_state(w)
+    r, B = w["r"], w["B"]
+    fires = [sum(1 for g in g0 if (g + t + 1) % r == 0) for t in range(3 * r)]
+    for W in (20, 32, r):
+        for t0 in range(2 * r):
+            n = sum(fires[t0:t0 + W])
+            assert abs(n - W * B / r) <= 1 + (B // r), (W, t0, n)
+    assert sum(fires[:r]) == B  # every sequence once per r steps
+
+
 def _free_port():
     s = socket.socket()
     s.bind(("127.0.0.1", 0))
@@ -114,3 +130,32 @@ def test_roofline_falls_back_to_the_per_launch_events_without_eviction_free_step
     assert r["timing"] == r["serialized"]["timing"] and r["peak_source"].startswith("fallback")
     assert r["traffic"] is None
     assert bench.attention_roofline(None, [], 1, 1, {"hbm_gbs": 1.0}, "measured", None) is None
+
+
+def _kern(us, by, n):
+    return {"launches": n, "ms_total": us * n / 1000.0, "us_per_launch": us, "bytes_per_launch": by,
+            "algorithmic_GBps": by / (us * 1e-6) / 1e9}
+
+
+def test_eviction_roofline_prices_the_copy_kernel_and_the_round():
+    peaks = {"hbm_gbs": 6000.0}
+    kern = {"attn": _kern(200.0, 1.2e9, 640), "select": _kern(10.0, 0.0, 20), "compact": _kern(20.0, 68e6, 20)}
+    r = bench.eviction_roofline(kern, 20, peaks, "measured", 70e6)
+    assert r["kernel"].startswith("compact_kernel") and r["bound"] == "hbm" and r["unit"] == "GB/s"
+    assert r["achieved"] == pytest.approx(68e6 / 20e-6 / 1e9)
+    assert r["frac"] == pytest.approx(r["achieved"] / 6000.0)
+    assert r["frac_of_nominal_8TBps"] == pytest.approx(r["achieved"] / 8000.0)
+    assert r["round"]["us_per_round"] == pytest.approx(30.0)
+    assert r["round"]["bytes_per_round"] == pytest.approx(68e6)
+    assert r["round"]["frac"] == pytest.approx(68e6 / 30e-6 / 1e9 / 6000.0)
+    assert r["traffic"] == 70e6 and r["launches"] == 20
+    # the fused kernel, when present, is the one priced; order-free select reported beside it
+    kern2 = {"evict": _kern(12.0, 68e6, 10)}
+    hole = ({"select": _kern(5.0, 2e6, 10)}, 10)
+    r2 = bench.eviction_roofline(kern2, 10, peaks, "fallback", None, hole)
+    assert r2["kernel"].startswith("evict_kernel") and r2["peak_source"].startswith("fallback")
+    assert r2["round"]["us_per_round"] == pytest.approx(12.0)
+    assert r2["holefill_select"]["achieved"] == pytest.approx(2e6 / 5e-6 / 1e9)
+    assert r2["holefill_select"]["us_per_round"] == pytest.approx(5.0)
+    # no eviction in the evented pass: nothing to report
+    assert bench.eviction_roofline({"attn": kern["attn"]}, 0, peaks, "measured") is None

@@ -4,9 +4,13 @@ running while another framework owns every device allocation, or inside a
 region where cudaMalloc is not allowed).  Its split-K scratch is a fixed
 device array inside the library, so the call allocates nothing.
 
-It is called through the C ABI and must give the same result as ra_decode_attn,
-within the attention tolerance, on two calls in a row (the shared array keeps
-the previous call's contents, which must not leak into the next result).
+It is called through the C ABI and must give the same result as ra_decode_attn
+on two calls in a row -- bit for bit, since it runs the same kernel with the same
+split and merge order; only the scratch differs -- and that result is itself within
+the attention tolerance of the fp64 oracle elsewhere.  The shared array keeps the
+previous call's contents, which must not leak into the next result: before the
+compared calls, a call on a context of another shape leaves its own partial
+records and counters behind.
 This file sorts last so that a stop-at-first-failure run has already run every
 other test; it also passes on its own in a fresh process.
 """
@@ -38,6 +42,15 @@ def test_noalloc_matches_decode_attn_on_two_calls():
         run.step()
     lib = ra.lib()
     stream = torch.cuda.current_stream().cuda_stream
+    # another shape first (G = 8, long split heads): its partials and counters stay in the array
+    other = Runner(L=1, H=16, KVH=2, prompt_lens=[2500, 1200], K=256, r=64, eseed=4, dseed=9)
+    for _ in range(3):
+        other.step()
+    qo = other.up(np.stack([synth.q_rows(9, 0, b, np.arange(16), 7, 128) for b in range(2)]))
+    oo = torch.zeros((2, 16, 128), dtype=torch.int16, device="cuda")
+    assert lib.ra_decode_attn_noalloc(other.ctx, 0, qo.data_ptr(), oo.data_ptr(), ctypes.c_float(0.0), stream) == 0
+    torch.cuda.synchronize()
+    other.close()
     for layer in range(run.L):
         for call in range(2):
             q = np.stack([synth.q_rows(8, layer, b, np.arange(run.H), 1000 + call, 128) for b in range(run.B)])
@@ -48,6 +61,7 @@ def test_noalloc_matches_decode_attn_on_two_calls():
             rc = lib.ra_decode_attn_noalloc(run.ctx, layer, tq.data_ptr(), got.data_ptr(), ctypes.c_float(0.0), stream)
             assert rc == 0, ra.ra_last_error(run.ctx)
             torch.cuda.synchronize()
+            assert torch.equal(got, ref), f"layer {layer} call {call}"
             _close(got.cpu().numpy(), ref.cpu().numpy())
     run.close()
 
