@@ -447,19 +447,44 @@ def attention_window(wl, steps, t_next):
     def evictions_layer0():  # the host mirror's counts; every layer of a sequence evicts on the same step
         return sum(ra.ra_get_counters(wl.ctx, b, 0)[2] for b in range(wl.B))
 
+    ev_kinds = [ra.KERNEL_NAMES.index(n) for n in EVICT_KINDS if n in ra.KERNEL_NAMES]
+
+    def evict_bytes():  # algorithmic bytes of the eviction launches so far (library count)
+        return sum(ra.ra_profile_read(wl.ctx, k)[2] for k in ev_kinds)
+
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
     marks = []
     evs[0].record(wl.stream)
     for i, t in enumerate(range(t_next, t_next + steps)):
-        n0 = evictions_layer0()
+        n0, r0, e0 = evictions_layer0(), wl.evictions(), evict_bytes()
         _, l0, b0 = ra.ra_profile_read(wl.ctx, kind)
         wl.step(t)
         evs[i + 1].record(wl.stream)
         _, l1, b1 = ra.ra_profile_read(wl.ctx, kind)
-        marks.append((evictions_layer0() != n0, l1 - l0, b1 - b0))
+        marks.append((evictions_layer0() != n0, l1 - l0, b1 - b0, wl.evictions() - r0, evict_bytes() - e0))
     torch.cuda.synchronize()
-    clean = [(evs[i].elapsed_time(evs[i + 1]), n, by) for i, (fired, n, by) in enumerate(marks) if not fired and n > 0]
-    return clean, t_next + steps
+    steps_ms = [(evs[i].elapsed_time(evs[i + 1]),) + m for i, m in enumerate(marks)]
+    clean = [(ms, n, by) for (ms, fired, n, by, _, _) in steps_ms if not fired and n > 0]
+    evicting = [(ms, by, rounds, eby) for (ms, fired, n, by, rounds, eby) in steps_ms if fired and n > 0]
+    return clean, evicting, t_next + steps
+
+
+def eviction_window(clean, evicting):
+    """The eviction's cost on the critical path, measured in the step-boundary pass: a step in
+    which sequences evict takes its attention time (its attention bytes at the eviction-free
+    steps' attention bandwidth) plus what the eviction adds; that difference, over the steps'
+    (sequence, layer) rounds and eviction bytes.  It includes what overlaps: the eviction's row
+    loads start under programmatic dependent launch during the previous attention's tail."""
+    if not clean or not evicting:
+        return None
+    attn_ms_per_byte = sum(c[0] for c in clean) / sum(c[2] for c in clean)
+    extra_ms = sum(ms - by * attn_ms_per_byte for (ms, by, _, _) in evicting)
+    rounds = sum(e[2] for e in evicting)
+    ebytes = sum(e[3] for e in evicting)
+    if rounds <= 0 or extra_ms <= 0:
+        return None
+    return {"steps": len(evicting), "rounds": rounds, "us_per_round": 1000.0 * extra_ms / rounds,
+            "bytes_per_round": ebytes / rounds, "GBps": ebytes / (extra_ms * 1e-3) / 1e9}
 
 
 def attention_roofline(a, clean, steps, layers, peaks, peak_src, traffic):
@@ -497,7 +522,7 @@ def attention_roofline(a, clean, steps, layers, peaks, peak_src, traffic):
 EVICT_KINDS = ("score_stats", "score_sum", "select", "compact", "evict")
 
 
-def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None):
+def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None, windowed=None):
     """The bench line's roofline of the eviction: its copy kernel (the fused select + compaction
     kernel when the library ran it, else the compaction kernel) at its algorithmic bytes -- the
     survivors' K, V and position read and written, 2 (2 d 2 + 4) bytes per row -- over its
@@ -529,6 +554,11 @@ def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None
                      "frac": (round_bytes / (round_ms * 1e-3) / 1e9 / peaks["hbm_gbs"]) if round_ms else None,
                      "what": "every eviction kernel's evented time and algorithmic bytes per (sequence, layer) "
                              "round"}}
+    if windowed is not None:
+        out["windowed"] = dict(windowed, frac=windowed["GBps"] / peaks["hbm_gbs"],
+                               what="step-boundary pass: (device time of the steps in which sequences evict - their "
+                                    "attention bytes at the eviction-free steps' attention bandwidth) per (sequence, "
+                                    "layer) round; the eviction's cost on the critical path, overlap included")
     if holefill is not None:
         hk, hr = holefill
         sel = hk.get("select")
@@ -648,7 +678,8 @@ def run_ours(args, w):
     # Kernel durations: the same number of steps again with CUDA events around every launch ...
     kern, rounds, t_next = evented_steps(wl, args.steps, t_next)
     # ... and once more with events only at the step boundaries (attention launches overlapped).
-    clean, t_next = attention_window(wl, args.steps, t_next)
+    clean, evicting, t_next = attention_window(wl, args.steps, t_next)
+    win_evict = eviction_window(clean, evicting)
 
     ms_step, units = reduce_over_ranks(ms, float(wl.B), world)
     value = units / (ms_step * 1e-3)
@@ -724,7 +755,8 @@ def run_ours(args, w):
     if main_policy == 0 and args.compaction == "ordered" and args.variants == "on":
         holefill = run_holefill_variant(args, rank, world, barrier, peaks, ms_step, kern, rounds)
     roof_evict = eviction_roofline(kern, rounds, peaks, peak_src, args.traffic_evict,
-                                   (holefill["kernels"], holefill["rounds_in_evented_pass"]) if holefill else None)
+                                   (holefill["kernels"], holefill["rounds_in_evented_pass"]) if holefill else None,
+                                   win_evict)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)

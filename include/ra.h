@@ -71,7 +71,9 @@ enum ra_kernel_kind {
     RA_KERNEL_ATTN = 3,
     RA_KERNEL_SCORE_STATS = 4, /* scored comparator: normalisers of a restored query window */
     RA_KERNEL_SCORE_SUM = 5,   /* scored comparator: window attention summed per candidate */
-    RA_KERNEL_KINDS = 6
+    RA_KERNEL_EVICT = 6,       /* selection and order-preserving compaction in one launch */
+    RA_KERNEL_PLAN = 7,        /* evicted sets of the next step, computed beside the current one */
+    RA_KERNEL_KINDS = 8
 };
 
 /*
@@ -225,6 +227,27 @@ int ra_get_scores(ra_ctx* ctx, int layer, int seq, int kv_head, float* host_scor
 #define RA_ATTN_SHAPE_WIDE 1
 #define RA_ATTN_SHAPE_NARROW 2
 int ra_set_attention_shape(ra_ctx* ctx, int shape);
+
+/*
+ * Tuning: how an ordered-compaction round of the random policy (and of the shared, recency and
+ * block variants) runs.  RA_EVICT_AUTO (default) launches one kernel: for every triggered head
+ * one or more thread-block clusters each draw the keys, select the evicted set exactly across
+ * the cluster through distributed shared memory, and move their share of the survivors; the
+ * cluster size and the clusters per head are chosen from the number of triggered heads and the
+ * device's cluster occupancy.  For the random and shared draws the selection first takes the
+ * candidates above a cut that about 2m + 32 of them pass (m = candidates - K evicted) and ranks
+ * those exactly; if fewer than m pass it falls back to exact radix passes over the keys, which
+ * RA_EVICT_EXACT (or-ed into the mode) forces.  RA_EVICT_TWO_KERNELS runs the selection kernel
+ * (one CTA per head, writing the evicted list to global memory) and then the compaction kernel.
+ * A value in [2, 16] forces that cluster size (raised to the minimum that holds a head's keys,
+ * ceil((K + r) / 2112) CTAs, or to the next size the device can schedule).  Results are
+ * identical in every mode.  The scored policy, order-free and in-attention compaction, and
+ * buffers of r > 512 always use the selection kernel.
+ */
+#define RA_EVICT_AUTO 0
+#define RA_EVICT_TWO_KERNELS 1
+#define RA_EVICT_EXACT 256
+int ra_set_eviction_kernel(ra_ctx* ctx, int mode);
 
 /* Mark sequence `seq` active (1) or finished (0); finished ones are skipped by every call. */
 int ra_set_active(ra_ctx* ctx, int seq, int active);

@@ -25,8 +25,10 @@ RA_ERR_CUDA = -4
 RA_ERR_DEVICE_TIMEOUT = -5
 RA_ERR_UNSUPPORTED = -6
 RA_MAX_BATCH = 512
-RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN, RA_KERNEL_SCORE_STATS, RA_KERNEL_SCORE_SUM = range(6)
-KERNEL_NAMES = ["append", "select", "compact", "attn", "score_stats", "score_sum"]
+(RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN, RA_KERNEL_SCORE_STATS, RA_KERNEL_SCORE_SUM,
+ RA_KERNEL_EVICT, RA_KERNEL_PLAN) = range(8)
+KERNEL_NAMES = ["append", "select", "compact", "attn", "score_stats", "score_sum", "evict", "plan"]
+RA_EVICT_AUTO, RA_EVICT_TWO_KERNELS, RA_EVICT_EXACT = 0, 1, 256
 
 # Exported C symbols and their ctypes signatures (kept in the order of include/ra.h).
 _vp, _i, _u64, _sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint64, ctypes.c_size_t
@@ -44,6 +46,7 @@ SIGNATURES = {
     "ra_set_policy": (_i, [_vp, _i, _i]),
     "ra_set_compaction": (_i, [_vp, _i]),
     "ra_set_attention_shape": (_i, [_vp, _i]),
+    "ra_set_eviction_kernel": (_i, [_vp, _i]),
     "ra_restore_queries": (_i, [_vp, _i, _vp, ctypes.c_float, _vp]),
     "ra_get_scores": (_i, [_vp, _i, _i, _i, ctypes.POINTER(ctypes.c_float), _i, _ip, _vp]),
     "ra_set_active": (_i, [_vp, _i, _i]),
@@ -155,6 +158,10 @@ RA_ATTN_SHAPE_AUTO, RA_ATTN_SHAPE_WIDE, RA_ATTN_SHAPE_NARROW = 0, 1, 2
 
 def ra_set_attention_shape(ctx, shape):
     return _check(lib().ra_set_attention_shape(ctx, int(shape)), ctx)
+
+
+def ra_set_eviction_kernel(ctx, mode):
+    return _check(lib().ra_set_eviction_kernel(ctx, int(mode)), ctx)
 
 
 def ra_set_compaction(ctx, mode):

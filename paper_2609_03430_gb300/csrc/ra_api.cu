@@ -53,7 +53,7 @@ struct ra_ctx {
     size_t partial_records = 0;  // split-K partial records the arena holds
     // arena layout (byte offsets)
     size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_poff, off_plan, off_partial, off_arrive,
-        off_err, bytes;
+        off_err, off_evplan, bytes;
     // scored policy: query window, scores and pass-1 statistics after the base arena
     bool scoring = false;
     size_t base_bytes = 0, off_qring = 0, off_qstats = 0, off_scores = 0, off_stats = 0;
@@ -62,6 +62,7 @@ struct ra_ctx {
     bool bound = false;
     int device = -1;
     int sms = 0;
+    int evict_active[kEvMaxCluster + 1] = {0};  // clusters of each size the device runs at once
     uint8_t* arena = nullptr;
     DevLayout lay{};
     CUtensorMap tmap_k[kAttnShapes]{}, tmap_v[kAttnShapes]{};  // per attention shape (tile rows)
@@ -74,7 +75,20 @@ struct ra_ctx {
     int block = 1;
     int compaction = RA_COMPACT_ORDERED;  // ra_set_compaction
     int attn_shape = RA_ATTN_SHAPE_AUTO;  // ra_set_attention_shape
+    int evict_mode = RA_EVICT_AUTO;       // ra_set_eviction_kernel
     std::vector<int32_t> score_n;    // [L][B] candidates of the latest scored round
+    // Mirror of the device region tables.  Every head of a (layer, seq) evicts together, so the
+    // region of (l, b, h) is always region_base * KVH + h: rbase[l * B + b], and the spare of
+    // (b, h) is sbase[b] * KVH + h; an ordered compaction swaps the two.
+    std::vector<int32_t> rbase, sbase;
+    // Evicted sets computed one step ahead (ra_decode_step): plan_kernel runs on a side stream
+    // beside the current step's attention and writes half (step parity) of the plan buffer;
+    // plan_g / plan_n [2][L * B] record the firing (g, candidates) each half holds (-1: none).
+    cudaStream_t side = nullptr;
+    cudaEvent_t fork_ev = nullptr, plan_ev = nullptr;
+    bool plan_pending = false;
+    int parity = 0;
+    std::vector<int32_t> plan_g, plan_n;
     // profiling
     bool prof = false;
     std::vector<ProfRec> pending;
@@ -334,10 +348,36 @@ double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
     return rows * kRowBytes;
 }
 
+int run_eviction_launches(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention,
+                          int score_early);
+
+// Evicted sets can be computed ahead for the one-launch eviction of the policies whose keys read
+// no cache data (random, shared, recency) with ordered compaction outside the attention pass.
+bool plan_usable(const ra_ctx* ctx)
+{
+    return ctx->compaction == RA_COMPACT_ORDERED && ctx->r <= kEvMaxEvicted &&
+           (ctx->evict_mode & ~RA_EVICT_EXACT) != RA_EVICT_TWO_KERNELS && ctx->evict_active[1] > 0 &&
+           (ctx->policy == RA_POLICY_RANDOM || ctx->policy == RA_POLICY_SHARED || ctx->policy == RA_POLICY_RECENCY);
+}
+
 // One eviction round of the triggered sequences in p: [score passes,] select, compact (unless
 // the caller's attention launch does the compaction).
 int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention = false,
                  int score_early = 0)
+{
+    for (int i = 0; i < p.n_trig; ++i) {
+        p.trig_src[i] = ctx->rbase[(size_t)p.layer * ctx->B + p.trig[i]];
+        p.trig_dst[i] = ctx->sbase[p.trig[i]];
+    }
+    int rc = run_eviction_launches(ctx, p, moved, s, compact_in_attention, score_early);
+    if (rc == RA_OK && !p.holefill)  // every ordered compaction (any kernel) swaps region and spare
+        for (int i = 0; i < p.n_trig; ++i)
+            std::swap(ctx->rbase[(size_t)p.layer * ctx->B + p.trig[i]], ctx->sbase[p.trig[i]]);
+    return rc;
+}
+
+int run_eviction_launches(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention,
+                          int score_early)
 {
     cudaError_t e;
     if (p.policy == RA_POLICY_SNAPKV) {  // window scores with the normalisers recorded at decode time
@@ -350,6 +390,47 @@ int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool
         p.early = select_early;
         ps.done();
         if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
+    }
+    // The random policy and its key-per-ordinal variants with ordered compaction: one launch,
+    // a cluster per triggered head.
+    // A head's candidates are split over the CTAs of a cluster (at most kEvMaxLocal keys each);
+    // each of a head's `reps` clusters selects on its own and the copy is split over all of
+    // them.  The automatic shape maximises the CTAs working on each head at once,
+    // cl x reps / waves, from the device's cluster occupancy (a GPC holds a whole cluster, so
+    // sizes that pack its SMs win; ties go to the larger cluster, which draws fewer keys per
+    // CTA).  A device that cannot schedule a usable size takes the two kernels.
+    const int least = std::max(1, (ctx->K + ctx->r + kEvMaxLocal - 1) / kEvMaxLocal);
+    const int heads = std::max(1, p.n_trig * ctx->KVH);
+    const int forced = ctx->evict_mode & ~RA_EVICT_EXACT;
+    int cl = 0, reps = 1;
+    double best = 0;
+    if (p.ev_plan) {  // the evicted sets are known: no cluster, the copy spread over about one CTA per SM
+        cl = 1;
+        reps = std::max(1, std::min(64, ctx->evict_active[1] / heads));
+    }
+    for (int x = std::max(least, forced >= 2 ? forced : least); x <= kEvMaxCluster && !p.ev_plan; ++x) {
+        const int act = ctx->evict_active[x];
+        if (act <= 0) continue;
+        const int rp = std::max(1, std::min(act / heads, 64));
+        const double waves = std::ceil((double)heads * rp / act);
+        const double score = x * rp / waves;
+        if (score >= best) {
+            best = score;
+            cl = x;
+            reps = rp;
+        }
+        if (forced >= 2) break;  // the forced size (or the next one the device can schedule)
+    }
+    const bool one_launch = !p.holefill && !compact_in_attention && p.policy != RA_POLICY_SNAPKV &&
+                            forced != RA_EVICT_TWO_KERNELS && cl > 0 && ctx->r <= kEvMaxEvicted;
+    if (one_launch) {
+        p.ev_reps = reps;
+        p.ev_exact = (ctx->evict_mode & RA_EVICT_EXACT) ? 1 : 0;
+        ProfScope ps(ctx, RA_KERNEL_EVICT, moved * 2.0 * (2 * kRowBytes + 4), s);
+        e = launch_evict(p, cl, s);
+        ps.done();
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "evict launch");
+        return RA_OK;
     }
     {
         // with order-free compaction the select kernel also moves m rows per head (read and write)
@@ -454,6 +535,7 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);
     ctx->off_err = take(256);
+    ctx->off_evplan = take((size_t)2 * layers * batch * kv_heads * (r + 1) * 4);
     ctx->base_bytes = o;
     int maxlp = 0;
     for (int b = 0; b < batch; ++b) maxlp = std::max(maxlp, (int)prompt_lens[b]);
@@ -513,6 +595,7 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.partial = (float*)(a + ctx->off_partial);
     Ly.arrive = (int32_t*)(a + ctx->off_arrive);
     Ly.err = (int32_t*)(a + ctx->off_err);
+    Ly.evplan = (int32_t*)(a + ctx->off_evplan);
     Ly.qring = ctx->scoring ? (uint16_t*)(a + ctx->off_qring) : nullptr;
     Ly.qstats = ctx->scoring ? (float2*)(a + ctx->off_qstats) : nullptr;
     Ly.scores = ctx->scoring ? (float*)(a + ctx->off_scores) : nullptr;
@@ -558,6 +641,7 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
         if ((rc = make_tmap(ctx, &ctx->tmap_v[sh], Ly.vpool, ctx->total_rows, tile)) != RA_OK) return rc;
         if ((e = attn_prepare(sh, ctx->G)) != cudaSuccess) return cuda_fail(ctx, e, "attention kernel attributes");
     }
+    if ((e = evict_prepare(ctx->evict_active)) != cudaSuccess) return cuda_fail(ctx, e, "eviction kernel attributes");
     if (ctx->scoring) {
         if ((rc = make_tmap(ctx, &ctx->tmap_ks, Ly.kpool, ctx->total_rows, kScoreTile)) != RA_OK) return rc;
         const long long win_rows = (long long)ctx->L * ctx->B * ctx->KVH * ctx->r * ctx->G;
@@ -573,6 +657,20 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     std::fill(ctx->c.begin(), ctx->c.end(), 0);
     std::fill(ctx->nev.begin(), ctx->nev.end(), 0);
     std::fill(ctx->score_n.begin(), ctx->score_n.end(), 0);
+    if (!ctx->side) {
+        if ((e = cudaStreamCreateWithFlags(&ctx->side, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&ctx->fork_ev, cudaEventDisableTiming)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&ctx->plan_ev, cudaEventDisableTiming)) != cudaSuccess)
+            return cuda_fail(ctx, e, "side stream");
+    }
+    ctx->plan_pending = false;
+    ctx->parity = 0;
+    ctx->plan_g.assign((size_t)2 * ctx->L * ctx->B, -1);
+    ctx->plan_n.assign((size_t)2 * ctx->L * ctx->B, -1);
+    ctx->rbase.resize((size_t)ctx->L * ctx->B);
+    ctx->sbase.resize((size_t)ctx->B);
+    for (size_t i = 0; i < ctx->rbase.size(); ++i) ctx->rbase[i] = (int32_t)i;
+    for (int b = 0; b < ctx->B; ++b) ctx->sbase[b] = ctx->L * ctx->B + b;
     return RA_OK;
 }
 
@@ -651,6 +749,7 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block)
     }
     ctx->policy = policy;
     ctx->block = policy == RA_POLICY_BLOCK ? block : 1;
+    std::fill(ctx->plan_g.begin(), ctx->plan_g.end(), -1);  // sets computed ahead under another policy
     return RA_OK;
 }
 
@@ -671,6 +770,17 @@ int ra_set_attention_shape(ra_ctx* ctx, int shape)
     if (shape < RA_ATTN_SHAPE_AUTO || shape > RA_ATTN_SHAPE_NARROW)
         return fail(ctx, RA_ERR_INVALID_ARG, "unknown attention shape %d", shape);
     ctx->attn_shape = shape;
+    return RA_OK;
+}
+
+int ra_set_eviction_kernel(ra_ctx* ctx, int mode)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    const int base = mode & ~RA_EVICT_EXACT;
+    if (mode < 0 || base > kEvMaxCluster || (mode & ~(RA_EVICT_EXACT | 31)))
+        return fail(ctx, RA_ERR_INVALID_ARG, "eviction kernel mode %d: expected [0, %d], optionally | RA_EVICT_EXACT",
+                    mode, kEvMaxCluster);
+    ctx->evict_mode = mode;
     return RA_OK;
 }
 
@@ -832,8 +942,22 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
     return RA_OK;
 }
 
+namespace {
+int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                      uint16_t* out, float scale, void* stream, int plan_parity);
+}
+
 int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
                     uint16_t* out, float scale, void* stream)
+{
+    return decode_layer_impl(ctx, layer, q, k_new, v_new, out, scale, stream, -1);
+}
+
+namespace {
+// plan_parity >= 0: evicted sets computed ahead into that half of the plan buffer may be used
+// (ra_decode_step, which has ordered the stream after their computation)
+int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                      uint16_t* out, float scale, void* stream, int plan_parity)
 {
     int rc;
     if ((rc = check_bound(ctx)) != RA_OK) return rc;
@@ -886,6 +1010,17 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
         }
     }
     double compacted = 0;  // rows the attention launch writes as compaction
+    if (n > 0 && plan_parity >= 0 && !ep.holefill && !fuse_compaction && plan_usable(ctx)) {
+        bool all = true;  // every triggered sequence's evicted sets were computed ahead for this round
+        for (int i = 0; i < n && all; ++i) {
+            const size_t k = (size_t)plan_parity * ctx->L * ctx->B + (size_t)layer * ctx->B + ep.trig[i];
+            all = ctx->plan_g[k] == ep.trig_g[i] && ctx->plan_n[k] == ep.trig_n[i];
+        }
+        if (all) {
+            ep.ev_plan = ctx->lay.evplan;
+            ep.ev_plan_parity = plan_parity;
+        }
+    }
     if (n > 0) {
         ep.n_trig = n;
         if ((rc = run_eviction(ctx, ep, moved, s, fuse_compaction, score_early)) != RA_OK) return rc;
@@ -951,6 +1086,8 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     return RA_OK;
 }
 
+}  // namespace
+
 int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, const uint16_t* v_all, uint16_t* out_all,
                    float scale, void* stream)
 {
@@ -963,10 +1100,63 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
             if (ctx->active[b] && ctx->c[(size_t)l * ctx->B + b] >= ctx->Cmax)
                 return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d is full (evict not called)", l, b);
     const size_t qs = (size_t)ctx->B * ctx->H * kHeadDim, ks = (size_t)ctx->B * ctx->KVH * kHeadDim;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e;
+    if (ctx->plan_pending) {  // the evicted sets of this step, computed during the previous one
+        if ((e = cudaStreamWaitEvent(s, ctx->plan_ev, 0)) != cudaSuccess) return cuda_fail(ctx, e, "plan wait");
+        ctx->plan_pending = false;
+    }
+    const int cur = ctx->parity, nxt = 1 - cur;
+    std::fill(ctx->plan_g.begin() + (size_t)nxt * ctx->L * ctx->B, ctx->plan_g.begin() + (size_t)(nxt + 1) * ctx->L * ctx->B,
+              -1);
+    if (plan_usable(ctx)) {
+        // The sequences whose trigger fires at the next step (from layer 0's counters after this
+        // step): their evicted sets in every layer, computed on the side stream beside this step.
+        // The fork orders the plan after the previous step, the last reader of half nxt.
+        EvictParams pp{};
+        pp.lay = ctx->lay;
+        pp.policy = ctx->policy;
+        pp.ev_exact = (ctx->evict_mode & RA_EVICT_EXACT) ? 1 : 0;
+        pp.ev_plan_parity = nxt;
+        int n = 0;
+        for (int b = 0; b < ctx->B; ++b) {
+            if (!ctx->active[b]) continue;
+            const int g1 = ctx->g[b] + 1, c1 = ctx->c[b] + 1;
+            const bool fires = g1 % ctx->r == 0 && c1 - ctx->r > ctx->K;
+            const int g2 = g1 + 1, c2 = (fires ? ctx->K + ctx->r : c1) + 1;
+            if (g2 % ctx->r == 0 && c2 - ctx->r > ctx->K && c2 - ctx->r <= ctx->K + ctx->r) {
+                pp.trig[n] = (int16_t)b;
+                pp.trig_g[n] = g2;
+                pp.trig_n[n] = c2 - ctx->r;
+                ++n;
+            }
+        }
+        if (n > 0) {
+            pp.n_trig = n;
+            if ((e = cudaEventRecord(ctx->fork_ev, s)) != cudaSuccess ||
+                (e = cudaStreamWaitEvent(ctx->side, ctx->fork_ev, 0)) != cudaSuccess)
+                return cuda_fail(ctx, e, "plan fork");
+            {
+                ProfScope ps(ctx, RA_KERNEL_PLAN, 0.0, ctx->side);
+                e = launch_plan(pp, ctx->side);
+                ps.done();
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "plan launch");
+            if ((e = cudaEventRecord(ctx->plan_ev, ctx->side)) != cudaSuccess) return cuda_fail(ctx, e, "plan record");
+            ctx->plan_pending = true;
+            for (int i = 0; i < n; ++i)
+                for (int l = 0; l < ctx->L; ++l) {
+                    const size_t k = (size_t)nxt * ctx->L * ctx->B + (size_t)l * ctx->B + pp.trig[i];
+                    ctx->plan_g[k] = pp.trig_g[i];
+                    ctx->plan_n[k] = pp.trig_n[i];
+                }
+        }
+    }
     for (int l = 0; l < ctx->L; ++l)
-        if ((rc = ra_decode_layer(ctx, l, q_all + l * qs, k_all + l * ks, v_all + l * ks, out_all + l * qs, scale,
-                                  stream)) != RA_OK)
+        if ((rc = decode_layer_impl(ctx, l, q_all + l * qs, k_all + l * ks, v_all + l * ks, out_all + l * qs, scale,
+                                    stream, cur)) != RA_OK)
             return rc;
+    ctx->parity = nxt;
     return RA_OK;
 }
 
@@ -1127,6 +1317,12 @@ int ra_profile_read(ra_ctx* ctx, int kind, double* total_ms, int64_t* launches, 
 void ra_destroy(ra_ctx* ctx)
 {
     if (!ctx) return;
+    if (ctx->side) {
+        cudaStreamSynchronize(ctx->side);
+        cudaStreamDestroy(ctx->side);
+        cudaEventDestroy(ctx->fork_ev);
+        cudaEventDestroy(ctx->plan_ev);
+    }
     for (auto& pr : ctx->pending) {
         cudaEventSynchronize(pr.stop);
         cudaEventDestroy(pr.start);

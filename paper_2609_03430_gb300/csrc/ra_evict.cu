@@ -14,6 +14,11 @@
 //                   slots every key follows the candidate's position.
 //                   With order-free slots the select CTA also refills the
 //                   evicted slots in place from the newest ones (no compact).
+//   evict_kernel    the random policy and its key-per-ordinal variants in one
+//                   launch: a thread-block cluster per triggered head draws the
+//                   keys, selects the evicted set exactly across the cluster
+//                   through distributed shared memory, and moves the survivors
+//                   order-preserving with bulk copies (details below).
 //   compact_kernel  many CTAs per triggered head: order-preserving move of the
 //                   survivors (kept candidates, then the buffer rows) into
 //                   the head's spare region with coalesced 16-byte copies
@@ -21,6 +26,7 @@
 //                   the cache into it).  Out of place, so CTAs never wait on
 //                   each other; the old region becomes the spare.
 #include <cuda_runtime.h>
+#include <limits.h>
 #include <stdint.h>
 
 #include "ra_internal.h"
@@ -406,6 +412,634 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
     }
 }
 
+// ----------------------------------------------------------------------------- evict (select + compact)
+// One launch per eviction round: for every triggered (seq, KV head), `reps` thread-block clusters
+// of CL CTAs.  Each cluster selects the head's evicted set on its own (the replicas of a head
+// compute the same set); the head's cached slots are cut into reps x CL equal row ranges, one
+// per CTA, for the copy.  CTA k of a cluster draws the keys of the candidates
+// [k N / CL, (k + 1) N / CL).
+//
+//   1. Keys of the own candidates (the same key rules as select_kernel), while the region
+//      tables load; then every warp starts TMA bulk copies of its first chunks of K and V rows
+//      into shared memory: the rows are read whatever the draw decides (about r of K + r are
+//      evicted), so the copies overlap the selection, and with early = 1 the previous kernel's
+//      tail too.
+//   2. The evicted set is the m = N - K largest (key, ordinal) pairs, found exactly.
+//      Random and shared draws (uniform 32-bit keys) first try a cut: only keys >= tau, with
+//      tau set so that about 2m + 32 of the N candidates pass; each CTA lists its passing
+//      candidates, the cluster exchanges the lists through distributed shared memory (one
+//      barrier) and ranks them exactly.  If at least m passed (all but certainly), the top m
+//      are the evicted set, since every candidate below the cut ranks lower.  Otherwise, and
+//      for the other policies, radix passes over 8-bit digits from the top: each CTA's
+//      histogram is summed by every CTA through distributed shared memory until the digit bin
+//      holding the boundary has at most kEvCap candidates, which are gathered and ranked; if
+//      all 32 bits tie, the largest ordinals are evicted first, CTA by CTA.  The CTAs then
+//      exchange their evicted ordinals.  Either way every CTA ends with the whole ascending
+//      list of evicted ordinals.
+//   3. Slot j moves to j - (evicted ordinals below j); each warp stores the runs of surviving
+//      rows of its chunks with bulk copies shared -> global (positions by plain stores),
+//      refilling its buffers as they drain.  Out of place into the head's spare region, as
+//      compact_kernel; CTA 0 of replica 0 swaps the region tables.
+constexpr int kEvThreads = 256;
+constexpr int kEvWarps = kEvThreads / 32;
+constexpr int kEvCap = kEvMaxEvicted;  // candidates gathered for an exact ranking; also the most a round evicts
+constexpr uint64_t kEvWaitLimitNs = 2000000000ull;
+static_assert(kEvThreads == 256, "one thread per histogram bin");
+static_assert(kEvCap <= 2 * kEvThreads, "a plan's ordinals are read two per thread");
+static_assert(kEvMaxLocal % 32 == 0, "whole bitmap words");
+static_assert(kMaxCandidates + 128 <= 65536, "ordinals and the CTA rank share one 32-bit word");
+
+struct EvShared {
+    uint32_t keys[kEvMaxLocal];
+    uint32_t hist[2][256];            // this CTA's histogram of the current digit (double-buffered)
+    uint32_t tot[256];                // the cluster's
+    uint2 blist[kEvCap];              // own listed candidates: (key, ordinal)
+    uint2 ball[kEvCap];               // everyone's: (key, rank << 16 | ordinal), ordered as (key, ordinal)
+    int32_t evlist[kEvCap];           // every evicted ordinal, ascending
+    int32_t evown[kEvCap];            // the cut: the evicted ordinals in any order; radix passes: own, ascending
+    uint32_t evown_n;
+    uint32_t bcnt, nev;
+    uint32_t sel[6];
+    uint32_t cnt[kEvMaxCluster];
+    uint64_t bar[kEvWarps][kEvBufs];
+};
+
+// Gather the cluster's lists (S.blist of every CTA, S.bcnt entries each) into S.ball, tagging
+// each entry with its CTA's rank; returns the total.  Entries keep the (key, ordinal) order.
+__device__ __forceinline__ int gather_lists(EvShared& S, int CL, int tid)
+{
+    if (tid < CL) S.cnt[tid] = ld_dsmem_u32(dsmem_addr(&S.bcnt, tid));
+    __syncthreads();
+    int total = 0;
+    for (int k = 0; k < CL; ++k) total += (int)S.cnt[k];
+    if (total > kEvCap) return total;
+    for (int e = tid; e < total; e += kEvThreads) {
+        int k = 0, off = 0;
+        while (e >= off + (int)S.cnt[k]) off += (int)S.cnt[k++];
+        const uint2 x = ld_dsmem_u32x2(dsmem_addr(&S.blist[e - off], k));
+        S.ball[e] = make_uint2(x.x, ((uint32_t)k << 16) | x.y);  // ranks grow with ordinals: order kept
+    }
+    return total;
+}
+
+// Number of evicted ordinals below j (S.evlist ascending, n entries).
+__device__ __forceinline__ int ev_below(const EvShared& S, int n, int j)
+{
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (S.evlist[mid] < j) lo = mid + 1; else hi = mid;
+    }
+    return lo;
+}
+
+template <int R, int NB>
+__global__ void __launch_bounds__(kEvThreads, 1) evict_kernel(const __grid_constant__ EvictParams p)
+{
+    static_assert(R <= 32 && NB >= 3 && NB == kEvBufs, "a lane per row of a chunk; refills trail by one chunk");
+    extern __shared__ __align__(128) uint8_t ev_dyn[];  // [warp][buffer][K rows R][V rows R]
+    __shared__ EvShared S;
+    constexpr int kBufBytes = 2 * R * kRowBytes;
+    const DevLayout& L = p.lay;
+    const int CL = (int)gridDim.x, reps = p.ev_reps;
+    const uint32_t rank = cluster_ctarank();
+    const int h = blockIdx.y / reps, rep = blockIdx.y - h * reps, t = blockIdx.z;
+    const int b = p.trig[t];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int c = p.trig_c[t], N = p.trig_n[t], g = p.trig_g[t];
+    const int m = N - L.K;
+    const int head_id = b * L.KVH + h;
+    // The host mirror rules these out; every CTA of the launch decides alike, so they leave together.
+    // (a CTA keeps the keys of its candidates only when it selects itself, without a plan)
+    if (m < 1 || m > L.r || m > kEvCap || N > c || N > kMaxCandidates ||
+        (!p.ev_plan && (N + CL - 1) / CL > kEvMaxLocal) || CL > kEvMaxCluster || reps < 1) {
+        pdl_wait();
+        pdl_launch_dependents();
+        if (tid == 0 && rank == 0 && rep == 0) atomicExch(L.err, kDeviceErrPlan);
+        return;
+    }
+    const int j0 = (int)((long long)rank * N / CL), nloc = (int)((long long)(rank + 1) * N / CL) - j0;
+    const int U = reps * CL, u = rep * CL + (int)rank;  // this CTA's share of the copy
+    const int s0 = (int)((long long)u * c / U), s1 = (int)((long long)(u + 1) * c / U);
+    uint8_t* wbuf = ev_dyn + (size_t)warp * NB * kBufBytes;
+    uint64_t* wbar = S.bar[warp];
+    S.hist[0][tid] = 0;
+    if (tid == 0) S.bcnt = 0;
+    __syncthreads();
+    // With p.early the host has checked that the previous kernel writes none of this layer's
+    // rows or positions: the copies and the selection start before waiting for it.  The regions
+    // come from the host's mirror of the tables (checked against them below).
+    if (!p.early) pdl_wait();
+    const int src = p.trig_src[t] * L.KVH + h, dst = p.trig_dst[t] * L.KVH + h;
+
+    // 1. keys (random / shared / recency keys need no memory, so they overlap the table loads),
+    //    the cut's list or the first digit's histogram, then the first copies
+    const bool cut = (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) && !p.ev_exact;
+    // tau = 2^32 (1 - E / N) with E = 2m + 32 expected to pass (all of them when E >= N)
+    const uint64_t E = 2ull * (uint64_t)m + 32ull;
+    const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
+    const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
+    const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
+    const int32_t* spos = L.pos + (size_t)src * L.Cmax;
+    auto record = [&](int i, uint32_t key) {  // the key of local candidate i: kept, listed or counted
+        S.keys[i] = key;
+        if (!cut) {
+            atomicAdd(&S.hist[0][key >> 24], 1u);
+        } else if (key >= tau) {
+            const uint32_t at = atomicAdd(&S.bcnt, 1u);
+            if (at < (uint32_t)kEvCap) S.blist[at] = make_uint2(key, (uint32_t)(j0 + i));
+        }
+    };
+    // a precomputed plan: the evicted ordinals of this head, [count][ordinals ascending]
+    const int32_t* plan = p.ev_plan ? p.ev_plan + (size_t)(((size_t)p.ev_plan_parity * L.L + p.layer) * L.B * L.KVH +
+                                                           (size_t)b * L.KVH + h) * (L.r + 1)
+                                    : nullptr;
+    // the plan's count and this thread's share of its ordinals, read before the row copies
+    // start, so that the reads do not queue behind them
+    int plan_n = 0, plan_v0 = 0, plan_v1 = 0;
+    if (plan) {
+        plan_n = __ldcg(plan);
+        if (tid < m) plan_v0 = __ldcg(plan + 1 + tid);
+        if (tid + kEvThreads < m) plan_v1 = __ldcg(plan + 1 + tid + kEvThreads);
+    } else if (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) {
+        // four independent Philox chains per thread at a time (each chain is 10 serial rounds)
+        for (int i0 = tid; i0 < nloc; i0 += 4 * kEvThreads) {
+            uint32_t kq[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                kq[q] = philox4x32_10_w0((uint32_t)(j0 + i0 + q * kEvThreads), (uint32_t)g, (uint32_t)p.layer, id, k0, k1);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                if (i0 + q * kEvThreads < nloc) record(i0 + q * kEvThreads, kq[q]);
+        }
+    } else {
+        for (int i = tid; i < nloc; i += kEvThreads) {
+            const int j = j0 + i;
+            record(i, p.policy == RA_POLICY_RECENCY  // the K newest candidates score lowest
+                          ? (uint32_t)(N - 1 - j)
+                          : philox4x32_10_w0((uint32_t)(__ldg(spos + j) / p.block), (uint32_t)g, (uint32_t)p.layer,
+                                             (uint32_t)head_id, k0, k1));
+        }
+    }
+    if (lane == 0) {  // this warp's copy barriers
+        for (int i = 0; i < NB; ++i) mbar_init(&wbar[i], 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    const long long srow0 = L.gen_row0 + (long long)src * L.Cmax, drow0 = L.gen_row0 + (long long)dst * L.Cmax;
+    int32_t* dpos = L.pos + (size_t)dst * L.Cmax;
+    // chunk w + k * kEvWarps of the CTA's rows goes to buffer k % NB of warp w
+    const int nch = (s1 - s0 + R - 1) / R;
+    auto issue_load = [&](int k) {
+        const int a = s0 + (warp + k * kEvWarps) * R, n = min(R, s1 - a);
+        uint8_t* buf = wbuf + (k % NB) * kBufBytes;
+        mbar_arrive_expect_tx(&wbar[k % NB], 2u * (uint32_t)n * kRowBytes);
+        bulk_load(buf, L.kpool + (srow0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &wbar[k % NB]);
+        bulk_load(buf + R * kRowBytes, L.vpool + (srow0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &wbar[k % NB]);
+    };
+    const int mine = nch > warp ? (nch - warp + kEvWarps - 1) / kEvWarps : 0;  // this warp's chunks
+    int issued = min(NB, mine);
+    if (lane == 0)
+        for (int k = 0; k < issued; ++k) issue_load(k);
+
+    // 2. the selection
+    bool done = false;  // S.evlist holds the evicted set
+    if (plan) {  // computed ahead: check that it is an ascending list of m candidates
+        if (tid == 0) S.bcnt = 0;
+        const int n = plan_n;
+        if (n == m) {
+            if (tid < m) S.evlist[tid] = plan_v0;
+            if (tid + kEvThreads < m) S.evlist[tid + kEvThreads] = plan_v1;
+        }
+        __syncthreads();
+        bool bad = n != m;
+        for (int i = tid; i < m && !bad; i += kEvThreads)
+            bad = S.evlist[i] < 0 || S.evlist[i] >= N || (i + 1 < m && S.evlist[i] >= S.evlist[i + 1]);
+        if (bad) S.bcnt = 1;
+        __syncthreads();
+        if (tid == 0) S.nev = S.bcnt ? 0u : (uint32_t)m;  // a bad plan fails the check below
+        done = true;
+    }
+    if (!done && cut) {
+        cluster_sync();  // every CTA's list is complete
+        const int total = gather_lists(S, CL, tid);
+        __syncthreads();
+        if (total >= m && total <= kEvCap) {  // the top m of the list are the evicted set
+            if (tid == 0) S.nev = 0;
+            __syncthreads();
+            for (int e = warp; e < total; e += kEvWarps) {  // rank among the listed pairs, a warp per pair
+                const uint2 x = S.ball[e];
+                int above = 0;
+                for (int f = lane; f < total; f += 32) {
+                    const uint2 y = S.ball[f];
+                    above += (y.x > x.x || (y.x == x.x && y.y > x.y)) ? 1 : 0;
+                }
+                above = __reduce_add_sync(0xffffffffu, above);
+                if (lane == 0 && above < m) S.evown[atomicAdd(&S.nev, 1u)] = (int32_t)(x.y & 0xFFFFu);  // evicted
+            }
+            __syncthreads();
+            for (int e = warp; e < m; e += kEvWarps) {  // position among the m evicted, by ordinal
+                const int je = S.evown[e];
+                int below = 0;
+                for (int f = lane; f < m; f += 32) below += S.evown[f] < je ? 1 : 0;
+                below = __reduce_add_sync(0xffffffffu, below);
+                if (lane == 0) S.evlist[below] = je;
+            }
+            done = true;
+        }
+        // (otherwise: the radix passes below, from the first digit's histogram)
+        if (!done) {
+            for (int i = tid; i < nloc; i += kEvThreads) atomicAdd(&S.hist[0][S.keys[i] >> 24], 1u);
+        }
+    }
+    if (!done) {
+        uint32_t prefix = 0, mask = 0, need = (uint32_t)m;  // evicted still to find at or below the prefix
+        uint32_t T = 0xFFFFFFFFu;
+        int jT = INT_MAX;
+        int hb = 0;
+        for (int d = 0; d < 4; ++d) {
+            const int shift = 24 - 8 * d;
+            cluster_sync();  // every CTA's S.hist[hb] is complete (and, after the cut, no list is read any more)
+            uint32_t v[kEvMaxCluster];  // bin tid of every CTA's histogram, all loads in flight at once
+#pragma unroll
+            for (int k = 0; k < kEvMaxCluster; ++k) v[k] = k < CL ? ld_dsmem_u32(dsmem_addr(&S.hist[hb][tid], k)) : 0u;
+            {
+                uint32_t sum = 0;
+#pragma unroll
+                for (int k = 0; k < kEvMaxCluster; ++k) sum += v[k];
+                S.tot[tid] = sum;
+            }
+            __syncthreads();
+            if (warp == 0) {  // the bin of the need-th largest, scanning from the top
+                uint32_t loc[8], sum = 0;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    loc[q] = S.tot[255 - (8 * lane + q)];
+                    sum += loc[q];
+                }
+                uint32_t incl = sum;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const uint32_t x = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += x;
+                }
+                const uint32_t excl = incl - sum;
+                if (excl < need && need <= incl) {
+                    uint32_t cum = excl;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        if (need <= cum + loc[q]) {
+                            S.sel[0] = 255u - (uint32_t)(8 * lane + q);
+                            S.sel[1] = cum;
+                            S.sel[2] = loc[q];
+                            break;
+                        }
+                        cum += loc[q];
+                    }
+                }
+            }
+            __syncthreads();
+            const uint32_t B = S.sel[0], cnt = S.sel[2];
+            need -= S.sel[1];
+            prefix |= B << shift;
+            mask |= 0xFFu << shift;
+            if (cnt <= (uint32_t)kEvCap) {  // gather the boundary candidates and rank them exactly
+                if (tid == 0) S.bcnt = 0;
+                __syncthreads();
+                for (int i = tid; i < nloc; i += kEvThreads) {
+                    const uint32_t key = S.keys[i];
+                    if ((key & mask) == prefix) S.blist[atomicAdd(&S.bcnt, 1u)] = make_uint2(key, (uint32_t)(j0 + i));
+                }
+                cluster_sync();
+                const int total = gather_lists(S, CL, tid);
+                __syncthreads();
+                for (int e = warp; e < total; e += kEvWarps) {  // a warp per pair
+                    const uint2 x = S.ball[e];
+                    uint32_t above = 0;
+                    for (int f = lane; f < total; f += 32) {
+                        const uint2 y = S.ball[f];
+                        above += (y.x > x.x || (y.x == x.x && y.y > x.y)) ? 1u : 0u;
+                    }
+                    above = __reduce_add_sync(0xffffffffu, above);
+                    if (lane == 0 && above == need - 1) {  // the smallest evicted pair
+                        S.sel[3] = x.x;
+                        S.sel[4] = x.y & 0xFFFFu;
+                    }
+                }
+                __syncthreads();
+                T = S.sel[3];
+                jT = (int)S.sel[4];
+                break;
+            }
+            if (d == 3) {  // more than kEvCap candidates share all 32 bits: the largest ordinals go first
+                if (tid == (int)B) {  // this thread read bin B of every CTA: their tie counts
+                    uint32_t after = 0;
+#pragma unroll
+                    for (int k = kEvMaxCluster - 1; k >= 0; --k) {
+                        if (k >= CL) continue;
+                        const uint32_t e = need > after ? min(need - after, v[k]) : 0u;  // ties CTA k evicts
+                        if (k == (int)rank) {
+                            S.sel[3] = v[k] - e;  // local index of the first evicted tie
+                            S.sel[4] = e;
+                        }
+                        after += v[k];
+                    }
+                }
+                __syncthreads();
+                T = prefix;
+                if (S.sel[4] > 0 && warp == 0) {  // ordinal of local tie number S.sel[3]
+                    uint32_t seen = 0;
+                    const uint32_t want = S.sel[3];
+                    for (int i0 = 0; i0 < nloc; i0 += 32) {
+                        const int i = i0 + lane;
+                        const uint32_t eq = __ballot_sync(0xffffffffu, i < nloc && S.keys[i] == T);
+                        if (seen + __popc(eq) > want) {
+                            uint32_t e = eq;
+                            for (uint32_t q = seen; q < want; ++q) e &= e - 1u;
+                            if (lane == 0) S.sel[5] = (uint32_t)(j0 + i0 + __ffs(e) - 1);
+                            break;
+                        }
+                        seen += __popc(eq);
+                    }
+                }
+                __syncthreads();
+                jT = S.sel[4] > 0 ? (int)S.sel[5] : INT_MAX;
+                break;
+            }
+            hb ^= 1;  // this buffer was last read by the other CTAs before the barrier above
+            S.hist[hb][tid] = 0;
+            __syncthreads();
+            for (int i = tid; i < nloc; i += kEvThreads) {
+                const uint32_t key = S.keys[i];
+                if ((key & mask) == prefix) atomicAdd(&S.hist[hb][(key >> (shift - 8)) & 255u], 1u);
+            }
+        }
+        // own evicted ordinals, ascending (ballot compaction), then every CTA's, in rank order
+        // (into lists of their own: other CTAs may still be reading the boundary lists)
+        if (warp == 0) {
+            uint32_t off = 0;
+            for (int i0 = 0; i0 < nloc; i0 += 32) {
+                const int i = i0 + lane;
+                const uint32_t key = i < nloc ? S.keys[i] : 0u;
+                const bool ev = i < nloc && (key > T || (key == T && j0 + i >= jT));
+                const uint32_t bits = __ballot_sync(0xffffffffu, ev);
+                const uint32_t at = off + __popc(bits & ((1u << lane) - 1u));
+                if (ev && at < (uint32_t)kEvCap) S.evown[at] = j0 + i;
+                off += __popc(bits);
+            }
+            if (lane == 0) S.evown_n = off;
+        }
+        cluster_sync();  // every CTA's evicted list is complete
+        if (tid < CL) S.cnt[tid] = ld_dsmem_u32(dsmem_addr(&S.evown_n, tid));
+        __syncthreads();
+        int total = 0;
+        for (int k = 0; k < CL; ++k) total += (int)S.cnt[k];
+        if (total <= kEvCap) {
+            for (int e = tid; e < total; e += kEvThreads) {
+                int k = 0, off = 0;
+                while (e >= off + (int)S.cnt[k]) off += (int)S.cnt[k++];
+                S.evlist[e] = (int32_t)ld_dsmem_u32(dsmem_addr(&S.evown[e - off], k));
+            }
+        }
+        if (tid == 0) S.nev = (uint32_t)total;  // (a total other than m fails the check below)
+    }
+    cluster_arrive();  // the last read of another CTA's shared memory; waited for before exit
+    __syncthreads();
+    const int nev = (int)S.nev;
+    const bool ok = nev == m;  // the same in every CTA of the launch
+
+    if (p.early) pdl_wait();
+    pdl_launch_dependents();
+    if (tid == 0 && rank == 0 && rep == 0) {
+        int32_t* reg = L.region + ((size_t)p.layer * L.B + b) * L.KVH + h;
+        int32_t* spr = L.spare + b * L.KVH + h;
+        if (ok && *reg == src && *spr == dst) {
+            *reg = dst;
+            *spr = src;
+        } else {
+            atomicExch(L.err, kDeviceErrPlan);
+        }
+    }
+    // 3. the survivors' rows, chunk by chunk as their copies land; a buffer is refilled one chunk
+    //    later, once its stores have read it
+    for (int k = 0; k < issued; ++k) {
+        const int a = s0 + (warp + k * kEvWarps) * R, n = min(R, s1 - a);
+        const uint8_t* buf = wbuf + (k % NB) * kBufBytes;
+        // lane 0 alone reads the buffer (its bulk stores), so lane 0 alone waits; the verdict is the warp's
+        bool landed = true;
+        if (lane == 0) landed = mbar_wait_bounded(&wbar[k % NB], (uint32_t)((k / NB) & 1), kEvWaitLimitNs);
+        if (!__shfl_sync(0xffffffffu, (int)landed, 0)) {
+            if (lane == 0) {
+                atomicExch(L.err, kDeviceErrTimeout);
+                for (int q = k + 1; q < issued; ++q)  // let the copies already issued land (bounded)
+                    (void)mbar_wait_bounded(&wbar[q % NB], (uint32_t)((q / NB) & 1), kEvWaitLimitNs);
+            }
+            break;
+        }
+        if (ok) {
+            if (lane < n) {
+                const int j = a + lane, e = ev_below(S, nev, j);
+                if (e == nev || S.evlist[e] != j) dpos[j - e] = spos[j];
+            }
+            if (lane == 0) {
+                int e = ev_below(S, nev, a);  // evicted ordinals below the run start
+                for (int q = a; q < a + n;) {
+                    const int nx = e < nev ? S.evlist[e] : INT_MAX;
+                    const int v = min(a + n, nx);
+                    if (v > q) {
+                        const long long drow = drow0 + (q - e);
+                        bulk_store(L.kpool + drow * kHeadDim, buf + (q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
+                        bulk_store(L.vpool + drow * kHeadDim, buf + (R + q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
+                    }
+                    if (nx < a + n) {  // skip the evicted row
+                        q = nx + 1;
+                        ++e;
+                    } else {
+                        q = v;
+                    }
+                }
+                bulk_commit();
+                if (k >= 1 && issued < mine) {  // chunk issued = k + NB - 1 into the buffer of chunk k - 1
+                    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                    issue_load(issued);
+                }
+            }
+            if (k >= 1 && issued < mine) ++issued;  // warp-uniform
+        }
+        __syncwarp();
+    }
+    if (lane == 0) bulk_wait_all();
+    cluster_wait();
+}
+
+// ----------------------------------------------------------------------------- plan (evicted sets ahead)
+// The random draw reads no cache data: a candidate's key depends only on (ordinal, step, layer,
+// head), so the evicted set of a firing step is known as soon as the counters are.  plan_kernel
+// computes it ahead, one CTA per (layer, sequence, KV head), with the same exact rules as
+// evict_kernel: the sampled cut and an exact ranking of the listed pairs, or -- when fewer than
+// m pass, for recency keys, or with RA_EVICT_EXACT -- four radix passes over recomputed keys
+// (no key is stored: 7 KB of shared memory, so the kernel fits beside an attention CTA on the
+// same SM) and one ascending sweep that writes the evicted ordinals in order, ties at the
+// threshold evicted from the largest ordinal down.  Output: [m][ordinals ascending].
+constexpr int kPlanThreads = 256;
+constexpr int kPlanWarps = kPlanThreads / 32;
+
+struct PlanShared {
+    uint2 list[kEvCap];
+    int32_t ev[kEvCap];
+    uint32_t hist[256];
+    uint32_t wsum[2][kPlanWarps];
+    uint32_t cnt, nev;
+    uint32_t sel[4];
+};
+
+__device__ __forceinline__ uint32_t plan_key(const EvictParams& p, int layer, uint32_t id, int N, int g, int j)
+{
+    if (p.policy == RA_POLICY_RECENCY) return (uint32_t)(N - 1 - j);
+    return philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)layer, id, (uint32_t)p.lay.seed,
+                            (uint32_t)(p.lay.seed >> 32));
+}
+
+__global__ void __launch_bounds__(kPlanThreads) plan_kernel(const __grid_constant__ EvictParams p)
+{
+    __shared__ PlanShared S;
+    const DevLayout& L = p.lay;
+    const int h = blockIdx.x, t = blockIdx.y, layer = blockIdx.z;
+    const int b = p.trig[t], N = p.trig_n[t], g = p.trig_g[t];
+    const int m = N - L.K;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    int32_t* out = L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
+    if (m < 1 || m > L.r || m > kEvCap || N > kMaxCandidates) {  // the host rules this out; the copy rejects it
+        if (tid == 0) out[0] = -1;
+        return;
+    }
+    const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)(b * L.KVH + h);
+    const bool cut = (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) && !p.ev_exact;
+    if (cut) {
+        const uint64_t E = 2ull * (uint64_t)m + 32ull;
+        const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
+        if (tid == 0) {
+            S.cnt = 0;
+            S.nev = 0;
+        }
+        __syncthreads();
+        for (int j0 = tid; j0 < N; j0 += 4 * kPlanThreads) {  // four independent Philox chains at a time
+            uint32_t kq[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) kq[q] = plan_key(p, layer, id, N, g, j0 + q * kPlanThreads);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int j = j0 + q * kPlanThreads;
+                if (j < N && kq[q] >= tau) {
+                    const uint32_t at = atomicAdd(&S.cnt, 1u);
+                    if (at < (uint32_t)kEvCap) S.list[at] = make_uint2(kq[q], (uint32_t)j);
+                }
+            }
+        }
+        __syncthreads();
+        const int total = (int)S.cnt;
+        if (total >= m && total <= kEvCap) {  // the top m of the list are the evicted set
+            for (int e = tid; e < total; e += kPlanThreads) {
+                const uint2 x = S.list[e];
+                int above = 0;
+#pragma unroll 8
+                for (int f = 0; f < total; ++f) {
+                    const uint2 y = S.list[f];
+                    above += (y.x > x.x || (y.x == x.x && y.y > x.y)) ? 1 : 0;
+                }
+                if (above < m) S.ev[atomicAdd(&S.nev, 1u)] = (int32_t)x.y;
+            }
+            __syncthreads();
+            for (int e = tid; e < m; e += kPlanThreads) {  // ascending by ordinal
+                const int je = S.ev[e];
+                int below = 0;
+#pragma unroll 8
+                for (int f = 0; f < m; ++f) below += S.ev[f] < je ? 1 : 0;
+                out[1 + below] = je;
+            }
+            if (tid == 0) out[0] = m;
+            return;
+        }
+    }
+    // exact radix passes over recomputed keys: the need-th largest key T after four digits
+    uint32_t prefix = 0, mask = 0, need = (uint32_t)m, ties = 0;
+    for (int d = 0; d < 4; ++d) {
+        const int shift = 24 - 8 * d;
+        S.hist[tid] = 0;
+        __syncthreads();
+        for (int j = tid; j < N; j += kPlanThreads) {
+            const uint32_t key = plan_key(p, layer, id, N, g, j);
+            if ((key & mask) == prefix) atomicAdd(&S.hist[(key >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (warp == 0) {
+            uint32_t loc[8], sum = 0;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                loc[q] = S.hist[255 - (8 * lane + q)];
+                sum += loc[q];
+            }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t x = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += x;
+            }
+            const uint32_t excl = incl - sum;
+            if (excl < need && need <= incl) {
+                uint32_t cum = excl;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    if (need <= cum + loc[q]) {
+                        S.sel[0] = 255u - (uint32_t)(8 * lane + q);
+                        S.sel[1] = cum;
+                        S.sel[2] = loc[q];
+                        break;
+                    }
+                    cum += loc[q];
+                }
+            }
+        }
+        __syncthreads();
+        need -= S.sel[1];
+        ties = S.sel[2];
+        prefix |= S.sel[0] << shift;
+        mask |= 0xFFu << shift;
+        __syncthreads();  // S.sel and S.hist are rewritten by the next pass
+    }
+    // evicted: key > T, and among the `ties` keys equal to T the `need` largest ordinals;
+    // an ascending sweep writes them in order
+    const uint32_t T = prefix, tie_from = ties - need;  // tie index from which ties are evicted
+    uint32_t base_ev = 0, base_tie = 0;
+    for (int c0 = 0; c0 < N; c0 += kPlanThreads) {
+        const int j = c0 + tid;
+        const uint32_t key = j < N ? plan_key(p, layer, id, N, g, j) : 0u;
+        const bool eq = j < N && key == T, gt = j < N && key > T;
+        const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+        if (lane == 0) S.wsum[0][warp] = __popc(eqb);
+        __syncthreads();
+        uint32_t tie_before = base_tie + __popc(eqb & ((1u << lane) - 1u)), tie_chunk = 0;
+        for (int w = 0; w < kPlanWarps; ++w) {
+            tie_before += w < warp ? S.wsum[0][w] : 0u;
+            tie_chunk += S.wsum[0][w];
+        }
+        const bool ev = gt || (eq && tie_before >= tie_from);
+        const uint32_t evb = __ballot_sync(0xffffffffu, ev);
+        if (lane == 0) S.wsum[1][warp] = __popc(evb);
+        __syncthreads();
+        uint32_t pos = base_ev + __popc(evb & ((1u << lane) - 1u)), ev_chunk = 0;
+        for (int w = 0; w < kPlanWarps; ++w) {
+            pos += w < warp ? S.wsum[1][w] : 0u;
+            ev_chunk += S.wsum[1][w];
+        }
+        if (ev && pos < (uint32_t)m) out[1 + pos] = j;
+        base_ev += ev_chunk;
+        base_tie += tie_chunk;
+        __syncthreads();  // S.wsum is rewritten by the next chunk
+    }
+    if (tid == 0) out[0] = base_ev == (uint32_t)m ? m : -1;
+}
+
 // ----------------------------------------------------------------------------- timeout probe
 // The failure path of every bounded wait, run on purpose: one arrival with 16 bytes of
 // transfer expected, and no copy ever issued, so the barrier's phase cannot complete; the
@@ -520,6 +1154,67 @@ cudaError_t launch_compact(const EvictParams& p, cudaStream_t s)
     const int chunks = (Cmax + kCompactChunk - 1) / kCompactChunk;
     return launch_pdl(compact_kernel, dim3(chunks, p.n_trig * p.lay.KVH), dim3(kCompactThreads),
                       p.lay.r * sizeof(int32_t), s, p);
+}
+
+namespace {
+constexpr size_t kEvSmem = (size_t)kEvWarps * kEvBufs * 2 * kEvRows * kRowBytes;
+
+cudaLaunchConfig_t evict_config(int cluster, int heads_reps, int n_trig, cudaStream_t s, cudaLaunchAttribute* attr)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)cluster, (unsigned)heads_reps, (unsigned)n_trig);
+    cfg.blockDim = dim3(kEvThreads);
+    cfg.dynamicSmemBytes = kEvSmem;
+    cfg.stream = s;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cfg;
+}
+}  // namespace
+
+// One-time attributes, and how many clusters of each size 1..kEvMaxCluster the device runs at
+// once (active[cl], 0 where that size cannot be scheduled).
+cudaError_t evict_prepare(int* active)
+{
+    auto kernel = evict_kernel<kEvRows, kEvBufs>;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kEvSmem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    bool any = false;
+    active[0] = 0;
+    for (int cl = 1; cl <= kEvMaxCluster; ++cl) {
+        cudaLaunchAttribute attr[2];
+        cudaLaunchConfig_t cfg = evict_config(cl, 1, 1, 0, attr);
+        cfg.numAttrs = 1;  // the cluster shape only
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+            (void)cudaGetLastError();
+            n = 0;
+        }
+        active[cl] = n;
+        any = any || n > 0;
+    }
+    return any ? cudaSuccess : cudaErrorInvalidConfiguration;
+}
+
+cudaError_t launch_evict(const EvictParams& p, int cluster, cudaStream_t s)
+{
+    if (cluster < 1 || cluster > kEvMaxCluster) return cudaErrorInvalidValue;
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = evict_config(cluster, p.lay.KVH * p.ev_reps, p.n_trig, s, attr);
+    return cudaLaunchKernelEx(&cfg, evict_kernel<kEvRows, kEvBufs>, p);
+}
+
+cudaError_t launch_plan(const EvictParams& p, cudaStream_t s)
+{
+    plan_kernel<<<dim3((unsigned)p.lay.KVH, (unsigned)p.n_trig, (unsigned)p.lay.L), kPlanThreads, 0, s>>>(p);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s)

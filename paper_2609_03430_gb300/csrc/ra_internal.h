@@ -36,6 +36,7 @@ struct DevLayout {
     float* partial;        // attention split partials
     int32_t* arrive;       // [B*KVH] split-piece arrival counters
     int32_t* err;          // device error word
+    int32_t* evplan;       // [2][L][B][KVH][r + 1] evicted sets computed ahead (plan_kernel)
     // scored policy (null when the context was bound without its buffers)
     uint16_t* qring;       // [L][B][KVH][r][G][128] bf16: query of step s in slot (s - 1) mod r
     float* scores;         // [L][B][KVH][Cmax] raw window score of each candidate of the latest round
@@ -75,9 +76,21 @@ struct EvictParams {
     int32_t trig_c[RA_MAX_BATCH];  // rows in the cache (a pending new token is not among them)
     int32_t trig_n[RA_MAX_BATCH];  // candidates (all rows but the newest r, counting a pending token)
     int32_t trig_g[RA_MAX_BATCH];  // step of the draw: generated tokens including this step's
+    // the host's mirror of the region tables: the triggered sequence's current region and its
+    // spare are region_base * KVH + kv_head (one-launch eviction; checked against the tables)
+    int32_t trig_src[RA_MAX_BATCH];
+    int32_t trig_dst[RA_MAX_BATCH];
     // scored policy: tiles (of kScoreTile rows) per CTA of each pass, CTAs per head of each pass
     int ch1, ch2, nch1, nch2;
     float qk_scale_log2;  // restore pass: the scale * log2 e the restored queries are taken at
+    // one-launch eviction: clusters per head (each selects on its own, the copy is split over
+    // all of them) and whether to skip the sampled cut (exact radix passes only)
+    int ev_reps;
+    int ev_exact;
+    // evicted sets computed ahead by plan_kernel ([2][L][B][KVH][r + 1]: count, then the ordinals
+    // ascending) and which half this launch reads; null: the kernel selects itself
+    const int32_t* ev_plan;
+    int ev_plan_parity;
 };
 
 constexpr int kScoreTile = 64;      // key rows per scoring tile
@@ -132,6 +145,21 @@ cudaError_t launch_select(const EvictParams& p, cudaStream_t s);
 size_t select_smem(int N, int r, bool scored);  // dynamic shared memory of one select CTA
 constexpr size_t kSelectSmemLimit = 220 * 1024;
 cudaError_t launch_compact(const EvictParams& p, cudaStream_t s);
+// Selection and order-preserving compaction in one launch, p.ev_reps clusters of `cluster` CTAs
+// per triggered head (random, shared, recency and block policies; ordered compaction).  Each
+// CTA holds the keys of at most kEvMaxLocal candidates: cluster >= ceil((K + r) / kEvMaxLocal).
+constexpr int kEvMaxLocal = 2112;
+constexpr int kEvMaxCluster = 16;
+constexpr int kEvMaxEvicted = 512;  // r bound of the one-launch path (the evicted list lives in shared memory)
+constexpr int kEvRows = 16;  // rows per copy buffer (8 KB of K and V)
+constexpr int kEvBufs = 3;   // copy buffers per warp: 192 KB per CTA, one CTA per SM
+cudaError_t launch_evict(const EvictParams& p, int cluster, cudaStream_t s);
+// The evicted sets of the triggered sequences' heads in every layer, from the counters alone
+// (the random draw reads no cache data), into half p.ev_plan_parity of lay.evplan; one CTA per
+// (layer, sequence, KV head), little shared memory, so that it runs beside the attention kernel.
+cudaError_t launch_plan(const EvictParams& p, cudaStream_t s);
+// One-time attributes; active[cl] (cl = 0..kEvMaxCluster) = clusters of cl CTAs the device runs at once.
+cudaError_t evict_prepare(int* active);
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s);
 cudaError_t launch_restore(const CopyRowsParams& p, cudaStream_t s);

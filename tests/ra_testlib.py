@@ -207,6 +207,29 @@ class Runner:
                     np.testing.assert_array_equal(kk, self.krows(l, b, h, allpos), err_msg=f"K rows l{l} b{b} h{h}")
                     np.testing.assert_array_equal(vv, self.vrows(l, b, h, allpos), err_msg=f"V rows l{l} b{b} h{h}")
 
+    def restore_full(self, g, layers=(0,)):
+        """Every sequence of the given layers: g tokens generated, the newest K + 2r - 1 of them cached
+        (one append short of capacity), prompt as prefilled; the oracle mirror gets the same state.
+        With g + 1 a multiple of r, the next step fires a round over K + r candidates."""
+        c = self.K + 2 * self.r - 1
+        for l in layers:
+            pos = np.zeros((self.B, self.KVH, c), np.int32)
+            kk = np.zeros((self.B, self.KVH, c, self.D), np.uint16)
+            vv = np.zeros_like(kk)
+            for b in range(self.B):
+                p = self.lp[b] + np.arange(g - c, g)
+                for h in range(self.KVH):
+                    pos[b, h] = p
+                    kk[b, h] = self.krows(l, b, h, p)
+                    vv[b, h] = self.vrows(l, b, h, p)
+                    self.orc.gen[(b, l, h)] = p.astype(np.int32)
+                self.orc.g[b, l] = g
+            tp = self.torch.from_numpy(pos).cuda()
+            tk, tv = self.up(kk), self.up(vv)
+            self.ra.ra_restore(self.ctx, l, [g] * self.B, [c] * self.B, tp.data_ptr(), tk.data_ptr(), tv.data_ptr(), c)
+            self.torch.cuda.synchronize()
+        self.step_idx = g
+
     def close(self):
         self.ra.ra_check_device(self.ctx)
         self.cache.close()

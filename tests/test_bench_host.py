@@ -159,3 +159,19 @@ def test_eviction_roofline_prices_the_copy_kernel_and_the_round():
     assert r2["holefill_select"]["us_per_round"] == pytest.approx(5.0)
     # no eviction in the evented pass: nothing to report
     assert bench.eviction_roofline({"attn": kern["attn"]}, 0, peaks, "measured") is None
+
+
+def test_eviction_window_is_the_step_time_beyond_the_attention_bytes():
+    # eviction-free steps: 2 x (1.0 ms for 6e9 attention bytes) -> 6e9 B/ms
+    clean = [(1.0, 64, 6e9), (1.0, 64, 6e9)]
+    # evicting steps: attention bytes 5.94e9 (0.99 ms at that rate) plus eviction time
+    evicting = [(1.99 + 0.0, 5.94e9, 64, 64 * 68e6), (1.5, 5.94e9, 64, 64 * 68e6)]
+    w = bench.eviction_window(clean, evicting)
+    extra = (1.99 - 0.99) + (1.5 - 0.99)
+    assert w["rounds"] == 128 and w["steps"] == 2
+    assert w["us_per_round"] == pytest.approx(1000.0 * extra / 128)
+    assert w["bytes_per_round"] == pytest.approx(68e6)
+    assert w["GBps"] == pytest.approx(128 * 68e6 / (extra * 1e-3) / 1e9)
+    assert bench.eviction_window([], evicting) is None and bench.eviction_window(clean, []) is None
+    r = bench.eviction_roofline({"evict": _kern(12.0, 68e6, 10)}, 10, {"hbm_gbs": 6000.0}, "measured", None, None, w)
+    assert r["windowed"]["frac"] == pytest.approx(w["GBps"] / 6000.0)

@@ -12,30 +12,6 @@ from ra_testlib import Runner, check_attention
 pytestmark = [pytest.mark.gpu, pytest.mark.skipif(not cuda_available(), reason="needs a CUDA GPU")]
 
 
-def _restore_full(run, g):
-    """Every sequence: g tokens generated, the newest K + 2r - 1 of them cached (one append short of
-    capacity), prompt as prefilled; the oracle mirror gets the same state."""
-    import paper_2609_03430_gb300 as ra
-
-    c = run.K + 2 * run.r - 1
-    pos = np.zeros((run.B, run.KVH, c), np.int32)
-    kk = np.zeros((run.B, run.KVH, c, run.D), np.uint16)
-    vv = np.zeros_like(kk)
-    for b in range(run.B):
-        p = run.lp[b] + np.arange(g - c, g)
-        for h in range(run.KVH):
-            pos[b, h] = p
-            kk[b, h] = run.krows(0, b, h, p)
-            vv[b, h] = run.vrows(0, b, h, p)
-            run.orc.gen[(b, 0, h)] = p.astype(np.int32)
-        run.orc.g[b, 0] = g
-    tp = run.torch.from_numpy(pos).cuda()
-    tk, tv = run.up(kk), run.up(vv)
-    ra.ra_restore(run.ctx, 0, [g] * run.B, [c] * run.B, tp.data_ptr(), tk.data_ptr(), tv.data_ptr(), c)
-    run.torch.cuda.synchronize()
-    run.step_idx = g
-
-
 @pytest.mark.parametrize("fused,compaction", [(False, 0), (True, 0), (True, 1)],
                          ids=["separate-ordered", "fused-ordered", "fused-holefill"])
 def test_random_eviction_at_max_candidates(fused, compaction):
@@ -43,7 +19,7 @@ def test_random_eviction_at_max_candidates(fused, compaction):
     run = Runner(L=1, H=4, KVH=2, prompt_lens=[64, 5], K=K, r=r, eseed=11, dseed=12, fused=fused,
                  compaction=compaction)
     g = 640 * r - 1  # the next step's token makes g a multiple of r with K + r candidates: it fires
-    _restore_full(run, g)
+    run.restore_full(g)
     fired = run.step(check_attn_layers=(0,))
     assert fired[0] == run.B
     run.check_state()
