@@ -37,9 +37,12 @@
  * Random draw (the paper fixes none; this is the library's mapping): the score
  * of candidate j (its ordinal in slot order among the c - r candidates) is
  * word 0 of Philox4x32-10 (Salmon et al., SC'11) with
- *     counter = (j, g, layer, seq * kv_heads + kv_head),  key = (seed lo, seed hi),
- * where g is the number of generated tokens appended when the eviction fires.
- * The K smallest (score, j) survive.
+ *     counter = (j, g, layer, (a << 16) | (seq * kv_heads + kv_head)),  key = (seed lo, seed hi),
+ * where g is the number of generated tokens appended when the eviction fires
+ * and a the number of requests admitted into slot seq before the current one
+ * (0 for the batch given at creation; see ra_admit), so that every request
+ * draws its own numbers (a per-request stream, as the paper's per-request
+ * seed).  The K smallest (score, j) survive.
  */
 #ifndef RA_H_
 #define RA_H_
@@ -248,6 +251,30 @@ int ra_set_attention_shape(ra_ctx* ctx, int shape);
 #define RA_EVICT_TWO_KERNELS 1
 #define RA_EVICT_EXACT 256
 int ra_set_eviction_kernel(ra_ctx* ctx, int mode);
+
+/*
+ * Prompt pool; set it BEFORE ra_device_bytes / ra_bind (default: exactly the prompts given at
+ * creation).  Prompt rows live in pages of 192 positions (all KV heads of one sequence, in every
+ * layer), listed per sequence in a page table that the kernels read tile by tile, so that a
+ * finished sequence's slot can take a new request with a prompt of another length (ra_admit).
+ * max_prompt_len: the longest prompt a slot will take; pool_positions: the prompt positions the
+ * pool holds over all slots (per layer and KV head), rounded up to pages and at least what the
+ * creation prompts use.  RA_ERR_STATE once bound.
+ */
+int ra_set_prompt_pool(ra_ctx* ctx, int max_prompt_len, long long pool_positions);
+
+/*
+ * Admit a new request into slot `seq`, which must be finished (ra_set_active(seq, 0)): the slot's
+ * prompt pages return to the pool and ceil(prompt_len / 192) pages are taken, the prompt rows
+ * k, v (device [layers][kv_heads][row_stride][head_dim], rows [0, prompt_len) used; post-RoPE
+ * keys, Appendix F) are written on `stream`, the slot's counters restart at g = c = 0 in every
+ * layer, and the slot is active again.  The generated regions are reused as they are; positions
+ * restart at 0 for the new request.  Its random stream is the slot's next one (admission count
+ * in the key; see the mapping above).  Errors leave the state unchanged: RA_ERR_STATE if the slot
+ * is active, RA_ERR_CAPACITY if prompt_len exceeds the pool's longest prompt or its free pages.
+ * (The paper's serving runs use vLLM's paged cache; this is that capability for the prompt.)
+ */
+int ra_admit(ra_ctx* ctx, int seq, int prompt_len, const uint16_t* k, const uint16_t* v, int row_stride, void* stream);
 
 /* Mark sequence `seq` active (1) or finished (0); finished ones are skipped by every call. */
 int ra_set_active(ra_ctx* ctx, int seq, int active);

@@ -71,22 +71,26 @@ def _load():
         lib.ora_evict_head.restype = ctypes.c_int
         lib.ora_attend.argtypes = [u16p, u16p, u16p, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                    ctypes.c_double, f64p]
+        lib.ora_head_stream.argtypes = [ctypes.c_uint32, ctypes.c_uint32]
+        lib.ora_head_stream.restype = ctypes.c_uint32
         lib.ora_policy_key.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_uint32,
                                        ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32,
-                                       ctypes.c_uint32, ctypes.c_int32, ctypes.c_int32]
+                                       ctypes.c_uint32, ctypes.c_int32, ctypes.c_int32, ctypes.c_uint32]
         lib.ora_policy_key.restype = ctypes.c_uint32
         lib.ora_evict_head_policy.argtypes = [i32p, ctypes.POINTER(ctypes.c_int), ctypes.c_int, ctypes.c_int,
                                               ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int,
-                                              ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, i32p]
+                                              ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                              ctypes.c_uint32, i32p]
         lib.ora_evict_head_policy.restype = ctypes.c_int
         lib.ora_attend.restype = None
         lib.ora_position_key.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_uint32,
                                          ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int32,
-                                         ctypes.c_int32]
+                                         ctypes.c_int32, ctypes.c_uint32]
         lib.ora_position_key.restype = ctypes.c_uint32
         lib.ora_evict_head_holefill.argtypes = [i32p, ctypes.POINTER(ctypes.c_int), ctypes.c_int, ctypes.c_int,
                                                 ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int,
-                                                ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, i32p]
+                                                ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_uint32, i32p]
         lib.ora_evict_head_holefill.restype = ctypes.c_int
         lib.ora_window_scores.argtypes = [u16p, i32p, ctypes.c_int, ctypes.c_int, u16p, i32p, ctypes.c_int,
                                           ctypes.c_int, ctypes.c_double, f64p]
@@ -159,7 +163,12 @@ POLICY_RANDOM, POLICY_SHARED, POLICY_RECENCY, POLICY_BLOCK, POLICY_SNAPKV = 0, 1
 SNAPKV_POOL_RADIUS = 3  # max-pool width 7: the paper gives no width, this is the library's stated choice
 
 
-def evict_head_policy(gen, g, K, r, seed, layer, seq, kv_heads, h, policy, block=1):
+def head_stream(admissions: int, head: int) -> int:
+    """Key stream of a head: the slot's earlier admissions above the head id (see ra_oracle.c)."""
+    return int(_load().ora_head_stream(admissions, head))
+
+
+def evict_head_policy(gen, g, K, r, seed, layer, seq, kv_heads, h, policy, block=1, admissions=0):
     """One eviction round under a policy variant (random / shared / recency / block)."""
     buf = np.ascontiguousarray(gen, dtype=np.int32).copy()
     c = ctypes.c_int(int(buf.size))
@@ -167,7 +176,7 @@ def evict_head_policy(gen, g, K, r, seed, layer, seq, kv_heads, h, policy, block
     if buf.size == 0:
         return buf, ev[:0]
     m = _load().ora_evict_head_policy(_ptr(buf, ctypes.c_int32), ctypes.byref(c), g, K, r, seed, layer, seq,
-                                      kv_heads, h, policy, block, _ptr(ev, ctypes.c_int32))
+                                      kv_heads, h, policy, block, admissions, _ptr(ev, ctypes.c_int32))
     if m < 0:
         raise RuntimeError("ora_evict_head_policy failed")
     return buf[: c.value].copy(), ev[:m].copy()
@@ -190,12 +199,12 @@ def attend(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float = 0.0) -> n
 COMPACT_ORDERED, COMPACT_HOLEFILL = 0, 1
 
 
-def position_key(policy, seed, layer, seq, kv_heads, h, step, position, block=1) -> int:
+def position_key(policy, seed, layer, seq, kv_heads, h, step, position, block=1, admissions=0) -> int:
     """Policy score of the candidate at `position` when slots carry no order."""
-    return int(_load().ora_position_key(policy, seed, layer, seq, kv_heads, h, step, position, block))
+    return int(_load().ora_position_key(policy, seed, layer, seq, kv_heads, h, step, position, block, admissions))
 
 
-def evict_head_holefill(gen, g, K, r, seed, layer, seq, kv_heads, h, policy=POLICY_RANDOM, block=1):
+def evict_head_holefill(gen, g, K, r, seed, layer, seq, kv_heads, h, policy=POLICY_RANDOM, block=1, admissions=0):
     """One eviction round with hole-filling compaction; returns (new_gen, evicted_ordinals)."""
     buf = np.ascontiguousarray(gen, dtype=np.int32).copy()
     c = ctypes.c_int(int(buf.size))
@@ -203,7 +212,7 @@ def evict_head_holefill(gen, g, K, r, seed, layer, seq, kv_heads, h, policy=POLI
     if buf.size == 0:
         return buf, ev[:0]
     m = _load().ora_evict_head_holefill(_ptr(buf, ctypes.c_int32), ctypes.byref(c), g, K, r, seed, layer, seq,
-                                        kv_heads, h, policy, block, _ptr(ev, ctypes.c_int32))
+                                        kv_heads, h, policy, block, admissions, _ptr(ev, ctypes.c_int32))
     if m < 0:
         raise RuntimeError("ora_evict_head_holefill failed")
     return buf[: c.value].copy(), ev[:m].copy()
@@ -295,12 +304,25 @@ class OracleCache:
             heads = [(b, l, h) for b in range(self.B) for l in range(layers) for h in range(kv_heads)]
         self.gen = {tuple(u): np.zeros(0, dtype=np.int32) for u in heads}
         self.n_evictions = np.zeros((self.B, layers), dtype=np.int64)
+        self.admissions = [0] * self.B  # requests each slot took after the first batch
 
     def restore(self, seq, layer, g, positions_by_head):
         self.g[seq, layer] = g
         for h in range(self.KVH):
             if (seq, layer, h) in self.gen:
                 self.gen[(seq, layer, h)] = np.asarray(positions_by_head[h], dtype=np.int32).copy()
+
+    def admit(self, seq, prompt_len):
+        """A new request in slot `seq` (the previous one finished): its own prompt of prompt_len
+        positions, nothing generated or cached in any layer, the slot's next key stream."""
+        self.prompt_lens[seq] = int(prompt_len)
+        self.admissions[seq] += 1
+        for l in range(self.L):
+            self.g[seq, l] = 0
+            self.n_evictions[seq, l] = 0
+            for h in range(self.KVH):
+                if (seq, l, h) in self.gen:
+                    self.gen[(seq, l, h)] = np.zeros(0, dtype=np.int32)
 
     def c(self, seq, layer):
         """Cached generated count (identical for every head of a (seq, layer))."""
@@ -333,16 +355,17 @@ class OracleCache:
             cur = self.gen[key]
             if not should_evict(g, int(cur.size), self.K, self.r):
                 continue
+            a = self.admissions[seq]
             if self.compaction == COMPACT_HOLEFILL:
                 new, ev = evict_head_holefill(cur, g, self.K, self.r, self.seed, layer, seq, self.KVH, h,
-                                              self.policy, self.block)
+                                              self.policy, self.block, a)
             elif self.policy == POLICY_RANDOM:
-                new, ev = evict_head(cur, g, self.K, self.r, self.seed, layer, seq * self.KVH + h)
+                new, ev = evict_head(cur, g, self.K, self.r, self.seed, layer, head_stream(a, seq * self.KVH + h))
             elif self.policy == POLICY_SNAPKV:
                 new, ev = evict_head_scored(cur, g, self.K, self.r, scorer(seq, layer, h, cur))
             else:
                 new, ev = evict_head_policy(cur, g, self.K, self.r, self.seed, layer, seq, self.KVH, h,
-                                            self.policy, self.block)
+                                            self.policy, self.block, a)
             self.gen[key] = new
             fired[h] = ev
         if fired:

@@ -83,8 +83,13 @@ void ora_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t ou
  *     counter = (j, step, layer, head_id),  key = (seed_lo, seed_hi),
  *     score   = word 0 of Philox4x32-10,
  * with j the candidate's ordinal in slot order, step = number of generated
- * tokens appended when the eviction fires, and head_id = seq * kv_heads + h.
+ * tokens appended when the eviction fires, and head_id = seq * kv_heads + h for
+ * the batch a context starts with.  A request admitted into a slot later draws
+ * its own stream: head_id = (a << 16) | (seq * kv_heads + h), a = the requests
+ * the slot took before (the paper's per-request seed, Appendix H; ora_head_stream).
  */
+uint32_t ora_head_stream(uint32_t admissions, uint32_t head) { return (admissions << 16) | head; }
+
 uint32_t ora_random_key(uint64_t seed, uint32_t layer, uint32_t head_id, uint32_t step, uint32_t j)
 {
     uint32_t ctr[4] = {j, step, layer, head_id};
@@ -108,17 +113,18 @@ uint32_t ora_random_key(uint64_t seed, uint32_t layer, uint32_t head_id, uint32_
  * Ties of equal score go to the lower ordinal, as everywhere.
  */
 uint32_t ora_policy_key(int policy, uint64_t seed, uint32_t layer, uint32_t seq, uint32_t kv_heads, uint32_t h,
-                        uint32_t step, uint32_t j, uint32_t n_cand, int32_t position, int32_t block)
+                        uint32_t step, uint32_t j, uint32_t n_cand, int32_t position, int32_t block, uint32_t admissions)
 {
     switch (policy) {
         case 1:
-            return ora_random_key(seed, layer, seq * kv_heads, step, j);
+            return ora_random_key(seed, layer, ora_head_stream(admissions, seq * kv_heads), step, j);
         case 2:
             return n_cand - 1u - j;
         case 3:
-            return ora_random_key(seed, layer, seq * kv_heads + h, step, (uint32_t)(position / block));
+            return ora_random_key(seed, layer, ora_head_stream(admissions, seq * kv_heads + h), step,
+                                  (uint32_t)(position / block));
         default:
-            return ora_random_key(seed, layer, seq * kv_heads + h, step, j);
+            return ora_random_key(seed, layer, ora_head_stream(admissions, seq * kv_heads + h), step, j);
     }
 }
 
@@ -232,7 +238,7 @@ int ora_evict_head(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int
  * candidates and compaction as ora_evict_head.
  */
 int ora_evict_head_policy(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int layer, int seq,
-                          int kv_heads, int h, int policy, int block, int32_t* evicted_out)
+                          int kv_heads, int h, int policy, int block, uint32_t admissions, int32_t* evicted_out)
 {
     int cc = *c;
     if (!ora_should_evict(g, cc, K, r)) return 0;
@@ -247,7 +253,7 @@ int ora_evict_head_policy(int32_t* gen, int* c, int g, int K, int r, uint64_t se
     }
     for (int j = 0; j < n; ++j)
         keys[j] = ora_policy_key(policy, seed, (uint32_t)layer, (uint32_t)seq, (uint32_t)kv_heads, (uint32_t)h,
-                                 (uint32_t)g, (uint32_t)j, (uint32_t)n, gen[j], block);
+                                 (uint32_t)g, (uint32_t)j, (uint32_t)n, gen[j], block, admissions);
     if (ora_select_keep(keys, n, K, keep) != 0) {
         free(keys); free(keep); free(next);
         return -1;
@@ -461,17 +467,19 @@ int ora_evict_head_scored(int32_t* gen, int* c, int g, int K, int r, const doubl
  *   3 block   -- as ordered: counter word 0 = position / block.
  */
 uint32_t ora_position_key(int policy, uint64_t seed, uint32_t layer, uint32_t seq, uint32_t kv_heads, uint32_t h,
-                          uint32_t step, int32_t position, int32_t block)
+                          uint32_t step, int32_t position, int32_t block, uint32_t admissions)
 {
     switch (policy) {
         case 1:
-            return ora_random_key(seed, layer, seq * kv_heads, step, (uint32_t)position);
+            return ora_random_key(seed, layer, ora_head_stream(admissions, seq * kv_heads), step, (uint32_t)position);
         case 2:
             return 0xFFFFFFFFu - (uint32_t)position;
         case 3:
-            return ora_random_key(seed, layer, seq * kv_heads + h, step, (uint32_t)(position / block));
+            return ora_random_key(seed, layer, ora_head_stream(admissions, seq * kv_heads + h), step,
+                                  (uint32_t)(position / block));
         default:
-            return ora_random_key(seed, layer, seq * kv_heads + h, step, (uint32_t)position);
+            return ora_random_key(seed, layer, ora_head_stream(admissions, seq * kv_heads + h), step,
+                                  (uint32_t)position);
     }
 }
 
@@ -486,7 +494,7 @@ uint32_t ora_position_key(int policy, uint64_t seed, uint32_t layer, uint32_t se
  * evicted ordinals, -1 on error.
  */
 int ora_evict_head_holefill(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int layer, int seq,
-                            int kv_heads, int h, int policy, int block, int32_t* evicted_out)
+                            int kv_heads, int h, int policy, int block, uint32_t admissions, int32_t* evicted_out)
 {
     const int cc = *c;
     if (!ora_should_evict(g, cc, K, r)) return 0;
@@ -502,7 +510,7 @@ int ora_evict_head_holefill(int32_t* gen, int* c, int g, int K, int r, uint64_t 
     }
     for (int j = 0; j < n; ++j)
         keys[j] = ora_position_key(policy, seed, (uint32_t)layer, (uint32_t)seq, (uint32_t)kv_heads, (uint32_t)h,
-                                   (uint32_t)g, gen[j], block);
+                                   (uint32_t)g, gen[j], block, admissions);
     if (ora_select_keep(keys, n, K, keep) != 0) {
         free(keys); free(keep); free(ev);
         return -1;

@@ -49,6 +49,8 @@ SIGNATURES = {
     "ra_set_eviction_kernel": (_i, [_vp, _i]),
     "ra_restore_queries": (_i, [_vp, _i, _vp, ctypes.c_float, _vp]),
     "ra_get_scores": (_i, [_vp, _i, _i, _i, ctypes.POINTER(ctypes.c_float), _i, _ip, _vp]),
+    "ra_set_prompt_pool": (_i, [_vp, _i, ctypes.c_longlong]),
+    "ra_admit": (_i, [_vp, _i, _i, _vp, _vp, _i, _vp]),
     "ra_set_active": (_i, [_vp, _i, _i]),
     "ra_append_kv": (_i, [_vp, _i, _vp, _vp, _vp]),
     "ra_evict": (_i, [_vp, _i, _ip, _vp]),
@@ -182,6 +184,14 @@ def ra_get_scores(ctx, layer, seq, kv_head, capacity, stream=None):
     return buf[: n.value].copy()
 
 
+def ra_set_prompt_pool(ctx, max_prompt_len, pool_positions):
+    return _check(lib().ra_set_prompt_pool(ctx, int(max_prompt_len), int(pool_positions)), ctx)
+
+
+def ra_admit(ctx, seq, prompt_len, k_ptr, v_ptr, row_stride, stream=None):
+    return _check(lib().ra_admit(ctx, int(seq), int(prompt_len), k_ptr, v_ptr, int(row_stride), _stream_ptr(stream)), ctx)
+
+
 def ra_set_active(ctx, seq, active):
     return _check(lib().ra_set_active(ctx, seq, int(bool(active))), ctx)
 
@@ -275,7 +285,7 @@ class RandomAttentionCache:
     """Owns a context and its torch-allocated device arena (uint8 CUDA tensor)."""
 
     def __init__(self, layers, q_heads, kv_heads, head_dim, prompt_lens, K, r=64, seed=0, device=None, stream=None,
-                 policy=RA_POLICY_RANDOM, block=1, compaction=RA_COMPACT_ORDERED):
+                 policy=RA_POLICY_RANDOM, block=1, compaction=RA_COMPACT_ORDERED, prompt_pool=None):
         import torch
 
         if isinstance(prompt_lens, int):
@@ -288,6 +298,8 @@ class RandomAttentionCache:
             ra_set_compaction(self.ctx, compaction)
         if policy != RA_POLICY_RANDOM:  # before sizing: the scored policy adds buffers to the arena
             ra_set_policy(self.ctx, policy, block)
+        if prompt_pool is not None:  # (max_prompt_len, pool_positions), before sizing
+            ra_set_prompt_pool(self.ctx, *prompt_pool)
         self.nbytes = ra_device_bytes(self.ctx)
         dev = torch.device("cuda") if device is None else torch.device(device)
         self.arena = torch.empty(self.nbytes + 256, dtype=torch.uint8, device=dev)

@@ -45,14 +45,20 @@ struct ra_ctx {
     int L, H, KVH, G, D, B, K, r, Cmax;
     uint64_t seed;
     std::vector<int32_t> lp;       // prompt lengths
-    std::vector<int32_t> poff;     // KVH * prefix sum of prompt lengths
+    // prompt pages (kPromptPage positions x KVH heads each, every layer alike): the pool, the
+    // longest prompt a slot takes, each sequence's pages and the free ones; admissions per slot
+    int max_prompt = 0, max_pages = 1;
+    long long pool_pages = 0;
+    std::vector<int32_t> pages;      // [B][max_pages]
+    std::vector<int32_t> free_pages;
+    std::vector<int32_t> admits;     // [B]
     long long prompt_rows_per_layer = 0;
     long long total_rows = 0;
     long long gen_rows = 0;
     int regions = 0;
     size_t partial_records = 0;  // split-K partial records the arena holds
     // arena layout (byte offsets)
-    size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_poff, off_plan, off_partial, off_arrive,
+    size_t off_k, off_v, off_pos, off_region, off_spare, off_lp, off_pages, off_plan, off_partial, off_arrive,
         off_err, off_evplan, bytes;
     // scored policy: query window, scores and pass-1 statistics after the base arena
     bool scoring = false;
@@ -291,6 +297,53 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     return RA_OK;
 }
 
+void layout_scoring(ra_ctx* ctx);
+
+// Arena layout from the shape and the prompt pool (pages, the longest prompt); then the scored
+// policy's buffers, if chosen.
+int layout_base(ra_ctx* ctx)
+{
+    const int layers = ctx->L, batch = ctx->B, kv_heads = ctx->KVH, r = ctx->r;
+    ctx->max_pages = std::max(1, (ctx->max_prompt + kPromptPage - 1) / kPromptPage);
+    ctx->prompt_rows_per_layer = ctx->pool_pages * kv_heads * kPromptPage;
+    ctx->regions = (layers + 1) * batch * kv_heads;
+    ctx->gen_rows = (long long)ctx->regions * ctx->Cmax;
+    ctx->total_rows = ctx->prompt_rows_per_layer * layers + ctx->gen_rows;
+    // every slot position and every row index must fit the int32 coordinates the kernels use
+    if (ctx->total_rows >= (1LL << 31) || ctx->prompt_rows_per_layer >= (1LL << 31))
+        return fail(nullptr, RA_ERR_UNSUPPORTED, "cache too large for 32-bit row coordinates");
+    size_t o = 0;
+    auto take = [&](size_t n) {
+        size_t at = o;
+        o = align_up(o + n, kAlign);
+        return at;
+    };
+    const size_t pool_bytes = (size_t)ctx->total_rows * kRowBytes;
+    ctx->off_k = take(pool_bytes);
+    ctx->off_v = take(pool_bytes);
+    ctx->off_pos = take((size_t)ctx->regions * ctx->Cmax * 4);
+    ctx->off_region = take((size_t)layers * batch * kv_heads * 4);
+    ctx->off_spare = take((size_t)batch * kv_heads * 4);
+    ctx->off_lp = take((size_t)batch * 4);
+    ctx->off_pages = take((size_t)batch * ctx->max_pages * 4);
+    ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
+    // chunks of the attention split: one per warp
+    const size_t max_chunks =
+        (size_t)kMaxSMs * std::max(attn_warps_per_cta(kAttnWide, ctx->G), attn_warps_per_cta(kAttnNarrow, ctx->G)) + 1;
+    ctx->partial_records = max_chunks + (size_t)batch * kv_heads;
+    ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
+    ctx->off_arrive = take((size_t)batch * kv_heads * 4);
+    ctx->off_err = take(256);
+    ctx->off_evplan = take((size_t)2 * layers * batch * kv_heads * (r + 1) * 4);
+    ctx->base_bytes = o;
+    // pass-1 chunks per head: at most one per tile of the longest head, capped (the host
+    // then takes chunks of several tiles)
+    const int tiles1 = (ctx->max_prompt + kScoreTile - 1) / kScoreTile + (ctx->Cmax + kScoreTile - 1) / kScoreTile;
+    ctx->stats_chunks = std::min(tiles1, 64);
+    layout_scoring(ctx);
+    return RA_OK;
+}
+
 // Arena size with (or without) the scored policy's buffers after the base layout.
 void layout_scoring(ra_ctx* ctx)
 {
@@ -368,6 +421,7 @@ int run_eviction(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool
     for (int i = 0; i < p.n_trig; ++i) {
         p.trig_src[i] = ctx->rbase[(size_t)p.layer * ctx->B + p.trig[i]];
         p.trig_dst[i] = ctx->sbase[p.trig[i]];
+        p.trig_admit[i] = (uint16_t)ctx->admits[p.trig[i]];
     }
     int rc = run_eviction_launches(ctx, p, moved, s, compact_in_attention, score_early);
     if (rc == RA_OK && !p.holefill)  // every ordered compaction (any kernel) swaps region and spare
@@ -494,56 +548,19 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->Cmax = K + 2 * r;
     ctx->seed = seed;
     ctx->lp.assign(prompt_lens, prompt_lens + batch);
-    ctx->poff.resize(batch);
-    long long acc = 0;
     for (int b = 0; b < batch; ++b) {
         if (prompt_lens[b] < 0) {
             delete ctx;
             return fail(nullptr, RA_ERR_INVALID_ARG, "prompt_lens[%d] < 0", b);
         }
-        ctx->poff[b] = (int32_t)(acc * kv_heads);
-        acc += prompt_lens[b];
+        ctx->max_prompt = std::max(ctx->max_prompt, (int)prompt_lens[b]);
+        ctx->pool_pages += (prompt_lens[b] + kPromptPage - 1) / kPromptPage;
     }
-    ctx->prompt_rows_per_layer = acc * kv_heads;
-    ctx->regions = (layers + 1) * batch * kv_heads;
-    ctx->gen_rows = (long long)ctx->regions * ctx->Cmax;
-    ctx->total_rows = ctx->prompt_rows_per_layer * layers + ctx->gen_rows;
-    // every slot position and every row index must fit the int32 coordinates the kernels use
-    if (ctx->total_rows >= (1LL << 31) || ctx->prompt_rows_per_layer >= (1LL << 31)) {
+    int rc = layout_base(ctx);
+    if (rc != RA_OK) {
         delete ctx;
-        return fail(nullptr, RA_ERR_UNSUPPORTED, "cache too large for 32-bit row coordinates");
+        return rc;
     }
-    size_t o = 0;
-    auto take = [&](size_t n) {
-        size_t at = o;
-        o = align_up(o + n, kAlign);
-        return at;
-    };
-    const size_t pool_bytes = (size_t)ctx->total_rows * kRowBytes;
-    ctx->off_k = take(pool_bytes);
-    ctx->off_v = take(pool_bytes);
-    ctx->off_pos = take((size_t)ctx->regions * ctx->Cmax * 4);
-    ctx->off_region = take((size_t)layers * batch * kv_heads * 4);
-    ctx->off_spare = take((size_t)batch * kv_heads * 4);
-    ctx->off_lp = take((size_t)batch * 4);
-    ctx->off_poff = take((size_t)batch * 4);
-    ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
-    // chunks of the attention split: one per warp
-    const size_t max_chunks =
-        (size_t)kMaxSMs * std::max(attn_warps_per_cta(kAttnWide, ctx->G), attn_warps_per_cta(kAttnNarrow, ctx->G)) + 1;
-    ctx->partial_records = max_chunks + (size_t)batch * kv_heads;
-    ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
-    ctx->off_arrive = take((size_t)batch * kv_heads * 4);
-    ctx->off_err = take(256);
-    ctx->off_evplan = take((size_t)2 * layers * batch * kv_heads * (r + 1) * 4);
-    ctx->base_bytes = o;
-    int maxlp = 0;
-    for (int b = 0; b < batch; ++b) maxlp = std::max(maxlp, (int)prompt_lens[b]);
-    // pass-1 chunks per head: at most one per tile of the longest head, capped (the host
-    // then takes chunks of several tiles)
-    const int tiles1 = (maxlp + kScoreTile - 1) / kScoreTile + (ctx->Cmax + kScoreTile - 1) / kScoreTile;
-    ctx->stats_chunks = std::min(tiles1, 64);
-    layout_scoring(ctx);
     ctx->g.assign((size_t)layers * batch, 0);
     ctx->c.assign((size_t)layers * batch, 0);
     ctx->nev.assign((size_t)layers * batch, 0);
@@ -590,7 +607,8 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.region = (int32_t*)(a + ctx->off_region);
     Ly.spare = (int32_t*)(a + ctx->off_spare);
     Ly.seq_lp = (int32_t*)(a + ctx->off_lp);
-    Ly.seq_poff = (int32_t*)(a + ctx->off_poff);
+    Ly.pages = (int32_t*)(a + ctx->off_pages);
+    Ly.max_pages = ctx->max_pages;
     Ly.plan = (int32_t*)(a + ctx->off_plan);
     Ly.partial = (float*)(a + ctx->off_partial);
     Ly.arrive = (int32_t*)(a + ctx->off_arrive);
@@ -613,6 +631,18 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     Ly.r = ctx->r;
     Ly.seed = ctx->seed;
 
+    // Prompt pages in sequence order, the rest of the pool free; no admissions yet.
+    ctx->pages.assign((size_t)ctx->B * ctx->max_pages, 0);
+    ctx->free_pages.clear();
+    {
+        long long next = 0;
+        for (int b = 0; b < ctx->B; ++b)
+            for (int j = 0; j < (ctx->lp[b] + kPromptPage - 1) / kPromptPage; ++j)
+                ctx->pages[(size_t)b * ctx->max_pages + j] = (int32_t)next++;
+        if (next > ctx->pool_pages) return fail(ctx, RA_ERR_CAPACITY, "prompts need more pages than the pool holds");
+        for (long long pg = ctx->pool_pages - 1; pg >= next; --pg) ctx->free_pages.push_back((int32_t)pg);
+    }
+    ctx->admits.assign(ctx->B, 0);
     // Tables: regions of (layer, seq, head) in order, one spare per (seq, head).
     const int BH = ctx->B * ctx->KVH;
     std::vector<int32_t> region((size_t)ctx->L * BH), spare(BH);
@@ -623,7 +653,8 @@ int ra_bind(ra_ctx* ctx, void* device_arena, size_t bytes, void* stream)
     if ((e = cudaMemcpyAsync(Ly.region, region.data(), region.size() * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.spare, spare.data(), spare.size() * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.seq_lp, ctx->lp.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(Ly.seq_poff, ctx->poff.data(), ctx->B * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(Ly.pages, ctx->pages.data(), ctx->pages.size() * 4, cudaMemcpyHostToDevice, s)) !=
+            cudaSuccess ||
         (e = cudaMemcpyAsync(Ly.err, &zero, 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemsetAsync(Ly.arrive, 0, (size_t)BH * 4, s)) != cudaSuccess)
         return cuda_fail(ctx, e, "table initialisation");
@@ -690,6 +721,7 @@ int ra_prefill(ra_ctx* ctx, int layer, const uint16_t* k, const uint16_t* v, int
     p.k = k;
     p.v = v;
     p.row_stride = row_stride;
+    p.only_seq = -1;
     for (int b = 0; b < ctx->B; ++b) p.n_rows[b] = ctx->lp[b];
     cudaError_t e = launch_prefill(p, (cudaStream_t)stream);
     return e == cudaSuccess ? RA_OK : cuda_fail(ctx, e, "prefill launch");
@@ -718,6 +750,7 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
     p.v = v;
     p.pos = pos;
     p.row_stride = row_stride;
+    p.only_seq = -1;
     for (int b = 0; b < ctx->B; ++b) p.n_rows[b] = c_host[b];
     cudaError_t e;
     if (maxc > 0 && (e = launch_restore(p, s)) != cudaSuccess) return cuda_fail(ctx, e, "restore launch");
@@ -770,6 +803,88 @@ int ra_set_attention_shape(ra_ctx* ctx, int shape)
     if (shape < RA_ATTN_SHAPE_AUTO || shape > RA_ATTN_SHAPE_NARROW)
         return fail(ctx, RA_ERR_INVALID_ARG, "unknown attention shape %d", shape);
     ctx->attn_shape = shape;
+    return RA_OK;
+}
+
+int ra_set_prompt_pool(ra_ctx* ctx, int max_prompt_len, long long pool_positions)
+{
+    if (!ctx) return fail(nullptr, RA_ERR_INVALID_ARG, "ctx is NULL");
+    if (ctx->bound) return fail(ctx, RA_ERR_STATE, "the prompt pool must be set before ra_device_bytes / ra_bind");
+    if (max_prompt_len < 0 || pool_positions < 0) return fail(ctx, RA_ERR_INVALID_ARG, "negative size");
+    long long need = 0;
+    int longest = 0;
+    for (int b = 0; b < ctx->B; ++b) {
+        need += (ctx->lp[b] + kPromptPage - 1) / kPromptPage;
+        longest = std::max(longest, (int)ctx->lp[b]);
+    }
+    const int old_max = ctx->max_prompt;
+    const long long old_pool = ctx->pool_pages;
+    ctx->max_prompt = std::max(longest, max_prompt_len);
+    ctx->pool_pages = std::max(need, (pool_positions + kPromptPage - 1) / kPromptPage);
+    int rc = layout_base(ctx);
+    if (rc != RA_OK) {  // too large: keep the previous pool
+        ctx->max_prompt = old_max;
+        ctx->pool_pages = old_pool;
+        layout_base(ctx);
+        return fail(ctx, rc, "%s", ra_last_error(nullptr));
+    }
+    return RA_OK;
+}
+
+int ra_admit(ra_ctx* ctx, int seq, int prompt_len, const uint16_t* k, const uint16_t* v, int row_stride, void* stream)
+{
+    int rc;
+    if ((rc = check_bound(ctx)) != RA_OK) return rc;
+    if (seq < 0 || seq >= ctx->B) return fail(ctx, RA_ERR_INVALID_ARG, "seq %d out of range", seq);
+    if (ctx->active[seq]) return fail(ctx, RA_ERR_STATE, "seq %d is active: finish it (ra_set_active 0) first", seq);
+    if (prompt_len < 0 || prompt_len > ctx->max_prompt)
+        return fail(ctx, RA_ERR_CAPACITY, "prompt of %d tokens: the slots take up to %d (ra_set_prompt_pool)", prompt_len,
+                    ctx->max_prompt);
+    if (prompt_len > 0 && (!k || !v || !aligned16(k) || !aligned16(v) || row_stride < prompt_len))
+        return fail(ctx, RA_ERR_INVALID_ARG, "k/v must be 16-byte aligned with row_stride >= prompt_len");
+    if (ctx->admits[seq] >= 0xFFFF) return fail(ctx, RA_ERR_CAPACITY, "slot %d has taken 65535 requests", seq);
+    const int old_n = (ctx->lp[seq] + kPromptPage - 1) / kPromptPage, new_n = (prompt_len + kPromptPage - 1) / kPromptPage;
+    if ((long long)ctx->free_pages.size() + old_n < new_n)
+        return fail(ctx, RA_ERR_CAPACITY, "prompt pool has %zu free pages, the request needs %d",
+                    ctx->free_pages.size() + old_n, new_n);
+    cudaStream_t s = (cudaStream_t)stream;
+    int32_t* row = ctx->pages.data() + (size_t)seq * ctx->max_pages;
+    for (int j = 0; j < old_n; ++j) ctx->free_pages.push_back(row[j]);
+    for (int j = 0; j < new_n; ++j) {
+        row[j] = ctx->free_pages.back();
+        ctx->free_pages.pop_back();
+    }
+    ctx->lp[seq] = prompt_len;
+    cudaError_t e;
+    // (pageable sources: the calls return once the values are staged)
+    if ((e = cudaMemcpyAsync(ctx->lay.pages + (size_t)seq * ctx->max_pages, row, (size_t)ctx->max_pages * 4,
+                             cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(ctx->lay.seq_lp + seq, &ctx->lp[seq], 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(ctx, e, "page table update");
+    if (prompt_len > 0) {
+        CopyRowsParams p{};
+        p.lay = ctx->lay;
+        p.k = k;
+        p.v = v;
+        p.row_stride = row_stride;
+        p.only_seq = seq;
+        p.n_rows[seq] = prompt_len;
+        for (int l = 0; l < ctx->L; ++l) {
+            p.layer = l;
+            p.k = k + (size_t)l * ctx->KVH * row_stride * kHeadDim;
+            p.v = v + (size_t)l * ctx->KVH * row_stride * kHeadDim;
+            if ((e = launch_prefill(p, s)) != cudaSuccess) return cuda_fail(ctx, e, "admit prefill launch");
+        }
+    }
+    // a fresh request: nothing generated, nothing cached, its own random stream
+    for (int l = 0; l < ctx->L; ++l) {
+        const size_t i = (size_t)l * ctx->B + seq;
+        ctx->g[i] = ctx->c[i] = ctx->nev[i] = 0;
+        ctx->score_n[i] = 0;
+        ctx->plan_g[i] = ctx->plan_g[(size_t)ctx->L * ctx->B + i] = -1;
+    }
+    ctx->admits[seq] += 1;
+    ctx->active[seq] = 1;
     return RA_OK;
 }
 
@@ -1126,6 +1241,7 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
             const int g2 = g1 + 1, c2 = (fires ? ctx->K + ctx->r : c1) + 1;
             if (g2 % ctx->r == 0 && c2 - ctx->r > ctx->K && c2 - ctx->r <= ctx->K + ctx->r) {
                 pp.trig[n] = (int16_t)b;
+                pp.trig_admit[n] = (uint16_t)ctx->admits[b];
                 pp.trig_g[n] = g2;
                 pp.trig_n[n] = c2 - ctx->r;
                 ++n;
@@ -1216,15 +1332,19 @@ int ra_get_kv(ra_ctx* ctx, int layer, int seq, int kv_head, uint16_t* host_k, ui
         return fail(ctx, RA_ERR_INVALID_ARG, "capacity %d < %d rows", capacity_rows, lp + c);
     int32_t reg;
     if ((rc = read_region(ctx, layer, seq, kv_head, &reg, (cudaStream_t)stream)) != RA_OK) return rc;
-    const long long prow = (long long)layer * ctx->prompt_rows_per_layer + ctx->poff[seq] + (long long)kv_head * lp;
     const long long grow = ctx->lay.gen_row0 + (long long)reg * ctx->Cmax;
     cudaError_t e;
     for (int w = 0; w < 2; ++w) {
         const uint16_t* pool = w ? ctx->lay.vpool : ctx->lay.kpool;
         uint16_t* dst = w ? host_v : host_k;
-        if (lp > 0 && (e = cudaMemcpy(dst, pool + prow * kHeadDim, (size_t)lp * kRowBytes, cudaMemcpyDeviceToHost)) !=
-                          cudaSuccess)
-            return cuda_fail(ctx, e, "prompt rows read");
+        for (int p0 = 0; p0 < lp; p0 += kPromptPage) {  // the prompt, page by page
+            const int32_t page = ctx->pages[(size_t)seq * ctx->max_pages + p0 / kPromptPage];
+            const long long prow = prompt_row(ctx->lay, layer, page, kv_head, 0);
+            const int n = std::min(kPromptPage, lp - p0);
+            if ((e = cudaMemcpy(dst + (size_t)p0 * kHeadDim, pool + prow * kHeadDim, (size_t)n * kRowBytes,
+                                cudaMemcpyDeviceToHost)) != cudaSuccess)
+                return cuda_fail(ctx, e, "prompt rows read");
+        }
         if (c > 0 && (e = cudaMemcpy(dst + (size_t)lp * kHeadDim, pool + grow * kHeadDim, (size_t)c * kRowBytes,
                                      cudaMemcpyDeviceToHost)) != cudaSuccess)
             return cuda_fail(ctx, e, "generated rows read");

@@ -111,6 +111,7 @@ struct Cfg {
     static constexpr int MCH = kHeadDim / LG;
     static_assert(G >= 1 && G <= 8, "the 16-row MMA holds up to 8 query heads");
     static_assert(TILE % 16 == 0 && TILE <= 256, "whole 16-row MMA batches; TMA box rows <= 256");
+    static_assert(kPromptPage % TILE == 0, "a prompt tile lies inside one page");
     static_assert(HALF_BYTES % 1024 == 0, "128-byte-swizzled TMA boxes start 1024-byte aligned");
     static_assert(WARPS >= 2, "shared-memory budget too small");
     static_assert(SMEM <= 232448, "fits the 227 KB opt-in shared memory of sm_100+");
@@ -127,7 +128,9 @@ struct TileIter {
     int nt, tp;                      // tiles in the head, prompt tiles among them
     int lp, gen;                     // prompt rows, generated rows (incl. a fused new token)
     bool comp;                       // the head compacts in this launch: its generated rows are the old region's
-    long long prow, grow;            // first prompt row / first generated row of the head
+    long long pbase, grow;           // the head's prompt rows: pbase + page * KVH * kPromptPage + offset; first generated row
+    const int32_t* ptab;             // the sequence's page table
+    int pg_i, pg_cur, pg_next;       // page-table entry i of the current prompt tile, and entry i + 1 (read ahead)
     bool piece_start;
 };
 
@@ -148,7 +151,13 @@ __device__ __forceinline__ void enter_head(TileIter& it, const AttnParams& p)
     it.lp = L.seq_lp[it.b];
     it.gen = p.seq_gen[it.b];
     it.tp = (it.lp + p.tile - 1) / p.tile;
-    it.prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[it.b] + (long long)it.h * it.lp;
+    it.pbase = prompt_row(L, p.layer, 0, it.h, 0);
+    it.ptab = L.pages + (size_t)it.b * L.max_pages;
+    it.pg_i = 0;
+    if (it.lp > 0) {
+        it.pg_cur = __ldg(it.ptab);
+        it.pg_next = it.lp > kPromptPage ? __ldg(it.ptab + 1) : 0;
+    }
     it.comp = COMPACT && ((p.compacting[it.b >> 5] >> (it.b & 31)) & 1u);
     const int reg = it.comp ? L.plan[(size_t)(it.b * L.KVH + it.h) * (kPlanHeader + L.r)]  // the old region
                             : L.region[((size_t)p.layer * L.B + it.b) * L.KVH + it.h];
@@ -193,9 +202,15 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int wa
     if (it.f >= it.end && !iter_next_chunk<COMPACT>(it, p, warp_id)) return false;
     const int T = p.tile;
     d.flags = (it.piece_start ? kFirst : 0) | (it.k == 0 ? kHead0 : 0);
-    if (it.k < it.tp) {
-        d.row = it.prow + (long long)it.k * T;
-        d.n = min(T, it.lp - it.k * T);
+    if (it.k < it.tp) {  // a prompt tile lies inside one page (kPromptPage is a multiple of T)
+        const int p0 = it.k * T, pi = p0 / kPromptPage;
+        if (pi != it.pg_i) {  // another page: the next one's entry was read ahead (a chunk may start mid-prompt)
+            it.pg_cur = pi == it.pg_i + 1 ? it.pg_next : __ldg(it.ptab + pi);
+            it.pg_i = pi;
+            it.pg_next = (pi + 1) * kPromptPage < it.lp ? __ldg(it.ptab + pi + 1) : 0;
+        }
+        d.row = it.pbase + (long long)it.pg_cur * p.lay.KVH * kPromptPage + p0 % kPromptPage;
+        d.n = min(T, it.lp - p0);
     } else {
         const int kg = it.k - it.tp;
         d.row = it.grow + (long long)kg * T;

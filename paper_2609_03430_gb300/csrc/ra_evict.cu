@@ -129,7 +129,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
     const int32_t* pos = L.pos + (size_t)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
     if (p.holefill && p.policy != RA_POLICY_BLOCK) {  // order-free slots: every key follows the position
-        const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
+        const uint32_t id = key_stream(p.trig_admit[blockIdx.x],
+                                       p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id);
 #pragma unroll 8
         for (int j = tid; j < N; j += kSelThreads) {
             const uint32_t pj = (uint32_t)__ldg(pos + j);
@@ -140,8 +141,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         for (int j = tid; j < N; j += kSelThreads) keys[j] = (uint32_t)(N - 1 - j);
     } else if (p.policy == RA_POLICY_BLOCK) {  // one draw per block of consecutive positions
         for (int j = tid; j < N; j += kSelThreads)
-            keys[j] = philox4x32_10_w0((uint32_t)(pos[j] / p.block), (uint32_t)g, (uint32_t)p.layer, (uint32_t)head_id,
-                                       k0, k1);
+            keys[j] = philox4x32_10_w0((uint32_t)(pos[j] / p.block), (uint32_t)g, (uint32_t)p.layer,
+                                       key_stream(p.trig_admit[blockIdx.x], (uint32_t)head_id), k0, k1);
     } else if (p.policy == RA_POLICY_SNAPKV) {
         // scored comparator: the window score max-pooled over +-kScorePoolRadius candidates;
         // larger scores must sort first, so the key is the order-reversed float
@@ -162,7 +163,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
             keys[j] = ~asc;
         }
     } else {  // random: an independent draw per KV head; shared: one draw for all heads of the sequence
-        const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
+        const uint32_t id = key_stream(p.trig_admit[blockIdx.x],
+                                       p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id);
         for (int j = tid; j < N; j += kSelThreads)
             keys[j] = philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)p.layer, id, k0, k1);
     }
@@ -539,7 +541,8 @@ __global__ void __launch_bounds__(kEvThreads, 1) evict_kernel(const __grid_const
     const uint64_t E = 2ull * (uint64_t)m + 32ull;
     const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
     const uint32_t k0 = (uint32_t)L.seed, k1 = (uint32_t)(L.seed >> 32);
-    const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id;
+    const uint32_t id =
+        key_stream(p.trig_admit[t], p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)head_id);
     const int32_t* spos = L.pos + (size_t)src * L.Cmax;
     auto record = [&](int i, uint32_t key) {  // the key of local candidate i: kept, listed or counted
         S.keys[i] = key;
@@ -578,7 +581,7 @@ __global__ void __launch_bounds__(kEvThreads, 1) evict_kernel(const __grid_const
             record(i, p.policy == RA_POLICY_RECENCY  // the K newest candidates score lowest
                           ? (uint32_t)(N - 1 - j)
                           : philox4x32_10_w0((uint32_t)(__ldg(spos + j) / p.block), (uint32_t)g, (uint32_t)p.layer,
-                                             (uint32_t)head_id, k0, k1));
+                                             key_stream(p.trig_admit[t], (uint32_t)head_id), k0, k1));
         }
     }
     if (lane == 0) {  // this warp's copy barriers
@@ -913,7 +916,8 @@ __global__ void __launch_bounds__(kPlanThreads) plan_kernel(const __grid_constan
         if (tid == 0) out[0] = -1;
         return;
     }
-    const uint32_t id = p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)(b * L.KVH + h);
+    const uint32_t id =
+        key_stream(p.trig_admit[t], p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)(b * L.KVH + h));
     const bool cut = (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) && !p.ev_exact;
     if (cut) {
         const uint64_t E = 2ull * (uint64_t)m + 32ull;
@@ -1059,24 +1063,24 @@ __global__ void __launch_bounds__(32) timeout_probe_kernel(int32_t* err, uint64_
 __global__ void __launch_bounds__(256) copy_rows_kernel(const __grid_constant__ CopyRowsParams p, int restore)
 {
     const DevLayout& L = p.lay;
-    const int b = blockIdx.x / L.KVH, h = blockIdx.x % L.KVH;
+    const int b = p.only_seq >= 0 ? p.only_seq : (int)blockIdx.x / L.KVH, h = blockIdx.x % L.KVH;
     const int n = p.n_rows[b];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    long long row0;
+    long long row0 = 0;
     int32_t* dpos = nullptr;
+    const int32_t* ptab = L.pages + (size_t)b * L.max_pages;
     if (restore) {
         const int reg = L.region[((size_t)p.layer * L.B + b) * L.KVH + h];
         row0 = L.gen_row0 + (long long)reg * L.Cmax;
         dpos = L.pos + (size_t)reg * L.Cmax;
-    } else {
-        row0 = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[b] + (long long)h * L.seq_lp[b];
     }
-    const size_t src0 = ((size_t)b * L.KVH + h) * (size_t)p.row_stride;
+    const size_t src0 = ((p.only_seq >= 0 ? 0 : (size_t)b * L.KVH) + h) * (size_t)p.row_stride;
     const uint16_t* sb = (lane < 16 ? p.k : p.v);
     uint16_t* db = (lane < 16 ? L.kpool : L.vpool);
     for (int i = warp; i < n; i += 8) {
         const uint4 v = reinterpret_cast<const uint4*>(sb + (src0 + i) * kHeadDim)[lane & 15];
-        reinterpret_cast<uint4*>(db + (row0 + i) * kHeadDim)[lane & 15] = v;
+        const long long row = restore ? row0 + i : prompt_row(L, p.layer, ptab[i / kPromptPage], h, i);
+        reinterpret_cast<uint4*>(db + row * kHeadDim)[lane & 15] = v;
         if (restore && lane == 0) dpos[i] = p.pos[src0 + i];
     }
 }
@@ -1225,7 +1229,7 @@ cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s
 
 cudaError_t launch_prefill(const CopyRowsParams& p, cudaStream_t s)
 {
-    copy_rows_kernel<<<p.lay.B * p.lay.KVH, 256, 0, s>>>(p, 0);
+    copy_rows_kernel<<<(p.only_seq >= 0 ? 1 : p.lay.B) * p.lay.KVH, 256, 0, s>>>(p, 0);
     return cudaGetLastError();
 }
 

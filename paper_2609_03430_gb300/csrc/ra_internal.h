@@ -20,6 +20,10 @@ constexpr int kMaxCandidates = 32768;    // K + r bound (select keeps one u32 ke
 // Split-K partial record of one (warp, KV head) piece: o[G][128], m[G], l[G] in fp32,
 // padded to a multiple of 4 floats so that every record starts 16-byte aligned.
 __host__ __device__ constexpr int partial_stride(int G) { return G * 128 + ((2 * G + 3) / 4) * 4; }
+// Prompt rows live in pages of kPromptPage positions x all KV heads of one sequence (a multiple of
+// every kernel's tile height: 48 and 32 rows for attention, 64 for scoring), listed per sequence
+// in a page table, so that a finished sequence's slot can take a new request of another length.
+constexpr int kPromptPage = 192;
 constexpr int kDeviceErrTimeout = 1;     // values of the device error word
 constexpr int kDeviceErrPlan = 2;
 
@@ -31,7 +35,7 @@ struct DevLayout {
     int32_t* region;       // [L][B][KVH] region index currently holding a head's generated slots
     int32_t* spare;        // [B][KVH] the free region that a head's next compaction writes into
     int32_t* seq_lp;       // [B] prompt length
-    int32_t* seq_poff;     // [B] row offset of a sequence's prompt block inside a layer (KVH * sum lp)
+    int32_t* pages;        // [B][max_pages] page of each kPromptPage-position block of a sequence's prompt
     int32_t* plan;         // [B*KVH][kPlanHeader + r] eviction plan of the current layer
     float* partial;        // attention split partials
     int32_t* arrive;       // [B*KVH] split-piece arrival counters
@@ -43,7 +47,8 @@ struct DevLayout {
     float2* qstats;        // [L][B][KVH][r][G] per window query: (its scale * log2 e, log2 of its softmax sum)
     float* stats;          // [B*KVH][stats_chunks][M][2] restore pass: softmax statistics (max, sum) per chunk
     int stats_chunks;      // chunks per head the stats buffer holds
-    long long prompt_rows_per_layer;
+    long long prompt_rows_per_layer;  // pool pages * KVH * kPromptPage
+    int max_pages;
     long long gen_row0;    // first row of the generated regions
     int L, B, KVH, H, G, Cmax, K, r;
     uint64_t seed;
@@ -80,6 +85,9 @@ struct EvictParams {
     // spare are region_base * KVH + kv_head (one-launch eviction; checked against the tables)
     int32_t trig_src[RA_MAX_BATCH];
     int32_t trig_dst[RA_MAX_BATCH];
+    // requests admitted into the slot before the current one: the key stream of a head is
+    // (admissions << 16) | head id, so that a new request draws its own numbers
+    uint16_t trig_admit[RA_MAX_BATCH];
     // scored policy: tiles (of kScoreTile rows) per CTA of each pass, CTAs per head of each pass
     int ch1, ch2, nch1, nch2;
     float qk_scale_log2;  // restore pass: the scale * log2 e the restored queries are taken at
@@ -132,12 +140,21 @@ struct AttnParams {
 struct CopyRowsParams {
     DevLayout lay;
     int layer;
-    const uint16_t* k;  // [B][KVH][row_stride][128]
+    const uint16_t* k;  // [B][KVH][row_stride][128] (one sequence's [KVH][row_stride][128] when only_seq >= 0)
     const uint16_t* v;
     const int32_t* pos; // restore only: [B][KVH][row_stride]
     int row_stride;
+    int only_seq;       // >= 0: the launch copies that sequence alone (one CTA per KV head)
     int32_t n_rows[RA_MAX_BATCH];  // rows to copy per sequence
 };
+
+// Cache row of prompt position `pos` of (layer, KV head h) in `page` (the sequence's page-table
+// entry for block pos / kPromptPage).
+__host__ __device__ inline long long prompt_row(const DevLayout& L, int layer, int32_t page, int h, int pos)
+{
+    return (long long)layer * L.prompt_rows_per_layer + ((long long)page * L.KVH + h) * kPromptPage + pos % kPromptPage;
+}
+__host__ __device__ inline uint32_t key_stream(uint32_t admissions, uint32_t head) { return (admissions << 16) | head; }
 
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_append(const AppendParams& p, int B, cudaStream_t s);

@@ -40,6 +40,7 @@
 #include "ra_ptx.cuh"
 
 namespace ra {
+static_assert(kPromptPage % kScoreTile == 0, "a scoring tile of the prompt lies inside one page");
 namespace {
 
 constexpr int kThreads = 256;
@@ -143,14 +144,18 @@ __global__ void __launch_bounds__(kThreads, MT <= 2 ? 2 : 1) score_stats_kernel(
     const int t0 = blockIdx.x * ch;
     if (t0 >= nt_head) return;  // (exiting counts as letting the successor start)
     const int ntile = min(ch, nt_head - t0);
-    const long long prow = (long long)p.layer * L.prompt_rows_per_layer + L.seq_poff[b] + (long long)h * lp;
+    const long long pbase = prompt_row(L, p.layer, 0, h, 0);
+    const int32_t* ptab = L.pages + (size_t)b * L.max_pages;
     const size_t lbh = ((size_t)p.layer * L.B + b) * L.KVH + h;
     const int reg = L.region[lbh];
     const long long grow = L.gen_row0 + (long long)reg * L.Cmax;
     const int hid = b * L.KVH + h;
 
     auto tile_row = [&](int k) -> long long {  // first cache row of the head's tile k
-        return k < tp ? prow + (long long)k * kScoreTile : grow + (long long)(k - tp) * kScoreTile;
+        // (a prompt tile lies inside one page: kPromptPage is a multiple of kScoreTile)
+        return k < tp ? pbase + (long long)__ldg(ptab + k * kScoreTile / kPromptPage) * L.KVH * kPromptPage +
+                            (k * kScoreTile) % kPromptPage
+                      : grow + (long long)(k - tp) * kScoreTile;
     };
     // thread 0: tile t0 + i into stage i % 2 (one arrival per phase: `extra` bytes of other copies
     // completing on the same barrier are expected together with the tile)

@@ -59,7 +59,7 @@ class Runner:
     """A small workload run through the C ABI with an oracle mirror of every head."""
 
     def __init__(self, L, H, KVH, prompt_lens, K, r, eseed, dseed, key_scale=None, D=128, fused=False, policy=0,
-                 block=1, compaction=0, attn_shape=0):
+                 block=1, compaction=0, attn_shape=0, prompt_pool=None):
         import torch
 
         import paper_2609_03430_gb300 as ra
@@ -71,8 +71,9 @@ class Runner:
         self.B = len(self.lp)
         self.K, self.r, self.eseed, self.dseed = K, r, eseed, dseed
         self.key_scale = key_scale  # fp32 [L][KVH][D] or None
+        self.req = [0] * self.B  # requests each slot took after the first (their rows differ: see sid)
         self.cache = ra.RandomAttentionCache(L, H, KVH, D, self.lp, K, r, eseed, policy=policy, block=block,
-                                             compaction=compaction)
+                                             compaction=compaction, prompt_pool=prompt_pool)
         self.ctx = self.cache.ctx
         if attn_shape:
             ra.ra_set_attention_shape(self.ctx, attn_shape)
@@ -102,12 +103,38 @@ class Runner:
     def up(self, a):
         return self.torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(self.dev)
 
+    def sid(self, b):
+        """The generator's sequence index of slot b's current request."""
+        return b + 64 * self.req[b]
+
     def krows(self, l, b, h, pos):
         sc = None if self.key_scale is None else self.key_scale[l, h]
-        return synth.kv_rows(self.dseed, 0, l, b, h, pos, self.D, sc)
+        return synth.kv_rows(self.dseed, 0, l, self.sid(b), h, pos, self.D, sc)
 
     def vrows(self, l, b, h, pos):
-        return synth.kv_rows(self.dseed, 1, l, b, h, pos, self.D)
+        return synth.kv_rows(self.dseed, 1, l, self.sid(b), h, pos, self.D)
+
+    def qrows(self, l, b, step):
+        return synth.q_rows(self.dseed, l, self.sid(b), np.arange(self.H), step, self.D)
+
+    def admit(self, b, prompt_len):
+        """Finish slot b's request and admit a new one with its own prompt (ra_admit)."""
+        self.set_active(b, False)
+        self.req[b] += 1
+        self.qsteps[b] = []  # the new request's decode steps
+        self.lp[b] = prompt_len
+        k = np.zeros((self.L, self.KVH, max(prompt_len, 1), self.D), np.uint16)
+        v = np.zeros_like(k)
+        for l in range(self.L):
+            for h in range(self.KVH):
+                if prompt_len:
+                    k[l, h, :prompt_len] = self.krows(l, b, h, np.arange(prompt_len))
+                    v[l, h, :prompt_len] = self.vrows(l, b, h, np.arange(prompt_len))
+        tk, tv = self.up(k), self.up(v)
+        self.ra.ra_admit(self.ctx, b, prompt_len, tk.data_ptr(), tv.data_ptr(), max(prompt_len, 1))
+        self.torch.cuda.synchronize()
+        self.orc.admit(b, prompt_len)
+        self.active[b] = True
 
     def set_active(self, b, on):
         self.active[b] = on
@@ -133,8 +160,7 @@ class Runner:
                     k[b, h] = self.krows(l, b, h, [pos])[0]
                     v[b, h] = self.vrows(l, b, h, [pos])[0]
             tk, tv = self.up(k), self.up(v)  # keep both alive: a freed temporary would be reused for the next
-            q = np.stack([synth.q_rows(self.dseed, l, b, np.arange(self.H), self.step_idx, self.D)
-                          for b in range(self.B)])
+            q = np.stack([self.qrows(l, b, self.step_idx) for b in range(self.B)])
             out = self.torch.zeros((self.B, self.H, self.D), dtype=self.torch.int16, device=self.dev)
             tq = self.up(q)
             if not scored:
@@ -162,7 +188,7 @@ class Runner:
         """Query rows [r][G][D] and positions of the window at an eviction after token g."""
         steps = range(g - self.r, g)  # 1-based decode steps of the window
         heads = np.arange(h * self.G, (h + 1) * self.G)
-        q = np.stack([synth.q_rows(self.dseed, l, b, heads, self.qsteps[b][s - 1], self.D) for s in steps])
+        q = np.stack([synth.q_rows(self.dseed, l, self.sid(b), heads, self.qsteps[b][s - 1], self.D) for s in steps])
         return q, np.array([self.lp[b] + s - 1 for s in steps], dtype=np.int32)
 
     def scorer(self, b, l, h, cur):

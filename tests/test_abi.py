@@ -69,7 +69,8 @@ def test_create_validation_is_host_only(ra):
 def test_device_bytes_cover_the_caches(ra):
     # config-2 shape: 36 layers, 16 seqs, 8 KV heads, prompt 512, K 2048, r 64
     ctx = ra.ra_create_batched(36, 32, 8, 128, [512] * 16, 2048, 64, 2)
-    rows = 36 * 16 * 8 * 512 + (36 + 1) * 16 * 8 * (2048 + 128)
+    # prompts in pages of 192 positions: 512 -> 3 pages
+    rows = 36 * 16 * 8 * 3 * 192 + (36 + 1) * 16 * 8 * (2048 + 128)
     assert ra.ra_device_bytes(ctx) >= 2 * rows * 256 + (36 + 1) * 16 * 8 * (2048 + 128) * 4
     assert ra.ra_device_bytes(ctx) < 2 * rows * 256 * 1.01 + (64 << 20)
     ra.ra_destroy(ctx)
@@ -129,3 +130,22 @@ def test_no_cpu_fallback_in_product_package():
             if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
                 src = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in src and "from oracle" not in src and "ra_oracle" not in src, f
+
+
+def test_prompt_pool_sizing_and_admission_validation(ra):
+    """The prompt pool is set before binding (pages of 192 positions); admission is refused on
+    unbound contexts, and the pool can only grow past what the creation prompts use."""
+    L = ra.lib()
+    ctx = ra.ra_create_batched(2, 8, 2, 128, [100, 300, 0], 64, 16, 0)
+    base = ra.ra_device_bytes(ctx)
+    ra.ra_set_prompt_pool(ctx, 4000, 3 * 4000)  # room for three 4000-token prompts
+    grown = ra.ra_device_bytes(ctx)
+    pages = -(-12000 // 192)
+    assert grown >= base + 2 * 2 * 2 * (pages - 3) * 192 * 256  # K and V, 2 layers, 2 heads, extra pages
+    ra.ra_set_prompt_pool(ctx, 0, 0)  # never below the creation prompts
+    assert ra.ra_device_bytes(ctx) == base
+    assert L.ra_admit(ctx, 0, 10, None, None, 10, None) == ra.RA_ERR_STATE  # unbound
+    with pytest.raises(ra.RAError) as e:
+        ra.ra_set_prompt_pool(ctx, -1, 0)
+    assert e.value.code == ra.RA_ERR_INVALID_ARG
+    ra.ra_destroy(ctx)
