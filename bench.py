@@ -452,16 +452,20 @@ def attention_window(wl, steps, t_next):
     def evict_bytes():  # algorithmic bytes of the eviction launches so far (library count)
         return sum(ra.ra_profile_read(wl.ctx, k)[2] for k in ev_kinds)
 
+    # (host bookkeeping between steps stays light -- a few calls -- so that the host keeps ahead of
+    # the device; every layer of a sequence evicts on the same step, so rounds = sequences x layers)
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
     marks = []
     evs[0].record(wl.stream)
+    n0, e0 = evictions_layer0(), evict_bytes()
+    _, l0, b0 = ra.ra_profile_read(wl.ctx, kind)
     for i, t in enumerate(range(t_next, t_next + steps)):
-        n0, r0, e0 = evictions_layer0(), wl.evictions(), evict_bytes()
-        _, l0, b0 = ra.ra_profile_read(wl.ctx, kind)
         wl.step(t)
         evs[i + 1].record(wl.stream)
+        n1, e1 = evictions_layer0(), evict_bytes()
         _, l1, b1 = ra.ra_profile_read(wl.ctx, kind)
-        marks.append((evictions_layer0() != n0, l1 - l0, b1 - b0, wl.evictions() - r0, evict_bytes() - e0))
+        marks.append((n1 != n0, l1 - l0, b1 - b0, (n1 - n0) * wl.L, e1 - e0))
+        n0, e0, l0, b0 = n1, e1, l1, b1
     torch.cuda.synchronize()
     steps_ms = [(evs[i].elapsed_time(evs[i + 1]),) + m for i, m in enumerate(marks)]
     clean = [(ms, n, by) for (ms, fired, n, by, _, _) in steps_ms if not fired and n > 0]

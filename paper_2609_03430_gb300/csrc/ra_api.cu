@@ -1254,7 +1254,7 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
                 return cuda_fail(ctx, e, "plan fork");
             {
                 ProfScope ps(ctx, RA_KERNEL_PLAN, 0.0, ctx->side);
-                e = launch_plan(pp, ctx->side);
+                e = launch_plan(pp, ctx->sms, ctx->side);
                 ps.done();
             }
             if (e != cudaSuccess) return cuda_fail(ctx, e, "plan launch");

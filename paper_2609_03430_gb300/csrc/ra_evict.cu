@@ -27,6 +27,8 @@
 //                   each other; the old region becomes the spare.
 #include <cuda_runtime.h>
 #include <limits.h>
+
+#include <algorithm>
 #include <stdint.h>
 
 #include "ra_internal.h"
@@ -878,22 +880,19 @@ __global__ void __launch_bounds__(kEvThreads, 1) evict_kernel(const __grid_const
 // ----------------------------------------------------------------------------- plan (evicted sets ahead)
 // The random draw reads no cache data: a candidate's key depends only on (ordinal, step, layer,
 // head), so the evicted set of a firing step is known as soon as the counters are.  plan_kernel
-// computes it ahead, one CTA per (layer, sequence, KV head), with the same exact rules as
-// evict_kernel: the sampled cut and an exact ranking of the listed pairs, or -- when fewer than
-// m pass, for recency keys, or with RA_EVICT_EXACT -- four radix passes over recomputed keys
-// (no key is stored: 7 KB of shared memory, so the kernel fits beside an attention CTA on the
-// same SM) and one ascending sweep that writes the evicted ordinals in order, ties at the
-// threshold evicted from the largest ordinal down.  Output: [m][ordinals ascending].
-constexpr int kPlanThreads = 256;
-constexpr int kPlanWarps = kPlanThreads / 32;
-
+// computes it ahead, beside the attention of the step before: one warp per CTA and about one CTA
+// per SM, each looping over (layer, sequence, KV head) items, so that it takes a sliver of each
+// SM's issue slots (7 KB of shared memory: it fits beside an attention CTA).  Per item, the
+// same exact rules as evict_kernel: the sampled cut and an exact ranking of the listed pairs, or
+// -- when fewer than m pass, for recency keys, or with RA_EVICT_EXACT -- four radix passes over
+// recomputed keys (none is stored) and one ascending sweep that writes the evicted ordinals in
+// order, ties at the threshold evicted from the largest ordinal down.  Output per item:
+// [m][ordinals ascending] (-1 if the item is out of range).
 struct PlanShared {
     uint2 list[kEvCap];
     int32_t ev[kEvCap];
     uint32_t hist[256];
-    uint32_t wsum[2][kPlanWarps];
     uint32_t cnt, nev;
-    uint32_t sel[4];
 };
 
 __device__ __forceinline__ uint32_t plan_key(const EvictParams& p, int layer, uint32_t id, int N, int g, int j)
@@ -903,80 +902,90 @@ __device__ __forceinline__ uint32_t plan_key(const EvictParams& p, int layer, ui
                             (uint32_t)(p.lay.seed >> 32));
 }
 
-__global__ void __launch_bounds__(kPlanThreads) plan_kernel(const __grid_constant__ EvictParams p)
+__global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictParams p)
 {
     __shared__ PlanShared S;
     const DevLayout& L = p.lay;
-    const int h = blockIdx.x, t = blockIdx.y, layer = blockIdx.z;
-    const int b = p.trig[t], N = p.trig_n[t], g = p.trig_g[t];
-    const int m = N - L.K;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    int32_t* out = L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
-    if (m < 1 || m > L.r || m > kEvCap || N > kMaxCandidates) {  // the host rules this out; the copy rejects it
-        if (tid == 0) out[0] = -1;
-        return;
-    }
-    const uint32_t id =
-        key_stream(p.trig_admit[t], p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)(b * L.KVH + h));
-    const bool cut = (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) && !p.ev_exact;
-    if (cut) {
-        const uint64_t E = 2ull * (uint64_t)m + 32ull;
-        const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
-        if (tid == 0) {
-            S.cnt = 0;
-            S.nev = 0;
+    const int lane = threadIdx.x;
+    const int items = L.L * p.n_trig * L.KVH;
+    for (int item = blockIdx.x; item < items; item += gridDim.x) {
+        const int h = item % L.KVH, t = (item / L.KVH) % p.n_trig, layer = item / (L.KVH * p.n_trig);
+        const int b = p.trig[t], N = p.trig_n[t], g = p.trig_g[t];
+        const int m = N - L.K;
+        int32_t* out =
+            L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
+        if (m < 1 || m > L.r || m > kEvCap || N > kMaxCandidates) {  // the host rules this out; the copy rejects it
+            if (lane == 0) out[0] = -1;
+            continue;
         }
-        __syncthreads();
-        for (int j0 = tid; j0 < N; j0 += 4 * kPlanThreads) {  // four independent Philox chains at a time
-            uint32_t kq[4];
+        const uint32_t id = key_stream(p.trig_admit[t],
+                                       p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)(b * L.KVH + h));
+        const bool cut = (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) && !p.ev_exact;
+        bool done = false;
+        if (cut) {
+            const uint64_t E = 2ull * (uint64_t)m + 32ull;
+            const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
+            uint32_t cnt = 0;  // warp-uniform
+            for (int j0 = lane; j0 < N; j0 += 4 * 32) {  // four independent Philox chains at a time
+                uint32_t kq[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) kq[q] = plan_key(p, layer, id, N, g, j0 + q * kPlanThreads);
+                for (int q = 0; q < 4; ++q) kq[q] = plan_key(p, layer, id, N, g, j0 + q * 32);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = j0 + q * kPlanThreads;
-                if (j < N && kq[q] >= tau) {
-                    const uint32_t at = atomicAdd(&S.cnt, 1u);
-                    if (at < (uint32_t)kEvCap) S.list[at] = make_uint2(kq[q], (uint32_t)j);
+                for (int q = 0; q < 4; ++q) {
+                    const int j = j0 + q * 32;
+                    const bool pass = j < N && kq[q] >= tau;
+                    const uint32_t bits = __ballot_sync(0xffffffffu, pass);
+                    const uint32_t at = cnt + __popc(bits & ((1u << lane) - 1u));
+                    if (pass && at < (uint32_t)kEvCap) S.list[at] = make_uint2(kq[q], (uint32_t)j);
+                    cnt += __popc(bits);
                 }
             }
-        }
-        __syncthreads();
-        const int total = (int)S.cnt;
-        if (total >= m && total <= kEvCap) {  // the top m of the list are the evicted set
-            for (int e = tid; e < total; e += kPlanThreads) {
-                const uint2 x = S.list[e];
-                int above = 0;
+            __syncwarp();
+            const int total = (int)cnt;
+            if (total >= m && total <= kEvCap) {  // the top m of the list are the evicted set
+                uint32_t nev = 0;
+                for (int e0 = 0; e0 < total; e0 += 32) {
+                    const int e = e0 + lane;
+                    bool ev = false;
+                    if (e < total) {
+                        const uint2 x = S.list[e];
+                        int above = 0;
 #pragma unroll 8
-                for (int f = 0; f < total; ++f) {
-                    const uint2 y = S.list[f];
-                    above += (y.x > x.x || (y.x == x.x && y.y > x.y)) ? 1 : 0;
+                        for (int f = 0; f < total; ++f) {
+                            const uint2 y = S.list[f];
+                            above += (y.x > x.x || (y.x == x.x && y.y > x.y)) ? 1 : 0;
+                        }
+                        ev = above < m;
+                    }
+                    const uint32_t bits = __ballot_sync(0xffffffffu, ev);
+                    if (ev) S.ev[nev + __popc(bits & ((1u << lane) - 1u))] = (int32_t)S.list[e].y;
+                    nev += __popc(bits);
                 }
-                if (above < m) S.ev[atomicAdd(&S.nev, 1u)] = (int32_t)x.y;
-            }
-            __syncthreads();
-            for (int e = tid; e < m; e += kPlanThreads) {  // ascending by ordinal
-                const int je = S.ev[e];
-                int below = 0;
+                __syncwarp();
+                for (int e = lane; e < m; e += 32) {  // ascending by ordinal
+                    const int je = S.ev[e];
+                    int below = 0;
 #pragma unroll 8
-                for (int f = 0; f < m; ++f) below += S.ev[f] < je ? 1 : 0;
-                out[1 + below] = je;
+                    for (int f = 0; f < m; ++f) below += S.ev[f] < je ? 1 : 0;
+                    out[1 + below] = je;
+                }
+                if (lane == 0) out[0] = m;
+                done = true;
             }
-            if (tid == 0) out[0] = m;
-            return;
+            __syncwarp();  // S.list and S.ev are rewritten by the next item
         }
-    }
-    // exact radix passes over recomputed keys: the need-th largest key T after four digits
-    uint32_t prefix = 0, mask = 0, need = (uint32_t)m, ties = 0;
-    for (int d = 0; d < 4; ++d) {
-        const int shift = 24 - 8 * d;
-        S.hist[tid] = 0;
-        __syncthreads();
-        for (int j = tid; j < N; j += kPlanThreads) {
-            const uint32_t key = plan_key(p, layer, id, N, g, j);
-            if ((key & mask) == prefix) atomicAdd(&S.hist[(key >> shift) & 255u], 1u);
-        }
-        __syncthreads();
-        if (warp == 0) {
+        if (done) continue;
+        // exact radix passes over recomputed keys: the need-th largest key T after four digits
+        uint32_t prefix = 0, mask = 0, need = (uint32_t)m, ties = 0;
+        for (int d = 0; d < 4; ++d) {
+            const int shift = 24 - 8 * d;
+            for (int i = lane; i < 256; i += 32) S.hist[i] = 0;
+            __syncwarp();
+            for (int j = lane; j < N; j += 32) {
+                const uint32_t key = plan_key(p, layer, id, N, g, j);
+                if ((key & mask) == prefix) atomicAdd(&S.hist[(key >> shift) & 255u], 1u);
+            }
+            __syncwarp();
             uint32_t loc[8], sum = 0;
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
@@ -990,58 +999,48 @@ __global__ void __launch_bounds__(kPlanThreads) plan_kernel(const __grid_constan
                 if (lane >= o) incl += x;
             }
             const uint32_t excl = incl - sum;
-            if (excl < need && need <= incl) {
+            uint32_t bin = 0, above = 0, cnt = 0;
+            const bool mine = excl < need && need <= incl;
+            if (mine) {
                 uint32_t cum = excl;
 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
                     if (need <= cum + loc[q]) {
-                        S.sel[0] = 255u - (uint32_t)(8 * lane + q);
-                        S.sel[1] = cum;
-                        S.sel[2] = loc[q];
+                        bin = 255u - (uint32_t)(8 * lane + q);
+                        above = cum;
+                        cnt = loc[q];
                         break;
                     }
                     cum += loc[q];
                 }
             }
+            const int src = __ffs(__ballot_sync(0xffffffffu, mine)) - 1;
+            bin = __shfl_sync(0xffffffffu, bin, src);
+            above = __shfl_sync(0xffffffffu, above, src);
+            ties = __shfl_sync(0xffffffffu, cnt, src);
+            need -= above;
+            prefix |= bin << shift;
+            mask |= 0xFFu << shift;
+            __syncwarp();  // S.hist is rewritten by the next pass
         }
-        __syncthreads();
-        need -= S.sel[1];
-        ties = S.sel[2];
-        prefix |= S.sel[0] << shift;
-        mask |= 0xFFu << shift;
-        __syncthreads();  // S.sel and S.hist are rewritten by the next pass
+        // evicted: key > T, and among the `ties` keys equal to T the `need` largest ordinals;
+        // an ascending sweep writes them in order
+        const uint32_t T = prefix, tie_from = ties - need;
+        uint32_t base_ev = 0, base_tie = 0;
+        for (int c0 = 0; c0 < N; c0 += 32) {
+            const int j = c0 + lane;
+            const uint32_t key = j < N ? plan_key(p, layer, id, N, g, j) : 0u;
+            const bool eq = j < N && key == T, gt = j < N && key > T;
+            const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+            const bool ev = gt || (eq && base_tie + __popc(eqb & ((1u << lane) - 1u)) >= tie_from);
+            const uint32_t evb = __ballot_sync(0xffffffffu, ev);
+            const uint32_t pos = base_ev + __popc(evb & ((1u << lane) - 1u));
+            if (ev && pos < (uint32_t)m) out[1 + pos] = j;
+            base_ev += __popc(evb);
+            base_tie += __popc(eqb);
+        }
+        if (lane == 0) out[0] = base_ev == (uint32_t)m ? m : -1;
     }
-    // evicted: key > T, and among the `ties` keys equal to T the `need` largest ordinals;
-    // an ascending sweep writes them in order
-    const uint32_t T = prefix, tie_from = ties - need;  // tie index from which ties are evicted
-    uint32_t base_ev = 0, base_tie = 0;
-    for (int c0 = 0; c0 < N; c0 += kPlanThreads) {
-        const int j = c0 + tid;
-        const uint32_t key = j < N ? plan_key(p, layer, id, N, g, j) : 0u;
-        const bool eq = j < N && key == T, gt = j < N && key > T;
-        const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
-        if (lane == 0) S.wsum[0][warp] = __popc(eqb);
-        __syncthreads();
-        uint32_t tie_before = base_tie + __popc(eqb & ((1u << lane) - 1u)), tie_chunk = 0;
-        for (int w = 0; w < kPlanWarps; ++w) {
-            tie_before += w < warp ? S.wsum[0][w] : 0u;
-            tie_chunk += S.wsum[0][w];
-        }
-        const bool ev = gt || (eq && tie_before >= tie_from);
-        const uint32_t evb = __ballot_sync(0xffffffffu, ev);
-        if (lane == 0) S.wsum[1][warp] = __popc(evb);
-        __syncthreads();
-        uint32_t pos = base_ev + __popc(evb & ((1u << lane) - 1u)), ev_chunk = 0;
-        for (int w = 0; w < kPlanWarps; ++w) {
-            pos += w < warp ? S.wsum[1][w] : 0u;
-            ev_chunk += S.wsum[1][w];
-        }
-        if (ev && pos < (uint32_t)m) out[1 + pos] = j;
-        base_ev += ev_chunk;
-        base_tie += tie_chunk;
-        __syncthreads();  // S.wsum is rewritten by the next chunk
-    }
-    if (tid == 0) out[0] = base_ev == (uint32_t)m ? m : -1;
 }
 
 // ----------------------------------------------------------------------------- timeout probe
@@ -1215,9 +1214,10 @@ cudaError_t launch_evict(const EvictParams& p, int cluster, cudaStream_t s)
     return cudaLaunchKernelEx(&cfg, evict_kernel<kEvRows, kEvBufs>, p);
 }
 
-cudaError_t launch_plan(const EvictParams& p, cudaStream_t s)
+cudaError_t launch_plan(const EvictParams& p, int sms, cudaStream_t s)
 {
-    plan_kernel<<<dim3((unsigned)p.lay.KVH, (unsigned)p.n_trig, (unsigned)p.lay.L), kPlanThreads, 0, s>>>(p);
+    const int items = p.lay.L * p.n_trig * p.lay.KVH;
+    plan_kernel<<<(unsigned)std::min(items, std::max(sms, 1)), 32, 0, s>>>(p);
     return cudaGetLastError();
 }
 

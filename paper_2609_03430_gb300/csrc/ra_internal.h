@@ -172,9 +172,10 @@ constexpr int kEvRows = 16;  // rows per copy buffer (8 KB of K and V)
 constexpr int kEvBufs = 3;   // copy buffers per warp: 192 KB per CTA, one CTA per SM
 cudaError_t launch_evict(const EvictParams& p, int cluster, cudaStream_t s);
 // The evicted sets of the triggered sequences' heads in every layer, from the counters alone
-// (the random draw reads no cache data), into half p.ev_plan_parity of lay.evplan; one CTA per
-// (layer, sequence, KV head), little shared memory, so that it runs beside the attention kernel.
-cudaError_t launch_plan(const EvictParams& p, cudaStream_t s);
+// (the random draw reads no cache data), into half p.ev_plan_parity of lay.evplan; one warp per
+// CTA, at most `sms` CTAs looping over the (layer, sequence, KV head) items, little shared memory,
+// so that it runs beside the attention kernel.
+cudaError_t launch_plan(const EvictParams& p, int sms, cudaStream_t s);
 // One-time attributes; active[cl] (cl = 0..kEvMaxCluster) = clusters of cl CTAs the device runs at once.
 cudaError_t evict_prepare(int* active);
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);
