@@ -94,6 +94,7 @@ struct ra_ctx {
     cudaEvent_t fork_ev = nullptr, plan_ev = nullptr;
     bool plan_pending = false;
     int parity = 0;
+    bool no_early_once = false;  // the next attention launch follows the whole-stack compaction
     std::vector<int32_t> plan_g, plan_n;
     // profiling
     bool prof = false;
@@ -1179,7 +1180,8 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
     // this step (else it is this layer's compaction) and more than one layer (else it is this
     // layer's previous step).  Kernels let successors start only after their own wait, so
     // everything older than the predecessor has completed.
-    p.early = (n == 0 && ctx->L >= 2) ? 1 : 0;
+    p.early = (n == 0 && ctx->L >= 2 && !ctx->no_early_once) ? 1 : 0;
+    ctx->no_early_once = false;
     {
         // rows read (a new token's from the caller), a new token's row written, q read, out written
         int n_pending = 0;
@@ -1266,6 +1268,48 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
                     ctx->plan_g[k] = pp.trig_g[i];
                     ctx->plan_n[k] = pp.trig_n[i];
                 }
+        }
+    }
+    // The sequences that fire at this step in every layer alike, with every layer's evicted set
+    // computed ahead: all their rounds in one launch, in place, before the first layer.
+    if (plan_usable(ctx)) {
+        EvictParams sp{};
+        sp.lay = ctx->lay;
+        sp.ev_plan_parity = cur;
+        int n = 0;
+        double moved = 0;
+        for (int b = 0; b < ctx->B; ++b) {
+            if (!ctx->active[b]) continue;
+            const int g = ctx->g[b], c = ctx->c[b];
+            if ((g + 1) % ctx->r != 0 || c + 1 - ctx->r <= ctx->K) continue;
+            bool all = true;
+            for (int l = 0; l < ctx->L && all; ++l) {
+                const size_t i = (size_t)l * ctx->B + b, k = (size_t)cur * ctx->L * ctx->B + i;
+                all = ctx->g[i] == g && ctx->c[i] == c && ctx->plan_g[k] == g + 1 && ctx->plan_n[k] == c + 1 - ctx->r;
+            }
+            if (!all) continue;
+            sp.trig[n] = (int16_t)b;
+            sp.trig_c[n] = c;
+            sp.trig_n[n] = c + 1 - ctx->r;
+            sp.trig_g[n] = g + 1;
+            ++n;
+            moved += (double)(ctx->K + ctx->r - 1) * ctx->KVH * ctx->L;
+        }
+        if (n > 0) {
+            sp.n_trig = n;
+            {
+                ProfScope ps(ctx, RA_KERNEL_EVICT, moved * 2.0 * (2 * kRowBytes + 4), s);
+                e = launch_compact_stack(sp, ctx->L, s);
+                ps.done();
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "whole-stack compaction launch");
+            for (int i = 0; i < n; ++i)
+                for (int l = 0; l < ctx->L; ++l) {
+                    const size_t k = (size_t)l * ctx->B + sp.trig[i];
+                    ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written
+                    ctx->nev[k] += 1;
+                }
+            ctx->no_early_once = true;
         }
     }
     for (int l = 0; l < ctx->L; ++l)

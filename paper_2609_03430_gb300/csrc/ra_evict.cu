@@ -1043,6 +1043,138 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
     }
 }
 
+// ----------------------------------------------------------------------------- compact_stack (in place)
+// At the start of a whole-stack step, every layer's round of the sequences that fire, in one
+// launch, from evicted sets computed ahead (plan_kernel): one CTA per (layer, sequence, KV head)
+// compacts the head's region in place.  A survivor moves down by the evicted ordinals below it
+// (at most m <= r rows), so a CTA that copies its rows in ascending chunks never overwrites a row
+// it has not read yet: every store of chunk i lands below chunk i + 1, and every later load reads
+// at or above it.  Chunks of kStkRows rows (K, V and positions) stream through a ring of stages
+// with TMA bulk copies; the survivors' runs go back with bulk stores, positions by plain stores.
+constexpr int kStkThreads = 128;
+constexpr int kStkRows = 64;    // rows per stage: 16 KB of K and 16 KB of V
+constexpr int kStkStages = 3;   // 96 KB of stages: two CTAs per SM
+constexpr size_t kStkSmem = (size_t)kStkStages * 2 * kStkRows * kRowBytes;
+static_assert(kStkStages >= 2 && kStkRows <= kStkThreads, "refills trail by one chunk; a thread per row");
+
+struct StkShared {
+    int32_t ev[kEvCap];                  // the evicted ordinals, ascending
+    int32_t pos[kStkStages][kStkRows + 4];
+    uint64_t bar[kStkStages];
+    int bad;
+};
+
+__global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid_constant__ EvictParams p)
+{
+    extern __shared__ __align__(128) uint8_t stk_dyn[];  // [stage][K rows][V rows]
+    __shared__ StkShared S;
+    constexpr int kStageBytes = 2 * kStkRows * kRowBytes;
+    const DevLayout& L = p.lay;
+    const int tid = threadIdx.x;
+    const int item = blockIdx.x;  // layer-major: (layer, triggered sequence, KV head)
+    const int h = item % L.KVH, t = (item / L.KVH) % p.n_trig, layer = item / (L.KVH * p.n_trig);
+    const int b = p.trig[t], c = p.trig_c[t], N = p.trig_n[t];
+    const int m = N - L.K;
+    pdl_wait();  // the rows were written by the previous step's attention
+    pdl_launch_dependents();
+    if (m < 1 || m > L.r || m > kEvCap || N > c || c > L.Cmax) {  // the host rules this out
+        if (tid == 0) atomicExch(L.err, kDeviceErrPlan);
+        return;
+    }
+    const int reg = L.region[((size_t)layer * L.B + b) * L.KVH + h];
+    const long long row0 = L.gen_row0 + (long long)reg * L.Cmax;
+    int32_t* gpos = L.pos + (size_t)reg * L.Cmax;
+    const int32_t* plan =
+        L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
+    const bool pos_bulk = (L.Cmax & 3) == 0;  // position chunks are 16-byte aligned
+    const int nch = (c + kStkRows - 1) / kStkRows;
+    auto issue = [&](int i) {  // chunk i into stage i % kStkStages (thread 0)
+        const int s = i % kStkStages, a = i * kStkRows, n = min(kStkRows, c - a);
+        uint8_t* st = stk_dyn + (size_t)s * kStageBytes;
+        const uint32_t pbytes = pos_bulk ? (uint32_t)min((n + 3) & ~3, L.Cmax - a) * 4u : 0u;
+        mbar_arrive_expect_tx(&S.bar[s], 2u * (uint32_t)n * kRowBytes + pbytes);
+        bulk_load(st, L.kpool + (row0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &S.bar[s]);
+        bulk_load(st + kStkRows * kRowBytes, L.vpool + (row0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &S.bar[s]);
+        if (pbytes) bulk_load(S.pos[s], gpos + a, pbytes, &S.bar[s]);
+    };
+    int issued = 0;  // thread 0's count of chunks whose copies are issued
+    if (tid == 0) {
+        S.bad = 0;
+        for (int s = 0; s < kStkStages; ++s) mbar_init(&S.bar[s], 1);
+        fence_mbar_init();
+        issued = min(kStkStages, nch);
+        for (int i = 0; i < issued; ++i) issue(i);
+    }
+    // the plan: m ordinals, ascending, below N
+    const int n_plan = __ldcg(plan);
+    for (int i = tid; i < m; i += kStkThreads) S.ev[i] = __ldcg(plan + 1 + i);
+    __syncthreads();
+    bool bad = n_plan != m;
+    for (int i = tid; i < m && !bad; i += kStkThreads)
+        bad = S.ev[i] < 0 || S.ev[i] >= N || (i + 1 < m && S.ev[i] >= S.ev[i + 1]);
+    if (bad) S.bad = 1;
+    __syncthreads();
+    if (S.bad) {  // a bad plan moves nothing: wait (bounded) for the copies issued, and leave
+        if (tid == 0) {
+            atomicExch(L.err, kDeviceErrPlan);
+            for (int q = 0; q < issued; ++q)
+                (void)mbar_wait_bounded(&S.bar[q % kStkStages], (uint32_t)((q / kStkStages) & 1), kEvWaitLimitNs);
+        }
+        return;
+    }
+    auto ev_below = [&](int j) {  // evicted ordinals below j
+        int lo = 0, hi = m;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (S.ev[mid] < j) lo = mid + 1; else hi = mid;
+        }
+        return lo;
+    };
+    for (int i = 0; i < nch; ++i) {  // every chunk's copies are issued by the time it is reached
+        const int s = i % kStkStages, a = i * kStkRows, n = min(kStkRows, c - a);
+        if (tid == 0 && !mbar_wait_bounded(&S.bar[s], (uint32_t)((i / kStkStages) & 1), kEvWaitLimitNs)) {
+            atomicExch(L.err, kDeviceErrTimeout);
+            for (int q = i + 1; q < issued; ++q)  // let the copies already issued land (bounded)
+                (void)mbar_wait_bounded(&S.bar[q % kStkStages], (uint32_t)((q / kStkStages) & 1), kEvWaitLimitNs);
+            S.bad = 2;
+        }
+        if (!pos_bulk && tid < n) S.pos[s][tid] = __ldcg(gpos + a + tid);  // (all read before any is written)
+        __syncthreads();
+        if (S.bad) break;
+        if (tid < n) {  // positions of the chunk's survivors
+            const int j = a + tid, e = ev_below(j);
+            if (e == m || S.ev[e] != j) gpos[j - e] = S.pos[s][tid];
+        }
+        if (tid == 0) {  // the runs of survivors, each to its place below
+            const uint8_t* st = stk_dyn + (size_t)s * kStageBytes;
+            int e = ev_below(a);
+            for (int q = a; q < a + n;) {
+                const int nx = e < m ? S.ev[e] : INT_MAX;
+                const int v = min(a + n, nx);
+                if (v > q) {
+                    const long long drow = row0 + (q - e);
+                    bulk_store(L.kpool + drow * kHeadDim, st + (q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
+                    bulk_store(L.vpool + drow * kHeadDim, st + (kStkRows + q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
+                }
+                if (nx < a + n) {
+                    q = nx + 1;
+                    ++e;
+                } else {
+                    q = v;
+                }
+            }
+            bulk_commit();
+        }
+        __syncthreads();  // the stage's positions are read
+        if (tid == 0 && i >= 1 && issued < nch) {  // chunk i + 2 into chunk i - 1's stage once its stores read it
+            asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+            issue(issued);
+            ++issued;
+        }
+    }
+    if (tid == 0) bulk_wait_all();
+}
+
 // ----------------------------------------------------------------------------- timeout probe
 // The failure path of every bounded wait, run on purpose: one arrival with 16 bytes of
 // transfer expected, and no copy ever issued, so the barrier's phase cannot complete; the
@@ -1219,6 +1351,18 @@ cudaError_t launch_plan(const EvictParams& p, int sms, cudaStream_t s)
     const int items = p.lay.L * p.n_trig * p.lay.KVH;
     plan_kernel<<<(unsigned)std::min(items, std::max(sms, 1)), 32, 0, s>>>(p);
     return cudaGetLastError();
+}
+
+cudaError_t launch_compact_stack(const EvictParams& p, int layers, cudaStream_t s)
+{
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(compact_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStkSmem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    return launch_pdl(compact_stack_kernel, dim3((unsigned)(layers * p.n_trig * p.lay.KVH)), dim3(kStkThreads), kStkSmem,
+                      s, p);
 }
 
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s)

@@ -176,6 +176,10 @@ cudaError_t launch_evict(const EvictParams& p, int cluster, cudaStream_t s);
 // CTA, at most `sms` CTAs looping over the (layer, sequence, KV head) items, little shared memory,
 // so that it runs beside the attention kernel.
 cudaError_t launch_plan(const EvictParams& p, int sms, cudaStream_t s);
+// Every layer's round of the triggered sequences (layers 0 .. layers - 1, counters alike in every
+// layer), in place, from the evicted sets in half p.ev_plan_parity of lay.evplan: one CTA per
+// (layer, sequence, KV head).
+cudaError_t launch_compact_stack(const EvictParams& p, int layers, cudaStream_t s);
 // One-time attributes; active[cl] (cl = 0..kEvMaxCluster) = clusters of cl CTAs the device runs at once.
 cudaError_t evict_prepare(int* active);
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);
