@@ -1046,32 +1046,36 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
 // ----------------------------------------------------------------------------- compact_stack (in place)
 // At the start of a whole-stack step, every layer's round of the sequences that fire, in one
 // launch, from evicted sets computed ahead (plan_kernel): one CTA per (layer, sequence, KV head)
-// compacts the head's region in place.  A survivor moves down by the evicted ordinals below it
-// (at most m <= r rows), so a CTA that copies its rows in ascending chunks never overwrites a row
-// it has not read yet: every store of chunk i lands below chunk i + 1, and every later load reads
-// at or above it.  Chunks of kStkRows rows (K, V and positions) stream through a ring of stages
-// with TMA bulk copies; the survivors' runs go back with bulk stores, positions by plain stores.
+// and array (K with the positions, or V) compacts the head's rows of that array in place.  A
+// survivor moves down by the evicted ordinals below it (at most m <= r rows), so a CTA that copies
+// its rows in ascending chunks never overwrites a row it has not read yet: every store of chunk i
+// lands below chunk i + 1, and every later load reads at or above it (and the two arrays are
+// separate, so their CTAs are independent).  Chunks of kStkRows rows stream through a ring of
+// stages with TMA bulk copies; the survivors' runs go back with bulk stores, positions by plain
+// stores.
 constexpr int kStkThreads = 128;
-constexpr int kStkRows = 64;    // rows per stage: 16 KB of K and 16 KB of V
+constexpr int kStkRows = 128;   // rows per stage: 32 KB of K or V
 constexpr int kStkStages = 3;   // 96 KB of stages: two CTAs per SM
-constexpr size_t kStkSmem = (size_t)kStkStages * 2 * kStkRows * kRowBytes;
+constexpr size_t kStkSmem = (size_t)kStkStages * kStkRows * kRowBytes;
 static_assert(kStkStages >= 2 && kStkRows <= kStkThreads, "refills trail by one chunk; a thread per row");
+static_assert(((kStkRows + 4) * 4) % 16 == 0, "every stage's positions start 16-byte aligned");
 
 struct StkShared {
     int32_t ev[kEvCap];                  // the evicted ordinals, ascending
-    int32_t pos[kStkStages][kStkRows + 4];
+    __align__(16) int32_t pos[kStkStages][kStkRows + 4];  // (bulk copy destinations: 16-byte aligned)
     uint64_t bar[kStkStages];
     int bad;
 };
 
 __global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid_constant__ EvictParams p)
 {
-    extern __shared__ __align__(128) uint8_t stk_dyn[];  // [stage][K rows][V rows]
-    __shared__ StkShared S;
-    constexpr int kStageBytes = 2 * kStkRows * kRowBytes;
+    extern __shared__ __align__(128) uint8_t stk_dyn[];  // [stage][rows of K or V]
+    __shared__ __align__(16) StkShared S;
+    constexpr int kStageBytes = kStkRows * kRowBytes;
     const DevLayout& L = p.lay;
     const int tid = threadIdx.x;
-    const int item = blockIdx.x;  // layer-major: (layer, triggered sequence, KV head)
+    const int item = blockIdx.x >> 1, part = blockIdx.x & 1;  // layer-major (layer, sequence, KV head); 0: K, 1: V
+    uint16_t* pool = part ? L.vpool : L.kpool;
     const int h = item % L.KVH, t = (item / L.KVH) % p.n_trig, layer = item / (L.KVH * p.n_trig);
     const int b = p.trig[t], c = p.trig_c[t], N = p.trig_n[t];
     const int m = N - L.K;
@@ -1086,15 +1090,15 @@ __global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid
     int32_t* gpos = L.pos + (size_t)reg * L.Cmax;
     const int32_t* plan =
         L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
-    const bool pos_bulk = (L.Cmax & 3) == 0;  // position chunks are 16-byte aligned
+    const bool with_pos = part == 0;
+    const bool pos_bulk = with_pos && (L.Cmax & 3) == 0;  // position chunks are 16-byte aligned
     const int nch = (c + kStkRows - 1) / kStkRows;
     auto issue = [&](int i) {  // chunk i into stage i % kStkStages (thread 0)
         const int s = i % kStkStages, a = i * kStkRows, n = min(kStkRows, c - a);
         uint8_t* st = stk_dyn + (size_t)s * kStageBytes;
         const uint32_t pbytes = pos_bulk ? (uint32_t)min((n + 3) & ~3, L.Cmax - a) * 4u : 0u;
-        mbar_arrive_expect_tx(&S.bar[s], 2u * (uint32_t)n * kRowBytes + pbytes);
-        bulk_load(st, L.kpool + (row0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &S.bar[s]);
-        bulk_load(st + kStkRows * kRowBytes, L.vpool + (row0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &S.bar[s]);
+        mbar_arrive_expect_tx(&S.bar[s], (uint32_t)n * kRowBytes + pbytes);
+        bulk_load(st, pool + (row0 + a) * kHeadDim, (uint32_t)n * kRowBytes, &S.bar[s]);
         if (pbytes) bulk_load(S.pos[s], gpos + a, pbytes, &S.bar[s]);
     };
     int issued = 0;  // thread 0's count of chunks whose copies are issued
@@ -1138,10 +1142,10 @@ __global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid
                 (void)mbar_wait_bounded(&S.bar[q % kStkStages], (uint32_t)((q / kStkStages) & 1), kEvWaitLimitNs);
             S.bad = 2;
         }
-        if (!pos_bulk && tid < n) S.pos[s][tid] = __ldcg(gpos + a + tid);  // (all read before any is written)
+        if (with_pos && !pos_bulk && tid < n) S.pos[s][tid] = __ldcg(gpos + a + tid);  // (all read before any is written)
         __syncthreads();
         if (S.bad) break;
-        if (tid < n) {  // positions of the chunk's survivors
+        if (with_pos && tid < n) {  // positions of the chunk's survivors
             const int j = a + tid, e = ev_below(j);
             if (e == m || S.ev[e] != j) gpos[j - e] = S.pos[s][tid];
         }
@@ -1153,8 +1157,7 @@ __global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid
                 const int v = min(a + n, nx);
                 if (v > q) {
                     const long long drow = row0 + (q - e);
-                    bulk_store(L.kpool + drow * kHeadDim, st + (q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
-                    bulk_store(L.vpool + drow * kHeadDim, st + (kStkRows + q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
+                    bulk_store(pool + drow * kHeadDim, st + (q - a) * kRowBytes, (uint32_t)(v - q) * kRowBytes);
                 }
                 if (nx < a + n) {
                     q = nx + 1;
@@ -1361,8 +1364,8 @@ cudaError_t launch_compact_stack(const EvictParams& p, int layers, cudaStream_t 
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    return launch_pdl(compact_stack_kernel, dim3((unsigned)(layers * p.n_trig * p.lay.KVH)), dim3(kStkThreads), kStkSmem,
-                      s, p);
+    return launch_pdl(compact_stack_kernel, dim3((unsigned)(2 * layers * p.n_trig * p.lay.KVH)), dim3(kStkThreads),
+                      kStkSmem, s, p);
 }
 
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s)
