@@ -76,7 +76,8 @@ enum ra_kernel_kind {
     RA_KERNEL_SCORE_SUM = 5,   /* scored comparator: window attention summed per candidate */
     RA_KERNEL_EVICT = 6,       /* selection and order-preserving compaction in one launch */
     RA_KERNEL_PLAN = 7,        /* evicted sets of the next step, computed beside the current one */
-    RA_KERNEL_KINDS = 8
+    RA_KERNEL_STACK = 8,       /* every layer's in-place compaction of the sequences firing at a whole-stack step */
+    RA_KERNEL_KINDS = 9
 };
 
 /*

@@ -26,8 +26,8 @@ RA_ERR_DEVICE_TIMEOUT = -5
 RA_ERR_UNSUPPORTED = -6
 RA_MAX_BATCH = 512
 (RA_KERNEL_APPEND, RA_KERNEL_SELECT, RA_KERNEL_COMPACT, RA_KERNEL_ATTN, RA_KERNEL_SCORE_STATS, RA_KERNEL_SCORE_SUM,
- RA_KERNEL_EVICT, RA_KERNEL_PLAN) = range(8)
-KERNEL_NAMES = ["append", "select", "compact", "attn", "score_stats", "score_sum", "evict", "plan"]
+ RA_KERNEL_EVICT, RA_KERNEL_PLAN, RA_KERNEL_STACK) = range(9)
+KERNEL_NAMES = ["append", "select", "compact", "attn", "score_stats", "score_sum", "evict", "plan", "stack"]
 RA_EVICT_AUTO, RA_EVICT_TWO_KERNELS, RA_EVICT_EXACT = 0, 1, 256
 
 # Exported C symbols and their ctypes signatures (kept in the order of include/ra.h).

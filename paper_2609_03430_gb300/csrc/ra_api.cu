@@ -1298,7 +1298,7 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
         if (n > 0) {
             sp.n_trig = n;
             {
-                ProfScope ps(ctx, RA_KERNEL_EVICT, moved * 2.0 * (2 * kRowBytes + 4), s);
+                ProfScope ps(ctx, RA_KERNEL_STACK, moved * 2.0 * (2 * kRowBytes + 4), s);
                 e = launch_compact_stack(sp, ctx->L, s);
                 ps.done();
             }

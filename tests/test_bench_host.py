@@ -157,6 +157,14 @@ def test_eviction_roofline_prices_the_copy_kernel_and_the_round():
     assert r2["round"]["us_per_round"] == pytest.approx(12.0)
     assert r2["holefill_select"]["achieved"] == pytest.approx(2e6 / 5e-6 / 1e9)
     assert r2["holefill_select"]["us_per_round"] == pytest.approx(5.0)
+    # the whole-stack compaction, when present, is the one priced; the others are listed beside it
+    kern3 = {"stack": _kern(600.0, 4.3e9, 1), "evict": _kern(12.0, 68e6, 10), "plan": _kern(100.0, 0.0, 2)}
+    r3 = bench.eviction_roofline(kern3, 74, peaks, "measured")
+    assert r3["kernel"].startswith("compact_stack_kernel") and r3["launches"] == 1
+    assert r3["achieved"] == pytest.approx(4.3e9 / 600e-6 / 1e9)
+    assert r3["also"]["evict"]["achieved"] == pytest.approx(68e6 / 12e-6 / 1e9)
+    assert r3["round"]["us_per_round"] == pytest.approx(720.0 / 74)  # the plan is not in the round
+    assert r3["plan"]["launches"] == 2 and "target" in r3
     # no eviction in the evented pass: nothing to report
     assert bench.eviction_roofline({"attn": kern["attn"]}, 0, peaks, "measured") is None
 
