@@ -485,10 +485,19 @@ def eviction_window(clean, evicting):
     extra_ms = sum(ms - by * attn_ms_per_byte for (ms, by, _, _) in evicting)
     rounds = sum(e[2] for e in evicting)
     ebytes = sum(e[3] for e in evicting)
-    if rounds <= 0 or extra_ms <= 0:
+    if rounds <= 0:
         return None
-    return {"steps": len(evicting), "rounds": rounds, "us_per_round": 1000.0 * extra_ms / rounds,
-            "bytes_per_round": ebytes / rounds, "GBps": ebytes / (extra_ms * 1e-3) / 1e9}
+    # the prediction's own noise: the clean steps' spread of time per byte, over the evicting
+    # steps' attention bytes; a difference within twice that is not resolved
+    rates = [c[0] / c[2] for c in clean if c[2] > 0]
+    mean = sum(rates) / len(rates)
+    sd = (sum((x - mean) ** 2 for x in rates) / len(rates)) ** 0.5
+    noise_ms = sd * sum(by * by for (_, by, _, _) in evicting) ** 0.5
+    out = {"steps": len(evicting), "rounds": rounds, "bytes_per_round": ebytes / rounds,
+           "noise_us_per_round": 1000.0 * noise_ms / rounds}
+    if extra_ms <= 2.0 * noise_ms:
+        return dict(out, resolved=False, us_per_round_at_most=1000.0 * (max(extra_ms, 0.0) + 2.0 * noise_ms) / rounds)
+    return dict(out, resolved=True, us_per_round=1000.0 * extra_ms / rounds, GBps=ebytes / (extra_ms * 1e-3) / 1e9)
 
 
 def attention_roofline(a, clean, steps, layers, peaks, peak_src, traffic):
@@ -574,7 +583,7 @@ def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None
                        "what": "plan_kernel: the next step's evicted sets, on a side stream beside the attention "
                                "(not on the critical path; not in the round figures)"}
     if windowed is not None:
-        out["windowed"] = dict(windowed, frac=windowed["GBps"] / peaks["hbm_gbs"],
+        out["windowed"] = dict(windowed, frac=windowed["GBps"] / peaks["hbm_gbs"] if windowed.get("GBps") else None,
                                what="step-boundary pass: (device time of the steps in which sequences evict - their "
                                     "attention bytes at the eviction-free steps' attention bandwidth) per (sequence, "
                                     "layer) round; the eviction's cost on the critical path, overlap included")

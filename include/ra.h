@@ -327,7 +327,15 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
  * One decode step of the whole layer stack: ra_decode_layer for l = 0..layers-1,
  * with q_all [layers][batch][q_heads][d], k_all / v_all [layers][batch][kv_heads][d],
  * out_all [layers][batch][q_heads][d].  Capacity is checked for every layer first,
- * so a step that fails changes nothing.
+ * so a step that fails changes nothing.  Same result as the per-layer calls, by a
+ * faster route: the keys of the random policy and its variants (not the scored
+ * one) need no cache data beyond positions, so during each step a kernel on a
+ * stream of the library's own (forked from and joined to `stream` by events)
+ * computes the next step's evicted sets in every layer, and at that step one
+ * launch compacts every layer of the sequences that fire (ordered or order-free,
+ * in place) before the first layer runs.  Sets computed ahead are used only
+ * where the counters they were computed from still hold; elsewhere the layers
+ * select as ra_decode_layer does.
  */
 int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, const uint16_t* v_all,
                    uint16_t* out_all, float scale, void* stream);

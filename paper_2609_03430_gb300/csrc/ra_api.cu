@@ -95,6 +95,7 @@ struct ra_ctx {
     bool plan_pending = false;
     int parity = 0;
     bool no_early_once = false;  // the next attention launch follows the whole-stack compaction
+    std::vector<uint8_t> stack_done;  // [B] sequences whose token this step's order-free fill wrote
     std::vector<int32_t> plan_g, plan_n;
     // profiling
     bool prof = false;
@@ -405,13 +406,22 @@ double plan_scoring(ra_ctx* ctx, EvictParams* p, int pass)
 int run_eviction_launches(ra_ctx* ctx, EvictParams& p, double moved, cudaStream_t s, bool compact_in_attention,
                           int score_early);
 
-// Evicted sets can be computed ahead for the one-launch eviction of the policies whose keys read
-// no cache data (random, shared, recency) with ordered compaction outside the attention pass.
+// Evicted sets can be computed ahead for the policies whose keys need no scores (random, shared,
+// recency, block), with ordered compaction outside the attention pass (the one-launch kernels) or
+// order-free slots.  Keys that follow positions (order-free slots, block draws) are read from the
+// cache, so their plans also need r >= 2: the next step's candidates then exclude the slot the
+// current step appends.
+bool keys_read_positions(const ra_ctx* ctx)
+{
+    return ctx->compaction == RA_COMPACT_HOLEFILL || ctx->policy == RA_POLICY_BLOCK;
+}
+
 bool plan_usable(const ra_ctx* ctx)
 {
-    return ctx->compaction == RA_COMPACT_ORDERED && ctx->r <= kEvMaxEvicted &&
-           (ctx->evict_mode & ~RA_EVICT_EXACT) != RA_EVICT_TWO_KERNELS && ctx->evict_active[1] > 0 &&
-           (ctx->policy == RA_POLICY_RANDOM || ctx->policy == RA_POLICY_SHARED || ctx->policy == RA_POLICY_RECENCY);
+    if (ctx->r > kEvMaxEvicted || (ctx->evict_mode & ~RA_EVICT_EXACT) == RA_EVICT_TWO_KERNELS) return false;
+    if (ctx->policy == RA_POLICY_SNAPKV || (keys_read_positions(ctx) && ctx->r < 2)) return false;
+    if (ctx->compaction == RA_COMPACT_HOLEFILL) return true;
+    return ctx->compaction == RA_COMPACT_ORDERED && ctx->evict_active[1] > 0;
 }
 
 // One eviction round of the triggered sequences in p: [score passes,] select, compact (unless
@@ -566,6 +576,7 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->c.assign((size_t)layers * batch, 0);
     ctx->nev.assign((size_t)layers * batch, 0);
     ctx->active.assign(batch, 1);
+    ctx->stack_done.assign(batch, 0);
     ctx->score_n.assign((size_t)layers * batch, 0);
     *out = ctx;
     return RA_OK;
@@ -756,8 +767,10 @@ int ra_restore(ra_ctx* ctx, int layer, const int32_t* g_host, const int32_t* c_h
     cudaError_t e;
     if (maxc > 0 && (e = launch_restore(p, s)) != cudaSuccess) return cuda_fail(ctx, e, "restore launch");
     for (int b = 0; b < ctx->B; ++b) {
-        ctx->g[(size_t)layer * ctx->B + b] = g_host[b];
-        ctx->c[(size_t)layer * ctx->B + b] = c_host[b];
+        const size_t i = (size_t)layer * ctx->B + b;
+        ctx->g[i] = g_host[b];
+        ctx->c[i] = c_host[b];
+        ctx->plan_g[i] = ctx->plan_g[(size_t)ctx->L * ctx->B + i] = -1;  // positions replaced
     }
     return RA_OK;
 }
@@ -795,6 +808,7 @@ int ra_set_compaction(ra_ctx* ctx, int mode)
     if (mode == RA_COMPACT_HOLEFILL && ctx->policy == RA_POLICY_SNAPKV)
         return fail(ctx, RA_ERR_UNSUPPORTED, "the scored policy needs ordered compaction");
     ctx->compaction = mode;
+    std::fill(ctx->plan_g.begin(), ctx->plan_g.end(), -1);  // keys per ordinal or per position
     return RA_OK;
 }
 
@@ -1115,6 +1129,10 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
         if (!ctx->active[b]) continue;
+        if (!ctx->stack_done.empty() && ctx->stack_done[b]) {  // evicted and appended by this step's fill
+            appended[b] = 1;
+            continue;
+        }
         const int g1 = ctx->g[base + b] + 1, c1 = ctx->c[base + b] + 1;
         if (g1 % ctx->r == 0 && c1 - ctx->r > ctx->K) {
             ep.trig[n] = (int16_t)b;
@@ -1233,13 +1251,17 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
         EvictParams pp{};
         pp.lay = ctx->lay;
         pp.policy = ctx->policy;
+        pp.block = ctx->block;
+        pp.holefill = ctx->compaction == RA_COMPACT_HOLEFILL;
         pp.ev_exact = (ctx->evict_mode & RA_EVICT_EXACT) ? 1 : 0;
         pp.ev_plan_parity = nxt;
+        const bool read_pos = keys_read_positions(ctx);
         int n = 0;
         for (int b = 0; b < ctx->B; ++b) {
             if (!ctx->active[b]) continue;
             const int g1 = ctx->g[b] + 1, c1 = ctx->c[b] + 1;
             const bool fires = g1 % ctx->r == 0 && c1 - ctx->r > ctx->K;
+            if (fires && read_pos) continue;  // this step rewrites the positions the keys would read
             const int g2 = g1 + 1, c2 = (fires ? ctx->K + ctx->r : c1) + 1;
             if (g2 % ctx->r == 0 && c2 - ctx->r > ctx->K && c2 - ctx->r <= ctx->K + ctx->r) {
                 pp.trig[n] = (int16_t)b;
@@ -1271,11 +1293,19 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
         }
     }
     // The sequences that fire at this step in every layer alike, with every layer's evicted set
-    // computed ahead: all their rounds in one launch, in place, before the first layer.
+    // computed ahead: all their rounds in one launch, in place, before the first layer.  Ordered:
+    // the survivors move down and the layers then append the token as usual.  Order-free: the
+    // evicted slots are refilled from the newest rows, the step's token included, so the layers
+    // attend with the token already cached.
+    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
     if (plan_usable(ctx)) {
+        const bool fill = ctx->compaction == RA_COMPACT_HOLEFILL;
         EvictParams sp{};
         sp.lay = ctx->lay;
         sp.ev_plan_parity = cur;
+        sp.holefill = fill ? 1 : 0;
+        sp.k_new = k_all;
+        sp.v_new = v_all;
         int n = 0;
         double moved = 0;
         for (int b = 0; b < ctx->B; ++b) {
@@ -1293,29 +1323,39 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
             sp.trig_n[n] = c + 1 - ctx->r;
             sp.trig_g[n] = g + 1;
             ++n;
-            moved += (double)(ctx->K + ctx->r - 1) * ctx->KVH * ctx->L;
+            // rows moved per head: the survivors below the token (ordered), the m refills (order-free)
+            moved += (double)(fill ? c + 1 - ctx->r - ctx->K : ctx->K + ctx->r - 1) * ctx->KVH * ctx->L;
         }
         if (n > 0) {
             sp.n_trig = n;
             {
                 ProfScope ps(ctx, RA_KERNEL_STACK, moved * 2.0 * (2 * kRowBytes + 4), s);
-                e = launch_compact_stack(sp, ctx->L, s);
+                e = fill ? launch_fill_stack(sp, ctx->L, s) : launch_compact_stack(sp, ctx->L, s);
                 ps.done();
             }
             if (e != cudaSuccess) return cuda_fail(ctx, e, "whole-stack compaction launch");
-            for (int i = 0; i < n; ++i)
+            for (int i = 0; i < n; ++i) {
                 for (int l = 0; l < ctx->L; ++l) {
                     const size_t k = (size_t)l * ctx->B + sp.trig[i];
-                    ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written
+                    if (fill) {  // K + r rows, the token's among them
+                        ctx->c[k] = ctx->K + ctx->r;
+                        ctx->g[k] += 1;
+                    } else {
+                        ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written
+                    }
                     ctx->nev[k] += 1;
                 }
+                if (fill) ctx->stack_done[sp.trig[i]] = 1;
+            }
             ctx->no_early_once = true;
         }
     }
     for (int l = 0; l < ctx->L; ++l)
         if ((rc = decode_layer_impl(ctx, l, q_all + l * qs, k_all + l * ks, v_all + l * ks, out_all + l * qs, scale,
                                     stream, cur)) != RA_OK)
-            return rc;
+            break;
+    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
+    if (rc != RA_OK) return rc;
     ctx->parity = nxt;
     return RA_OK;
 }

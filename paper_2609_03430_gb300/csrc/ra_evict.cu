@@ -25,6 +25,12 @@
 //                   (Appendix F keeps each keep-set in time order and gathers
 //                   the cache into it).  Out of place, so CTAs never wait on
 //                   each other; the old region becomes the spare.
+//   plan_kernel     the next step's evicted sets in every layer, beside the
+//                   current step (the draw needs no cache data but positions).
+//   compact_stack_kernel / fill_stack_kernel
+//                   at a whole-stack step, every layer's round of the firing
+//                   sequences in one launch, in place, from those sets:
+//                   order-preserving, or refilling the evicted slots.
 #include <cuda_runtime.h>
 #include <limits.h>
 
@@ -879,7 +885,9 @@ __global__ void __launch_bounds__(kEvThreads, 1) evict_kernel(const __grid_const
 
 // ----------------------------------------------------------------------------- plan (evicted sets ahead)
 // The random draw reads no cache data: a candidate's key depends only on (ordinal, step, layer,
-// head), so the evicted set of a firing step is known as soon as the counters are.  plan_kernel
+// head), so the evicted set of a firing step is known as soon as the counters are.  (Keys that
+// follow positions -- order-free slots, block draws -- read the candidates' positions, which no
+// kernel of the step before rewrites for a sequence that fires only at the next one.)  plan_kernel
 // computes it ahead, beside the attention of the step before: one warp per CTA and about one CTA
 // per SM, each looping over (layer, sequence, KV head) items, so that it takes a sliver of each
 // SM's issue slots (7 KB of shared memory: it fits beside an attention CTA).  Per item, the
@@ -895,11 +903,20 @@ struct PlanShared {
     uint32_t cnt, nev;
 };
 
-__device__ __forceinline__ uint32_t plan_key(const EvictParams& p, int layer, uint32_t id, int N, int g, int j)
+// The key of candidate j, by the rules of select_kernel: per ordinal, or per position (pos: the
+// head's positions) for order-free slots and block draws.
+__device__ __forceinline__ uint32_t plan_key(const EvictParams& p, int layer, uint32_t id, int N, int g, int j,
+                                             const int32_t* pos)
 {
+    const uint32_t k0 = (uint32_t)p.lay.seed, k1 = (uint32_t)(p.lay.seed >> 32);
+    if (p.policy == RA_POLICY_BLOCK)
+        return philox4x32_10_w0((uint32_t)(__ldcg(pos + j) / p.block), (uint32_t)g, (uint32_t)layer, id, k0, k1);
+    if (p.holefill) {
+        const uint32_t pj = (uint32_t)__ldcg(pos + j);
+        return p.policy == RA_POLICY_RECENCY ? 0xFFFFFFFFu - pj : philox4x32_10_w0(pj, (uint32_t)g, (uint32_t)layer, id, k0, k1);
+    }
     if (p.policy == RA_POLICY_RECENCY) return (uint32_t)(N - 1 - j);
-    return philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)layer, id, (uint32_t)p.lay.seed,
-                            (uint32_t)(p.lay.seed >> 32));
+    return philox4x32_10_w0((uint32_t)j, (uint32_t)g, (uint32_t)layer, id, k0, k1);
 }
 
 __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictParams p)
@@ -920,6 +937,7 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
         }
         const uint32_t id = key_stream(p.trig_admit[t],
                                        p.policy == RA_POLICY_SHARED ? (uint32_t)(b * L.KVH) : (uint32_t)(b * L.KVH + h));
+        const int32_t* pos = L.pos + (size_t)L.region[((size_t)layer * L.B + b) * L.KVH + h] * L.Cmax;
         const bool cut = (p.policy == RA_POLICY_RANDOM || p.policy == RA_POLICY_SHARED) && !p.ev_exact;
         bool done = false;
         if (cut) {
@@ -929,7 +947,7 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
             for (int j0 = lane; j0 < N; j0 += 4 * 32) {  // four independent Philox chains at a time
                 uint32_t kq[4];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) kq[q] = plan_key(p, layer, id, N, g, j0 + q * 32);
+                for (int q = 0; q < 4; ++q) kq[q] = plan_key(p, layer, id, N, g, min(j0 + q * 32, N - 1), pos);
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     const int j = j0 + q * 32;
@@ -982,7 +1000,7 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
             for (int i = lane; i < 256; i += 32) S.hist[i] = 0;
             __syncwarp();
             for (int j = lane; j < N; j += 32) {
-                const uint32_t key = plan_key(p, layer, id, N, g, j);
+                const uint32_t key = plan_key(p, layer, id, N, g, j, pos);
                 if ((key & mask) == prefix) atomicAdd(&S.hist[(key >> shift) & 255u], 1u);
             }
             __syncwarp();
@@ -1029,7 +1047,7 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
         uint32_t base_ev = 0, base_tie = 0;
         for (int c0 = 0; c0 < N; c0 += 32) {
             const int j = c0 + lane;
-            const uint32_t key = j < N ? plan_key(p, layer, id, N, g, j) : 0u;
+            const uint32_t key = j < N ? plan_key(p, layer, id, N, g, j, pos) : 0u;
             const bool eq = j < N && key == T, gt = j < N && key > T;
             const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
             const bool ev = gt || (eq && base_tie + __popc(eqb & ((1u << lane) - 1u)) >= tie_from);
@@ -1176,6 +1194,80 @@ __global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid
         }
     }
     if (tid == 0) bulk_wait_all();
+}
+
+// ----------------------------------------------------------------------------- fill_stack (order-free, in place)
+// The order-free counterpart of compact_stack_kernel: at the start of a whole-stack step, every
+// layer's round of the sequences that fire, in one launch, from evicted sets computed ahead.  One
+// CTA per (layer, sequence, KV head) refills evicted slot e_i with the row of slot top - m + i, as
+// select_kernel does within a layer: top counts the step's token, the newest of those rows, which
+// comes from the caller's rows of that layer ([layers][batch][kv_heads][d]) with its position.
+// Those m <= r slots are all buffer slots, so sources and destinations never overlap.
+constexpr int kFillThreads = 256;
+
+__global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_constant__ EvictParams p)
+{
+    __shared__ int32_t ev[kEvCap];
+    __shared__ int bad;
+    const DevLayout& L = p.lay;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int item = blockIdx.x;  // layer-major (layer, sequence, KV head)
+    const int h = item % L.KVH, t = (item / L.KVH) % p.n_trig, layer = item / (L.KVH * p.n_trig);
+    const int b = p.trig[t], c = p.trig_c[t], N = p.trig_n[t], g = p.trig_g[t];
+    const int m = N - L.K;
+    pdl_wait();  // the buffer rows were written by earlier steps' attention
+    pdl_launch_dependents();
+    if (m < 1 || m > L.r || m > kEvCap || N > c || c + 1 > L.Cmax) {  // the host rules this out
+        if (tid == 0) atomicExch(L.err, kDeviceErrPlan);
+        return;
+    }
+    const int32_t* plan =
+        L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
+    if (tid == 0) bad = __ldcg(plan) != m;
+    for (int i = tid; i < m; i += kFillThreads) ev[i] = __ldcg(plan + 1 + i);
+    __syncthreads();
+    bool wrong = false;  // the plan: m ordinals, ascending, below N
+    for (int i = tid; i < m; i += kFillThreads) wrong = wrong || ev[i] < 0 || ev[i] >= N || (i + 1 < m && ev[i] >= ev[i + 1]);
+    if (wrong) bad = 1;
+    __syncthreads();
+    if (bad) {  // a bad plan moves nothing
+        if (tid == 0) atomicExch(L.err, kDeviceErrPlan);
+        return;
+    }
+    const int reg = L.region[((size_t)layer * L.B + b) * L.KVH + h];
+    const long long row0 = L.gen_row0 + (long long)reg * L.Cmax;
+    int32_t* gpos = L.pos + (size_t)reg * L.Cmax;
+    const size_t tok = (((size_t)layer * L.B + b) * L.KVH + h) * kHeadDim;
+    const int top = c + 1, part = lane & 15;
+    uint16_t* pool = lane < 16 ? L.kpool : L.vpool;  // lanes 0-15 move K, 16-31 V, 16 bytes each
+    constexpr int kWarps = kFillThreads / 32, kBatch = 8;  // rows a warp has in flight
+    for (int i0 = warp; i0 < m; i0 += kWarps * kBatch) {
+        uint4 v[kBatch];
+        int32_t pv[kBatch];
+        int to[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {  // every load of the batch first ...
+            const int i = i0 + u * kWarps;
+            to[u] = -1;
+            if (i < m) {
+                const int from = top - m + i;
+                to[u] = ev[i];
+                if (from == c) {  // the step's token
+                    v[u] = reinterpret_cast<const uint4*>((lane < 16 ? p.k_new : p.v_new) + tok)[part];
+                    pv[u] = L.seq_lp[b] + g - 1;
+                } else {
+                    v[u] = reinterpret_cast<const uint4*>(pool + (row0 + from) * kHeadDim)[part];
+                    pv[u] = gpos[from];
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {  // ... then the stores
+            if (to[u] < 0) continue;
+            reinterpret_cast<uint4*>(pool + (row0 + to[u]) * kHeadDim)[part] = v[u];
+            if (lane == 0) gpos[to[u]] = pv[u];
+        }
+    }
 }
 
 // ----------------------------------------------------------------------------- timeout probe
@@ -1366,6 +1458,11 @@ cudaError_t launch_compact_stack(const EvictParams& p, int layers, cudaStream_t 
     }
     return launch_pdl(compact_stack_kernel, dim3((unsigned)(2 * layers * p.n_trig * p.lay.KVH)), dim3(kStkThreads),
                       kStkSmem, s, p);
+}
+
+cudaError_t launch_fill_stack(const EvictParams& p, int layers, cudaStream_t s)
+{
+    return launch_pdl(fill_stack_kernel, dim3((unsigned)(layers * p.n_trig * p.lay.KVH)), dim3(kFillThreads), 0, s, p);
 }
 
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s)

@@ -180,6 +180,9 @@ cudaError_t launch_plan(const EvictParams& p, int sms, cudaStream_t s);
 // layer), in place, from the evicted sets in half p.ev_plan_parity of lay.evplan: one CTA per
 // (layer, sequence, KV head).
 cudaError_t launch_compact_stack(const EvictParams& p, int layers, cudaStream_t s);
+// The same rounds with order-free slots: the evicted slots of every layer refilled in place from
+// the newest ones, the step's token (p.k_new / p.v_new: [layers][B][KVH][d]) included.
+cudaError_t launch_fill_stack(const EvictParams& p, int layers, cudaStream_t s);
 // One-time attributes; active[cl] (cl = 0..kEvMaxCluster) = clusters of cl CTAs the device runs at once.
 cudaError_t evict_prepare(int* active);
 cudaError_t launch_timeout_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);

@@ -183,3 +183,18 @@ def test_eviction_window_is_the_step_time_beyond_the_attention_bytes():
     assert bench.eviction_window([], evicting) is None and bench.eviction_window(clean, []) is None
     r = bench.eviction_roofline({"evict": _kern(12.0, 68e6, 10)}, 10, {"hbm_gbs": 6000.0}, "measured", None, None, w)
     assert r["windowed"]["frac"] == pytest.approx(w["GBps"] / 6000.0)
+    assert w["resolved"] and w["noise_us_per_round"] == 0.0
+
+
+def test_eviction_window_within_the_clean_steps_noise_is_not_resolved():
+    # clean steps 1.00 / 1.02 ms for 6e9 bytes: the prediction itself is uncertain by ~1%
+    clean = [(1.00, 64, 6e9), (1.02, 64, 6e9)]
+    rate = 2.02 / 12e9
+    evicting = [(5.94e9 * rate + 0.001, 5.94e9, 64, 64 * 1e6)]  # 1 us beyond the prediction
+    w = bench.eviction_window(clean, evicting)
+    sd = 0.01 / 6e9  # the two rates' population spread (ms per byte)
+    assert w["noise_us_per_round"] == pytest.approx(1000.0 * sd * 5.94e9 / 64)
+    assert not w["resolved"] and "GBps" not in w
+    assert w["us_per_round_at_most"] == pytest.approx(1000.0 * (0.001 + 2 * sd * 5.94e9) / 64)
+    r = bench.eviction_roofline({"stack": _kern(14.0, 33e6, 1)}, 64, {"hbm_gbs": 6000.0}, "measured", None, None, w)
+    assert r["windowed"]["frac"] is None

@@ -1,10 +1,13 @@
-"""Evicted sets computed one step ahead (ra_decode_step): the random draw reads no cache data, so
-while a step's attention runs, a kernel on a side stream computes the next step's evicted sets,
-and the eviction on the critical path only moves rows.  Checked against the oracle, bit-exact,
-over several rounds with sequences firing on different steps: every key-per-ordinal policy that
-reads no cache data (random, shared draw, protected recency -- the last through the exact radix
-passes), the exact passes forced for the random draw, and the block policy (whose keys read
-positions, so it keeps the in-step selection).  Attention of the last step within tolerance.
+"""Evicted sets computed one step ahead (ra_decode_step): the random draw needs no cache data but
+positions, so while a step's attention runs, a kernel on a side stream computes the next step's
+evicted sets, and at the firing step one launch moves every layer's rows.  Checked against the
+oracle, bit-exact, over several rounds with sequences firing on different steps, in both layouts:
+- ordered (order-preserving compaction, in place): random, shared draw, protected recency (the
+  exact radix passes), the exact passes forced for the random draw, block draws of 16 positions
+  (keys read positions; ties resolved by the radix sweep);
+- order-free (the evicted slots refilled from the newest rows, the step's token included): keys
+  per position for random, shared, recency and block draws.
+Attention of the last step within tolerance.
 """
 import numpy as np
 import pytest
@@ -67,15 +70,20 @@ def _step_all(run, t):
     return q, out.cpu().numpy(), fired
 
 
-@pytest.mark.parametrize("policy,block,mode", [(0, 1, 0), (1, 1, 0), (2, 1, 0), (0, 1, 256), (3, 16, 0)],
-                         ids=["random", "shared", "recency", "random-exact", "block16-in-step"])
-def test_evicted_sets_computed_ahead_match_the_oracle(policy, block, mode):
+CASES = [(0, 1, 0, 0), (1, 1, 0, 0), (2, 1, 0, 0), (0, 1, 256, 0), (3, 16, 0, 0),
+         (0, 1, 0, 1), (1, 1, 0, 1), (2, 1, 0, 1), (0, 1, 256, 1), (3, 16, 0, 1)]
+IDS = ["random", "shared", "recency", "random-exact", "block16",
+       "orderfree-random", "orderfree-shared", "orderfree-recency", "orderfree-random-exact", "orderfree-block16"]
+
+
+@pytest.mark.parametrize("policy,block,mode,compaction", CASES, ids=IDS)
+def test_evicted_sets_computed_ahead_match_the_oracle(policy, block, mode, compaction):
     import oracle
     import paper_2609_03430_gb300 as ra
 
     K, r = 480, 32
     run = Runner(L=3, H=24, KVH=4, prompt_lens=[40, 0, 17, 300, 5], K=K, r=r, eseed=61 + policy, dseed=62,
-                 policy=policy, block=block)
+                 policy=policy, block=block, compaction=compaction)
     ra.ra_set_eviction_kernel(run.ctx, mode)
     phases = [0, 7, 31, 16, 30]
     _restore_phased(run, phases, epoch=40)
@@ -96,8 +104,6 @@ def test_evicted_sets_computed_ahead_match_the_oracle(policy, block, mode):
                 ref = oracle.attend(q[l, b, h * G:(h + 1) * G], run.krows(l, b, h, pos), run.vrows(l, b, h, pos))
                 check_attention(got[l, b, h * G:(h + 1) * G], ref, f"layer {l} seq {b} head {h}")
     _, n_plan, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_PLAN)
-    if policy == 3:
-        assert n_plan == 0  # block keys read positions: selected in step
-    else:
-        assert n_plan > 0
+    _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
+    assert n_plan > 0 and n_stack > 0
     run.close()
