@@ -1215,9 +1215,12 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
     const int h = item % L.KVH, t = (item / L.KVH) % p.n_trig, layer = item / (L.KVH * p.n_trig);
     const int b = p.trig[t], c = p.trig_c[t], N = p.trig_n[t], g = p.trig_g[t];
     const int m = N - L.K;
-    pdl_wait();  // the buffer rows were written by earlier steps' attention
-    pdl_launch_dependents();
+    // The plan (complete: the stream waited for it), the tables and the prompt length are read
+    // before waiting for the predecessor; the rows and positions it may have written, after.
+    // Every exit waits first, so that no successor starts before the predecessor completes.
     if (m < 1 || m > L.r || m > kEvCap || N > c || c + 1 > L.Cmax) {  // the host rules this out
+        pdl_wait();
+        pdl_launch_dependents();
         if (tid == 0) atomicExch(L.err, kDeviceErrPlan);
         return;
     }
@@ -1225,16 +1228,19 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
         L.evplan + (size_t)((((size_t)p.ev_plan_parity * L.L + layer) * L.B + b) * L.KVH + h) * (L.r + 1);
     if (tid == 0) bad = __ldcg(plan) != m;
     for (int i = tid; i < m; i += kFillThreads) ev[i] = __ldcg(plan + 1 + i);
+    const int reg = L.region[((size_t)layer * L.B + b) * L.KVH + h];
+    const int32_t tok_pos = L.seq_lp[b] + g - 1;
     __syncthreads();
     bool wrong = false;  // the plan: m ordinals, ascending, below N
     for (int i = tid; i < m; i += kFillThreads) wrong = wrong || ev[i] < 0 || ev[i] >= N || (i + 1 < m && ev[i] >= ev[i + 1]);
     if (wrong) bad = 1;
     __syncthreads();
+    pdl_wait();  // the buffer rows were written by earlier steps' attention
+    pdl_launch_dependents();
     if (bad) {  // a bad plan moves nothing
         if (tid == 0) atomicExch(L.err, kDeviceErrPlan);
         return;
     }
-    const int reg = L.region[((size_t)layer * L.B + b) * L.KVH + h];
     const long long row0 = L.gen_row0 + (long long)reg * L.Cmax;
     int32_t* gpos = L.pos + (size_t)reg * L.Cmax;
     const size_t tok = (((size_t)layer * L.B + b) * L.KVH + h) * kHeadDim;
@@ -1254,7 +1260,7 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
                 to[u] = ev[i];
                 if (from == c) {  // the step's token
                     v[u] = reinterpret_cast<const uint4*>((lane < 16 ? p.k_new : p.v_new) + tok)[part];
-                    pv[u] = L.seq_lp[b] + g - 1;
+                    pv[u] = tok_pos;
                 } else {
                     v[u] = reinterpret_cast<const uint4*>(pool + (row0 + from) * kHeadDim)[part];
                     pv[u] = gpos[from];

@@ -151,8 +151,10 @@ def test_eviction_roofline_prices_the_copy_kernel_and_the_round():
     assert r["traffic"] == 70e6 and r["launches"] == 20
     # the fused kernel, when present, is the one priced; order-free select reported beside it
     kern2 = {"evict": _kern(12.0, 68e6, 10)}
-    hole = ({"select": _kern(5.0, 2e6, 10)}, 10)
+    hole = ({"select": _kern(5.0, 2e6, 10), "stack": _kern(14.0, 33e6, 2)}, 10)
     r2 = bench.eviction_roofline(kern2, 10, peaks, "fallback", None, hole)
+    assert r2["holefill_fill"]["achieved"] == pytest.approx(33e6 / 14e-6 / 1e9)
+    assert r2["holefill_fill"]["us_per_round"] == pytest.approx(2.8)
     assert r2["kernel"].startswith("evict_kernel") and r2["peak_source"].startswith("fallback")
     assert r2["round"]["us_per_round"] == pytest.approx(12.0)
     assert r2["holefill_select"]["achieved"] == pytest.approx(2e6 / 5e-6 / 1e9)
