@@ -176,7 +176,8 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block);
  *                       e_0 < ... < e_{m-1} are refilled in place from the m
  *                       newest slots (slot e_i takes slot c - m + i): m <= r
  *                       row moves per head and round, done by the selection
- *                       kernel itself.  ra_get_positions then lists positions
+ *                       kernel itself (in ra_decode_step, for every layer of
+ *                       the firing sequences in one launch).  ra_get_positions then lists positions
  *                       in slot order, which is no longer time order.  In
  *                       ra_decode_layer the step's token, the newest slot, is
  *                       written straight into the evicted slot it refills.
@@ -246,7 +247,8 @@ int ra_set_attention_shape(ra_ctx* ctx, int shape);
  * A value in [2, 16] forces that cluster size (raised to the minimum that holds a head's keys,
  * ceil((K + r) / 2112) CTAs, or to the next size the device can schedule).  Results are
  * identical in every mode.  The scored policy, order-free and in-attention compaction, and
- * buffers of r > 512 always use the selection kernel.
+ * buffers of r > 512 always use the selection kernel in the per-layer calls.  RA_EVICT_TWO_KERNELS
+ * also turns off the sets computed ahead in ra_decode_step, so every round selects in step.
  */
 #define RA_EVICT_AUTO 0
 #define RA_EVICT_TWO_KERNELS 1

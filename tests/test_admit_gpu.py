@@ -35,13 +35,15 @@ def test_finished_slots_take_new_requests(fused):
     run.close()
 
 
-def test_admission_through_the_whole_stack_step():
-    """ra_decode_step (evicted sets computed one step ahead) with admissions between steps."""
+@pytest.mark.parametrize("compaction", [0, 1], ids=["ordered", "orderfree"])
+def test_admission_through_the_whole_stack_step(compaction):
+    """ra_decode_step (evicted sets computed one step ahead) with admissions between steps, in both
+    layouts (order-free: keys per position, read by the plans)."""
     import paper_2609_03430_gb300 as ra
     import synth
 
     run = Runner(L=3, H=16, KVH=4, prompt_lens=[250, 17, 0], K=32, r=16, eseed=73, dseed=74,
-                 prompt_pool=(800, 1800))
+                 prompt_pool=(800, 1800), compaction=compaction)
     dev = run.dev
     for step in range(120):
         if step == 30:
