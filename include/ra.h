@@ -332,8 +332,9 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
  * so a step that fails changes nothing.  Same result as the per-layer calls, by a
  * faster route: the keys of the random policy and its variants (not the scored
  * one) need no cache data beyond positions, so during each step a kernel on a
- * stream of the library's own (forked from and joined to `stream` by events)
- * computes the next step's evicted sets in every layer, and at that step one
+ * stream of the library's own (forked from `stream` at the step's start and
+ * joined to it at its end, by events: once `stream` completes, so has all the
+ * step's work) computes the next step's evicted sets in every layer, and at that step one
  * launch compacts every layer of the sequences that fire (ordered or order-free,
  * in place) before the first layer runs.  Sets computed ahead are used only
  * where the counters they were computed from still hold; elsewhere the layers

@@ -1356,6 +1356,12 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
             break;
     std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
     if (rc != RA_OK) return rc;
+    // Join the side stream at the step's end (the plan finished long before the last layer), so
+    // that once `stream` completes, so has everything the step launched.
+    if (ctx->plan_pending) {
+        if ((e = cudaStreamWaitEvent(s, ctx->plan_ev, 0)) != cudaSuccess) return cuda_fail(ctx, e, "plan join");
+        ctx->plan_pending = false;
+    }
     ctx->parity = nxt;
     return RA_OK;
 }
