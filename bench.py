@@ -543,7 +543,12 @@ TARGET = ("the >= 0.70-of-HBM-bandwidth target is judged on frac, against the me
           "frac_of_nominal_8TBps is the same achieved figure over the nominal 8 TB/s")
 
 
-def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None, windowed=None):
+STACK_FILL = ("fill_stack_kernel (every layer's order-free refill of the m evicted slots per head of the sequences "
+              "firing at a step, in place, one launch per step, from evicted sets computed a step ahead)")
+
+
+def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None, windowed=None,
+                      compaction="ordered"):
     """The bench line's roofline of the eviction: its copy kernel (the fused select + compaction
     kernel when the library ran it, else the compaction kernel) at its algorithmic bytes -- the
     survivors' K, V and position read and written, 2 (2 d 2 + 4) bytes per row -- over its
@@ -557,7 +562,8 @@ def eviction_roofline(kern, rounds, peaks, peak_src, traffic=None, holefill=None
     achieved = k["bytes_per_launch"] / (k["us_per_launch"] * 1e-6) / 1e9
     round_ms = sum(kern[n]["ms_total"] for n in EVICT_KINDS if n in kern)
     round_bytes = sum(kern[n]["bytes_per_launch"] * kern[n]["launches"] for n in EVICT_KINDS if n in kern)
-    out = {"kernel": EVICT_KERNELS[name], "bound": "hbm", "target": TARGET, "achieved": achieved,
+    label = STACK_FILL if (name == "stack" and compaction == "holefill") else EVICT_KERNELS[name]
+    out = {"kernel": label, "bound": "hbm", "target": TARGET, "achieved": achieved,
            "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
            "peak_source": f"{peak_src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
            else "fallback 6.8 TB/s", "frac_of_nominal_8TBps": achieved / 8000.0,
@@ -789,7 +795,7 @@ def run_ours(args, w):
         holefill = run_holefill_variant(args, rank, world, barrier, peaks, ms_step, kern, rounds)
     roof_evict = eviction_roofline(kern, rounds, peaks, peak_src, args.traffic_evict,
                                    (holefill["kernels"], holefill["rounds_in_evented_pass"]) if holefill else None,
-                                   win_evict)
+                                   win_evict, args.compaction)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, budget_s=args.cpu_seconds, rank=0)

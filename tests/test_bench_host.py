@@ -167,6 +167,8 @@ def test_eviction_roofline_prices_the_copy_kernel_and_the_round():
     assert r3["also"]["evict"]["achieved"] == pytest.approx(68e6 / 12e-6 / 1e9)
     assert r3["round"]["us_per_round"] == pytest.approx(720.0 / 74)  # the plan is not in the round
     assert r3["plan"]["launches"] == 2 and "target" in r3
+    r4 = bench.eviction_roofline(kern3, 74, peaks, "measured", compaction="holefill")
+    assert r4["kernel"].startswith("fill_stack_kernel")
     # no eviction in the evented pass: nothing to report
     assert bench.eviction_roofline({"attn": kern["attn"]}, 0, peaks, "measured") is None
 
