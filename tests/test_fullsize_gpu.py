@@ -27,8 +27,8 @@ def _samples(w, n_heads, n_attn, seed):
     return sorted(heads), attn
 
 
-@pytest.mark.parametrize("cfg,compaction", [(2, 0), (3, 0), (4, 0), (5, 0), (5, 1)],
-                         ids=["cfg2", "cfg3", "cfg4", "cfg5", "cfg5-holefill"])
+@pytest.mark.parametrize("cfg,compaction", [(2, 0), (3, 0), (4, 0), (5, 0), (4, 1), (5, 1)],
+                         ids=["cfg2", "cfg3", "cfg4", "cfg5", "cfg4-holefill", "cfg5-holefill"])
 def test_workload_parity_sampled(cfg, compaction):
     import torch
 
