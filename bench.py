@@ -98,16 +98,27 @@ def describe(w):
             f"K={w['K']}, r={w['r']}")
 
 
+def decode_call(ra, ctx, calls, q, k, v, out, stream):
+    """One decode step through the public API: ra_decode_step over the stacked layers, or
+    ra_decode_layer for layers 0 .. L-1 in order (q, k, v, out: [L][...] device tensors)."""
+    if calls == "step":
+        ra.ra_decode_step(ctx, q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), 0.0, stream)
+    else:
+        for l in range(q.shape[0]):
+            ra.ra_decode_layer(ctx, l, q[l].data_ptr(), k[l].data_ptr(), v[l].data_ptr(), out[l].data_ptr(), 0.0, stream)
+
+
 class Workload:
     """Device-side setup of one workload through the public API."""
 
-    def __init__(self, cfg, rank=0, ring=4, policy=0, compaction=0):
+    def __init__(self, cfg, rank=0, ring=4, policy=0, compaction=0, calls="step"):
         import torch
 
         import paper_2609_03430_gb300 as ra
         import synth.gpu as sg
 
         self.torch, self.ra, self.sg = torch, ra, sg
+        self.calls = calls
         self.w = w = WORKLOADS[cfg]
         self.cfg = cfg
         self.L, self.H, self.KVH, self.B, self.K, self.r = w["L"], w["H"], w["KVH"], w["B"], w["K"], w["r"]
@@ -200,8 +211,7 @@ class Workload:
 
     def step(self, t):
         i = t % self.ring
-        self.ra.ra_decode_step(self.ctx, self.q[i].data_ptr(), self.kn[i].data_ptr(), self.vn[i].data_ptr(),
-                               self.out.data_ptr(), 0.0, self.stream)
+        decode_call(self.ra, self.ctx, self.calls, self.q[i], self.kn[i], self.vn[i], self.out, self.stream)
 
     def bytes_per_step(self):
         """Algorithmic cache bytes read by attention in one step (all layers), at the current state."""
@@ -388,7 +398,8 @@ def config_dict(w, args):
                       "sequence's last eviction (spread evenly over [0, r) for equal-length batches, drawn "
                       "for the ragged one)",
             "l2": "inputs larger than L2 (every step streams the whole cache)", "parallelism": f"replicas x{args.gpus}",
-            "policy": getattr(args, "policy", "random"), "compaction": getattr(args, "compaction", "ordered")}
+            "policy": getattr(args, "policy", "random"), "compaction": getattr(args, "compaction", "ordered"),
+            "calls": "ra_decode_layer per layer" if getattr(args, "calls", "step") == "layer" else "ra_decode_step"}
 
 
 # --------------------------------------------------------------------------- GPU run
@@ -689,7 +700,8 @@ def run_ours(args, w):
     else:
         torch.cuda.set_device(0)
     main_policy = POLICY_SNAPKV if args.policy == "snapkv" else 0
-    wl = Workload(args.config, rank=rank, policy=main_policy, compaction=COMPACTIONS[args.compaction])
+    wl = Workload(args.config, rank=rank, policy=main_policy, compaction=COMPACTIONS[args.compaction],
+                  calls=args.calls)
     stream = wl.stream
     ctx = wl.ctx
 
@@ -764,7 +776,7 @@ def run_ours(args, w):
             stream.wait_event(up[i])
             if t >= 2:
                 stream.wait_event(down[i])  # step t - 2's outputs are read back from buffer i
-            ra.ra_decode_step(ctx, dq[i].data_ptr(), dk[i].data_ptr(), dv[i].data_ptr(), do[i].data_ptr(), 0.0, stream)
+            decode_call(ra, ctx, wl.calls, dq[i], dk[i], dv[i], do[i], stream)
             done[i].record(stream)
             with torch.cuda.stream(cs):
                 cs.wait_event(done[i])
@@ -828,6 +840,8 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=256)
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--config", type=int, default=DEFAULT_CONFIG, choices=sorted(WORKLOADS))
+    ap.add_argument("--calls", choices=["step", "layer"], default="step",
+                    help="the public call a step goes through: ra_decode_step, or ra_decode_layer per layer")
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

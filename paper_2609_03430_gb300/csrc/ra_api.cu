@@ -96,6 +96,8 @@ struct ra_ctx {
     int parity = 0;
     bool no_early_once = false;  // the next attention launch follows the whole-stack compaction
     std::vector<uint8_t> stack_done;  // [B] sequences whose token this step's order-free fill wrote
+    bool step_open = false;  // a step's prologue ran (plans launched, stack evicted) and its end has not
+    int step_cur = 0;        // the plan half that step reads
     std::vector<int32_t> plan_g, plan_n;
     // profiling
     bool prof = false;
@@ -1077,17 +1079,10 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
                       uint16_t* out, float scale, void* stream, int plan_parity);
 }
 
-int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
-                    uint16_t* out, float scale, void* stream)
-{
-    return decode_layer_impl(ctx, layer, q, k_new, v_new, out, scale, stream, -1);
-}
-
 namespace {
-// plan_parity >= 0: evicted sets computed ahead into that half of the plan buffer may be used
-// (ra_decode_step, which has ordered the stream after their computation)
-int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
-                      uint16_t* out, float scale, void* stream, int plan_parity)
+// The host-side checks of one fused layer step (before anything changes).
+int check_layer_call(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                     const uint16_t* out)
 {
     int rc;
     if ((rc = check_bound(ctx)) != RA_OK) return rc;
@@ -1099,6 +1094,186 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
         if (ctx->active[b] && ctx->c[base + b] >= ctx->Cmax)
             return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d already caches K + 2r = %d generated tokens", layer, b,
                         ctx->Cmax);
+    return RA_OK;
+}
+
+// The start of a decode step of the whole stack (ra_decode_step, or ra_decode_layer of layer 0):
+// wait for the evicted sets computed during the previous step, launch the next step's on the
+// side stream, and run every layer's round of the sequences that fire now and have those sets,
+// in one launch.  k_all / v_all: the step's rows of every layer, [L][B][KVH][d], when the caller
+// has them all (ra_decode_step); without them only the ordered layout is served, since the
+// order-free fill writes each layer's token itself.
+int step_prologue(ra_ctx* ctx, const uint16_t* k_all, const uint16_t* v_all, cudaStream_t s)
+{
+    cudaError_t e;
+    const bool serve = plan_usable(ctx) && (k_all != nullptr || ctx->compaction == RA_COMPACT_ORDERED);
+    if (ctx->plan_pending) {  // the evicted sets of this step, computed during the previous one
+        if ((e = cudaStreamWaitEvent(s, ctx->plan_ev, 0)) != cudaSuccess) return cuda_fail(ctx, e, "plan wait");
+        ctx->plan_pending = false;
+    }
+    const int cur = ctx->parity, nxt = 1 - cur;
+    std::fill(ctx->plan_g.begin() + (size_t)nxt * ctx->L * ctx->B, ctx->plan_g.begin() + (size_t)(nxt + 1) * ctx->L * ctx->B,
+              -1);
+    if (serve) {
+        // The sequences whose trigger fires at the next step (from layer 0's counters after this
+        // step): their evicted sets in every layer, computed on the side stream beside this step.
+        // The fork orders the plan after the previous step, the last reader of half nxt.
+        EvictParams pp{};
+        pp.lay = ctx->lay;
+        pp.policy = ctx->policy;
+        pp.block = ctx->block;
+        pp.holefill = ctx->compaction == RA_COMPACT_HOLEFILL;
+        pp.ev_exact = (ctx->evict_mode & RA_EVICT_EXACT) ? 1 : 0;
+        pp.ev_plan_parity = nxt;
+        const bool read_pos = keys_read_positions(ctx);
+        int n = 0;
+        for (int b = 0; b < ctx->B; ++b) {
+            if (!ctx->active[b]) continue;
+            const int g1 = ctx->g[b] + 1, c1 = ctx->c[b] + 1;
+            const bool fires = g1 % ctx->r == 0 && c1 - ctx->r > ctx->K;
+            if (fires && read_pos) continue;  // this step rewrites the positions the keys would read
+            const int g2 = g1 + 1, c2 = (fires ? ctx->K + ctx->r : c1) + 1;
+            if (g2 % ctx->r == 0 && c2 - ctx->r > ctx->K && c2 - ctx->r <= ctx->K + ctx->r) {
+                pp.trig[n] = (int16_t)b;
+                pp.trig_admit[n] = (uint16_t)ctx->admits[b];
+                pp.trig_g[n] = g2;
+                pp.trig_n[n] = c2 - ctx->r;
+                ++n;
+            }
+        }
+        if (n > 0) {
+            pp.n_trig = n;
+            if ((e = cudaEventRecord(ctx->fork_ev, s)) != cudaSuccess ||
+                (e = cudaStreamWaitEvent(ctx->side, ctx->fork_ev, 0)) != cudaSuccess)
+                return cuda_fail(ctx, e, "plan fork");
+            {
+                ProfScope ps(ctx, RA_KERNEL_PLAN, 0.0, ctx->side);
+                e = launch_plan(pp, ctx->sms, ctx->side);
+                ps.done();
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "plan launch");
+            if ((e = cudaEventRecord(ctx->plan_ev, ctx->side)) != cudaSuccess) return cuda_fail(ctx, e, "plan record");
+            ctx->plan_pending = true;
+            for (int i = 0; i < n; ++i)
+                for (int l = 0; l < ctx->L; ++l) {
+                    const size_t k = (size_t)nxt * ctx->L * ctx->B + (size_t)l * ctx->B + pp.trig[i];
+                    ctx->plan_g[k] = pp.trig_g[i];
+                    ctx->plan_n[k] = pp.trig_n[i];
+                }
+        }
+    }
+    // The sequences that fire at this step in every layer alike, with every layer's evicted set
+    // computed ahead: all their rounds in one launch, in place, before the first layer.  Ordered:
+    // the survivors move down and the layers then append the token as usual.  Order-free: the
+    // evicted slots are refilled from the newest rows, the step's token included, so the layers
+    // attend with the token already cached.
+    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
+    if (serve) {
+        const bool fill = ctx->compaction == RA_COMPACT_HOLEFILL;
+        EvictParams sp{};
+        sp.lay = ctx->lay;
+        sp.ev_plan_parity = cur;
+        sp.holefill = fill ? 1 : 0;
+        sp.k_new = k_all;
+        sp.v_new = v_all;
+        int n = 0;
+        double moved = 0;
+        for (int b = 0; b < ctx->B; ++b) {
+            if (!ctx->active[b]) continue;
+            const int g = ctx->g[b], c = ctx->c[b];
+            if ((g + 1) % ctx->r != 0 || c + 1 - ctx->r <= ctx->K) continue;
+            bool all = true;
+            for (int l = 0; l < ctx->L && all; ++l) {
+                const size_t i = (size_t)l * ctx->B + b, k = (size_t)cur * ctx->L * ctx->B + i;
+                all = ctx->g[i] == g && ctx->c[i] == c && ctx->plan_g[k] == g + 1 && ctx->plan_n[k] == c + 1 - ctx->r;
+            }
+            if (!all) continue;
+            sp.trig[n] = (int16_t)b;
+            sp.trig_c[n] = c;
+            sp.trig_n[n] = c + 1 - ctx->r;
+            sp.trig_g[n] = g + 1;
+            ++n;
+            // rows moved per head: the survivors below the token (ordered), the m refills (order-free)
+            moved += (double)(fill ? c + 1 - ctx->r - ctx->K : ctx->K + ctx->r - 1) * ctx->KVH * ctx->L;
+        }
+        if (n > 0) {
+            sp.n_trig = n;
+            {
+                ProfScope ps(ctx, RA_KERNEL_STACK, moved * 2.0 * (2 * kRowBytes + 4), s);
+                e = fill ? launch_fill_stack(sp, ctx->L, s) : launch_compact_stack(sp, ctx->L, s);
+                ps.done();
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "whole-stack compaction launch");
+            for (int i = 0; i < n; ++i) {
+                for (int l = 0; l < ctx->L; ++l) {
+                    const size_t k = (size_t)l * ctx->B + sp.trig[i];
+                    if (fill) {  // K + r rows, the token's among them
+                        ctx->c[k] = ctx->K + ctx->r;
+                        ctx->g[k] += 1;
+                    } else {
+                        ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written
+                    }
+                    ctx->nev[k] += 1;
+                }
+                if (fill) ctx->stack_done[sp.trig[i]] = 1;
+            }
+            ctx->no_early_once = true;
+        }
+    }
+    ctx->step_open = true;
+    ctx->step_cur = cur;
+    return RA_OK;
+}
+
+// The end of the step: join the side stream (the plan finished long before the last layer), so
+// that once the caller's stream completes, so has everything the step launched; then the plan
+// halves swap roles.
+int step_epilogue(ra_ctx* ctx, cudaStream_t s)
+{
+    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
+    if (!ctx->step_open) return RA_OK;
+    ctx->step_open = false;
+    ctx->parity = 1 - ctx->step_cur;
+    if (ctx->plan_pending) {
+        const cudaError_t e = cudaStreamWaitEvent(s, ctx->plan_ev, 0);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "plan join");
+        ctx->plan_pending = false;
+    }
+    return RA_OK;
+}
+}  // namespace
+
+int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                    uint16_t* out, float scale, void* stream)
+{
+    // Layers called in order 0 .. L-1 form a step: layer 0 opens it (the evicted sets computed
+    // during the previous step; with ordered compaction every layer's round of the firing
+    // sequences in one launch), layer L-1 closes it.  Any other order is still correct: the
+    // sets computed ahead are used only where the counters they assumed still hold.
+    int rc;
+    if ((rc = check_layer_call(ctx, layer, q, k_new, v_new, out)) != RA_OK) return rc;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (layer == 0) {
+        if (ctx->step_open && (rc = step_epilogue(ctx, s)) != RA_OK) return rc;
+        if ((rc = step_prologue(ctx, nullptr, nullptr, s)) != RA_OK) return rc;
+    }
+    rc = decode_layer_impl(ctx, layer, q, k_new, v_new, out, scale, stream, ctx->step_open ? ctx->step_cur : -1);
+    if (layer == ctx->L - 1 && ctx->step_open) {
+        const int rc_end = step_epilogue(ctx, s);
+        if (rc == RA_OK) rc = rc_end;
+    }
+    return rc;
+}
+
+namespace {
+// plan_parity >= 0: evicted sets computed ahead into that half of the plan buffer may be used
+// (ra_decode_step, which has ordered the stream after their computation)
+int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                      uint16_t* out, float scale, void* stream, int plan_parity)
+{
+    int rc;
+    if ((rc = check_layer_call(ctx, layer, q, k_new, v_new, out)) != RA_OK) return rc;
+    const size_t base = (size_t)layer * ctx->B;
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
     std::vector<uint8_t> appended((size_t)ctx->B, 0);  // sequences whose token the eviction wrote
@@ -1236,134 +1411,14 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
                 return fail(ctx, RA_ERR_CAPACITY, "layer %d seq %d is full (evict not called)", l, b);
     const size_t qs = (size_t)ctx->B * ctx->H * kHeadDim, ks = (size_t)ctx->B * ctx->KVH * kHeadDim;
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e;
-    if (ctx->plan_pending) {  // the evicted sets of this step, computed during the previous one
-        if ((e = cudaStreamWaitEvent(s, ctx->plan_ev, 0)) != cudaSuccess) return cuda_fail(ctx, e, "plan wait");
-        ctx->plan_pending = false;
-    }
-    const int cur = ctx->parity, nxt = 1 - cur;
-    std::fill(ctx->plan_g.begin() + (size_t)nxt * ctx->L * ctx->B, ctx->plan_g.begin() + (size_t)(nxt + 1) * ctx->L * ctx->B,
-              -1);
-    if (plan_usable(ctx)) {
-        // The sequences whose trigger fires at the next step (from layer 0's counters after this
-        // step): their evicted sets in every layer, computed on the side stream beside this step.
-        // The fork orders the plan after the previous step, the last reader of half nxt.
-        EvictParams pp{};
-        pp.lay = ctx->lay;
-        pp.policy = ctx->policy;
-        pp.block = ctx->block;
-        pp.holefill = ctx->compaction == RA_COMPACT_HOLEFILL;
-        pp.ev_exact = (ctx->evict_mode & RA_EVICT_EXACT) ? 1 : 0;
-        pp.ev_plan_parity = nxt;
-        const bool read_pos = keys_read_positions(ctx);
-        int n = 0;
-        for (int b = 0; b < ctx->B; ++b) {
-            if (!ctx->active[b]) continue;
-            const int g1 = ctx->g[b] + 1, c1 = ctx->c[b] + 1;
-            const bool fires = g1 % ctx->r == 0 && c1 - ctx->r > ctx->K;
-            if (fires && read_pos) continue;  // this step rewrites the positions the keys would read
-            const int g2 = g1 + 1, c2 = (fires ? ctx->K + ctx->r : c1) + 1;
-            if (g2 % ctx->r == 0 && c2 - ctx->r > ctx->K && c2 - ctx->r <= ctx->K + ctx->r) {
-                pp.trig[n] = (int16_t)b;
-                pp.trig_admit[n] = (uint16_t)ctx->admits[b];
-                pp.trig_g[n] = g2;
-                pp.trig_n[n] = c2 - ctx->r;
-                ++n;
-            }
-        }
-        if (n > 0) {
-            pp.n_trig = n;
-            if ((e = cudaEventRecord(ctx->fork_ev, s)) != cudaSuccess ||
-                (e = cudaStreamWaitEvent(ctx->side, ctx->fork_ev, 0)) != cudaSuccess)
-                return cuda_fail(ctx, e, "plan fork");
-            {
-                ProfScope ps(ctx, RA_KERNEL_PLAN, 0.0, ctx->side);
-                e = launch_plan(pp, ctx->sms, ctx->side);
-                ps.done();
-            }
-            if (e != cudaSuccess) return cuda_fail(ctx, e, "plan launch");
-            if ((e = cudaEventRecord(ctx->plan_ev, ctx->side)) != cudaSuccess) return cuda_fail(ctx, e, "plan record");
-            ctx->plan_pending = true;
-            for (int i = 0; i < n; ++i)
-                for (int l = 0; l < ctx->L; ++l) {
-                    const size_t k = (size_t)nxt * ctx->L * ctx->B + (size_t)l * ctx->B + pp.trig[i];
-                    ctx->plan_g[k] = pp.trig_g[i];
-                    ctx->plan_n[k] = pp.trig_n[i];
-                }
-        }
-    }
-    // The sequences that fire at this step in every layer alike, with every layer's evicted set
-    // computed ahead: all their rounds in one launch, in place, before the first layer.  Ordered:
-    // the survivors move down and the layers then append the token as usual.  Order-free: the
-    // evicted slots are refilled from the newest rows, the step's token included, so the layers
-    // attend with the token already cached.
-    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
-    if (plan_usable(ctx)) {
-        const bool fill = ctx->compaction == RA_COMPACT_HOLEFILL;
-        EvictParams sp{};
-        sp.lay = ctx->lay;
-        sp.ev_plan_parity = cur;
-        sp.holefill = fill ? 1 : 0;
-        sp.k_new = k_all;
-        sp.v_new = v_all;
-        int n = 0;
-        double moved = 0;
-        for (int b = 0; b < ctx->B; ++b) {
-            if (!ctx->active[b]) continue;
-            const int g = ctx->g[b], c = ctx->c[b];
-            if ((g + 1) % ctx->r != 0 || c + 1 - ctx->r <= ctx->K) continue;
-            bool all = true;
-            for (int l = 0; l < ctx->L && all; ++l) {
-                const size_t i = (size_t)l * ctx->B + b, k = (size_t)cur * ctx->L * ctx->B + i;
-                all = ctx->g[i] == g && ctx->c[i] == c && ctx->plan_g[k] == g + 1 && ctx->plan_n[k] == c + 1 - ctx->r;
-            }
-            if (!all) continue;
-            sp.trig[n] = (int16_t)b;
-            sp.trig_c[n] = c;
-            sp.trig_n[n] = c + 1 - ctx->r;
-            sp.trig_g[n] = g + 1;
-            ++n;
-            // rows moved per head: the survivors below the token (ordered), the m refills (order-free)
-            moved += (double)(fill ? c + 1 - ctx->r - ctx->K : ctx->K + ctx->r - 1) * ctx->KVH * ctx->L;
-        }
-        if (n > 0) {
-            sp.n_trig = n;
-            {
-                ProfScope ps(ctx, RA_KERNEL_STACK, moved * 2.0 * (2 * kRowBytes + 4), s);
-                e = fill ? launch_fill_stack(sp, ctx->L, s) : launch_compact_stack(sp, ctx->L, s);
-                ps.done();
-            }
-            if (e != cudaSuccess) return cuda_fail(ctx, e, "whole-stack compaction launch");
-            for (int i = 0; i < n; ++i) {
-                for (int l = 0; l < ctx->L; ++l) {
-                    const size_t k = (size_t)l * ctx->B + sp.trig[i];
-                    if (fill) {  // K + r rows, the token's among them
-                        ctx->c[k] = ctx->K + ctx->r;
-                        ctx->g[k] += 1;
-                    } else {
-                        ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written
-                    }
-                    ctx->nev[k] += 1;
-                }
-                if (fill) ctx->stack_done[sp.trig[i]] = 1;
-            }
-            ctx->no_early_once = true;
-        }
-    }
+    if (ctx->step_open && (rc = step_epilogue(ctx, s)) != RA_OK) return rc;  // a per-layer step left open
+    if ((rc = step_prologue(ctx, k_all, v_all, s)) != RA_OK) return rc;
     for (int l = 0; l < ctx->L; ++l)
         if ((rc = decode_layer_impl(ctx, l, q_all + l * qs, k_all + l * ks, v_all + l * ks, out_all + l * qs, scale,
-                                    stream, cur)) != RA_OK)
+                                    stream, ctx->step_cur)) != RA_OK)
             break;
-    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
-    if (rc != RA_OK) return rc;
-    // Join the side stream at the step's end (the plan finished long before the last layer), so
-    // that once `stream` completes, so has everything the step launched.
-    if (ctx->plan_pending) {
-        if ((e = cudaStreamWaitEvent(s, ctx->plan_ev, 0)) != cudaSuccess) return cuda_fail(ctx, e, "plan join");
-        ctx->plan_pending = false;
-    }
-    ctx->parity = nxt;
-    return RA_OK;
+    const int rc_end = step_epilogue(ctx, s);
+    return rc != RA_OK ? rc : rc_end;
 }
 
 int ra_get_counters(const ra_ctx* ctx, int seq, int layer, int32_t* g, int32_t* c, int32_t* n_evictions)

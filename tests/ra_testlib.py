@@ -149,6 +149,10 @@ class Runner:
                 self.qsteps[b].append(self.step_idx)
         self.step_scale.append(scale)
         scored = self.policy == oracle.POLICY_SNAPKV
+        # (fused calls: layer 0's call may run every layer's round of the step, so each layer's
+        # evictions are counted from the step's start)
+        start = ([[self.ra.ra_get_counters(self.ctx, b, l)[2] for b in range(self.B)] for l in range(self.L)]
+                 if self.fused else None)
         for l in range(self.L):
             k = np.zeros((self.B, self.KVH, self.D), np.uint16)
             v = np.zeros_like(k)
@@ -166,9 +170,8 @@ class Runner:
             if not scored:
                 nf = sum(1 for b in range(self.B) if self.active[b] and self.orc.evict(b, l))
             if self.fused:
-                before = [self.ra.ra_get_counters(self.ctx, b, l)[2] for b in range(self.B)]
                 self.ra.ra_decode_layer(self.ctx, l, tq.data_ptr(), tk.data_ptr(), tv.data_ptr(), out.data_ptr(), scale)
-                n = sum(self.ra.ra_get_counters(self.ctx, b, l)[2] - before[b] for b in range(self.B))
+                n = sum(self.ra.ra_get_counters(self.ctx, b, l)[2] - start[l][b] for b in range(self.B))
             else:
                 self.ra.ra_append_kv(self.ctx, l, tk.data_ptr(), tv.data_ptr())
                 n = self.ra.ra_evict(self.ctx, l)

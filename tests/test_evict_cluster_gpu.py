@@ -48,12 +48,13 @@ def test_one_launch_eviction_matches_the_oracle(mode, policy, block, fused):
 
 def test_one_launch_eviction_with_many_heads_in_waves():
     """40 sequences x 8 KV heads firing together: 320 heads, more clusters than run at once, so the
-    launch runs in waves; two rounds in a row."""
+    launch runs in waves; two rounds in a row (the separate calls: no sets are computed ahead, so
+    both rounds take the cluster kernel)."""
     import paper_2609_03430_gb300 as ra
 
     K, r = 512, 32
     run = Runner(L=1, H=32, KVH=8, prompt_lens=[7 * (b % 5) for b in range(40)], K=K, r=r, eseed=41, dseed=42,
-                 fused=True)
+                 fused=False)
     run.restore_full(40 * r - 1)
     for _ in range(r + 1):
         run.step()

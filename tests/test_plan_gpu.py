@@ -107,3 +107,27 @@ def test_evicted_sets_computed_ahead_match_the_oracle(policy, block, mode, compa
     _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
     assert n_plan > 0 and n_stack > 0
     run.close()
+
+
+@pytest.mark.parametrize("policy,block", [(0, 1), (3, 16)], ids=["random", "block16"])
+def test_per_layer_calls_in_order_form_steps(policy, block):
+    """ra_decode_layer for layers 0 .. L-1 in order: layer 0's call runs the step's whole-stack
+    eviction from the sets computed during the previous step, exactly as ra_decode_step does.
+    Bit-exact against the oracle, with attention checked on some steps."""
+    import paper_2609_03430_gb300 as ra
+
+    K, r = 480, 32
+    run = Runner(L=3, H=24, KVH=4, prompt_lens=[40, 0, 17, 300, 5], K=K, r=r, eseed=81 + policy, dseed=82,
+                 fused=True, policy=policy, block=block)
+    _restore_phased(run, [0, 7, 31, 16, 30], epoch=40)
+    ra.ra_profile_reset(run.ctx)
+    for t in range(2 * r + 3):
+        run.step(check_attn_layers=(0, 2) if t % 9 == 0 else ())
+        if t % 11 == 0:
+            run.check_state()
+    run.check_state()
+    assert int(run.orc.n_evictions.min()) >= 2
+    _, n_plan, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_PLAN)
+    _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
+    assert n_plan > 0 and n_stack > 0
+    run.close()
