@@ -945,13 +945,15 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
             const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
             uint32_t cnt = 0;  // warp-uniform
             constexpr int kChains = 8;  // independent Philox chains (and position loads) in flight per lane
-            for (int j0 = lane; j0 < N; j0 += kChains * 32) {
+            // (warp-uniform trip count: every lane reaches each ballot, also when N < 32)
+            for (int c0 = 0; c0 < N; c0 += kChains * 32) {
                 uint32_t kq[kChains];
 #pragma unroll
-                for (int q = 0; q < kChains; ++q) kq[q] = plan_key(p, layer, id, N, g, min(j0 + q * 32, N - 1), pos);
+                for (int q = 0; q < kChains; ++q)
+                    kq[q] = plan_key(p, layer, id, N, g, min(c0 + q * 32 + lane, N - 1), pos);
 #pragma unroll
                 for (int q = 0; q < kChains; ++q) {
-                    const int j = j0 + q * 32;
+                    const int j = c0 + q * 32 + lane;
                     const bool pass = j < N && kq[q] >= tau;
                     const uint32_t bits = __ballot_sync(0xffffffffu, pass);
                     const uint32_t at = cnt + __popc(bits & ((1u << lane) - 1u));

@@ -131,3 +131,28 @@ def test_per_layer_calls_in_order_form_steps(policy, block):
     _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
     assert n_plan > 0 and n_stack > 0
     run.close()
+
+
+@pytest.mark.parametrize("compaction", [0, 1], ids=["ordered", "orderfree"])
+def test_evicted_sets_computed_ahead_with_fewer_candidates_than_a_warp(compaction):
+    """K + r < 32 candidates per head (K = 4, r = 8: 12), so a warp's lanes outnumber them."""
+    import oracle
+    import paper_2609_03430_gb300 as ra
+
+    K, r = 4, 8
+    run = Runner(L=2, H=8, KVH=2, prompt_lens=[3, 0, 20], K=K, r=r, eseed=91, dseed=92, compaction=compaction)
+    _restore_phased(run, [0, 3, 7], epoch=6)
+    ra.ra_profile_reset(run.ctx)
+    for t in range(3 * r + 1):
+        q, got, _ = _step_all(run, t)
+        run.check_state()
+    for l in range(run.L):
+        for b in range(run.B):
+            for h in range(run.KVH):
+                pos = run.orc.positions(b, l, h)
+                G = run.G
+                ref = oracle.attend(q[l, b, h * G:(h + 1) * G], run.krows(l, b, h, pos), run.vrows(l, b, h, pos))
+                check_attention(got[l, b, h * G:(h + 1) * G], ref, f"layer {l} seq {b} head {h}")
+    _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
+    assert n_stack > 0
+    run.close()
