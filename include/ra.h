@@ -173,14 +173,19 @@ int ra_set_policy(ra_ctx* ctx, int policy, int block);
  *                       (counter word 0 = its position instead of its ordinal;
  *                       recency keeps the largest positions), so the kept set
  *                       does not depend on the layout.  The m evicted slots
- *                       e_0 < ... < e_{m-1} are refilled in place from the m
- *                       newest slots (slot e_i takes slot c - m + i): m <= r
- *                       row moves per head and round, done by the selection
- *                       kernel itself (in ra_decode_step, for every layer of
- *                       the firing sequences in one launch).  ra_get_positions then lists positions
- *                       in slot order, which is no longer time order.  In
- *                       ra_decode_layer the step's token, the newest slot, is
- *                       written straight into the evicted slot it refills.
+ *                       e_0 < ... < e_{m-1} are refilled in place and the
+ *                       cache shrinks to c - m slots, c counting the step's
+ *                       token: slot e_i takes slot c - m + i for i < m - 1,
+ *                       and the newest row (the token) ends in the new last
+ *                       slot c - m - 1, whose own row, unless e_{m-1} is that
+ *                       slot, fills e_{m-1}.  At most m + 1 <= r + 1 row moves
+ *                       per head and round, done by the selection kernel (in
+ *                       a whole-stack step, for every layer of the firing
+ *                       sequences in one launch); in the fused forms the
+ *                       attention kernel appends the token into the last
+ *                       slot, as in the ordered layout.  ra_get_positions then
+ *                       lists positions in slot order, which is no longer
+ *                       time order.
  *   RA_COMPACT_FUSED    the ordered layout, but in ra_decode_layer the attention
  *                       pass itself does the compaction: it reads each evicting
  *                       head's old region (as it must read every survivor

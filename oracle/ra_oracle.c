@@ -25,8 +25,9 @@
  *     (section 2 "Notation"), grouped-query: a KV head's keep-set serves
  *     every query head of its group (Appendix F).
  *   - Order-free (hole-filling) compaction: keys drawn per position, the
- *     evicted slots refilled from the newest ones (attention is a sum over
- *     the cached set, so slot order carries nothing).
+ *     evicted slots refilled from the newest ones, the newest row kept in the
+ *     last slot (attention is a sum over the cached set, so slot order
+ *     carries nothing).
  *   - The scored comparator (section 2, "Baselines as choices of s"): the
  *     SnapKV score -- attention received from the last w queries, summed
  *     over the query heads of the group, max-pooled over neighbouring
@@ -487,11 +488,15 @@ uint32_t ora_position_key(int policy, uint64_t seed, uint32_t layer, uint32_t se
  * One eviction round with hole-filling compaction.  Same trigger and the same
  * top-K (the K smallest (key, ordinal) among the n = c - r candidates, keys
  * by position).  The m = n - K evicted slots e_0 < ... < e_{m-1} are refilled
- * from the m newest slots: slot e_i takes the row of slot c - m + i; the cache
- * shrinks to c - m slots.  Every other slot keeps its row.  Defined for
- * c <= K + 2r (the cache's capacity), where m <= r and the m newest slots are
- * all buffer slots.  Returns m (0 when the trigger does not fire) and the
- * evicted ordinals, -1 on error.
+ * and the cache shrinks to c - m slots, the newest row (slot c - 1) ending in
+ * the new last slot c - m - 1:
+ *   - slot e_i takes the row of slot c - m + i, for i < m - 1;
+ *   - if e_{m-1} is the new last slot, it takes the newest row; otherwise it
+ *     takes the row of the new last slot, which then takes the newest row.
+ * Every other slot keeps its row.  Defined for c <= K + 2r (the cache's
+ * capacity), where m <= r and slots c - m .. c - 1 are all buffer slots.
+ * Returns m (0 when the trigger does not fire) and the evicted ordinals, -1 on
+ * error.
  */
 int ora_evict_head_holefill(int32_t* gen, int* c, int g, int K, int r, uint64_t seed, int layer, int seq,
                             int kv_heads, int h, int policy, int block, uint32_t admissions, int32_t* evicted_out)
@@ -520,8 +525,16 @@ int ora_evict_head_holefill(int32_t* gen, int* c, int g, int K, int r, uint64_t 
         if (ki < K && keep[ki] == j) ++ki;
         else ev[m++] = j;
     }
+    const int last = cc - m - 1; /* the new last slot */
     for (int i = 0; i < m; ++i) {
-        gen[ev[i]] = gen[cc - m + i];
+        if (i < m - 1) {
+            gen[ev[i]] = gen[cc - m + i];
+        } else if (ev[i] == last) {
+            gen[last] = gen[cc - 1];
+        } else {
+            gen[ev[i]] = gen[last];
+            gen[last] = gen[cc - 1];
+        }
         if (evicted_out) evicted_out[i] = ev[i];
     }
     *c = cc - m;

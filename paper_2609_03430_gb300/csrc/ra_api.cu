@@ -95,7 +95,6 @@ struct ra_ctx {
     bool plan_pending = false;
     int parity = 0;
     bool no_early_once = false;  // the next attention launch follows the whole-stack compaction
-    std::vector<uint8_t> stack_done;  // [B] sequences whose token this step's order-free fill wrote
     bool step_open = false;  // a step's prologue ran (plans launched, stack evicted) and its end has not
     int step_cur = 0;        // the plan half that step reads
     std::vector<int32_t> plan_g, plan_n;
@@ -245,8 +244,7 @@ void fill_active(const ra_ctx* ctx, uint32_t* mask)
 // the cached generated rows plus one for a fused new token; the tiles are cut into one equal
 // chunk per warp.  *slots = rows attended.
 int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_active, int* ctas, double* slots,
-                   int* shape, const std::vector<uint8_t>* appended = nullptr,
-                   const std::vector<int32_t>* old_rows = nullptr)
+                   int* shape, const std::vector<int32_t>* old_rows = nullptr)
 {
     fill_active(ctx, p->active);
     // sequences whose compaction the launch does: their cached rows are the old region's
@@ -254,19 +252,15 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     if (old_rows)
         for (int b = 0; b < ctx->B; ++b)
             if ((*old_rows)[b] >= 0) p->compacting[b >> 5] |= 1u << (b & 31);
-    // fused: every active sequence's token is pending, except those an eviction already appended
+    // fused: every active sequence's token is pending
     for (int i = 0; i < RA_MAX_BATCH / 32; ++i) p->pending[i] = fused ? p->active[i] : 0u;
-    if (fused && appended)
-        for (int b = 0; b < ctx->B; ++b)
-            if ((*appended)[b]) p->pending[b >> 5] &= ~(1u << (b & 31));
     long long acc = 0, rows = 0;
     int na = 0;
     for (int b = 0; b < ctx->B; ++b) {
         const int cached = (old_rows && (*old_rows)[b] >= 0) ? (*old_rows)[b] : ctx->c[(size_t)layer * ctx->B + b];
         const int gen = cached + (int)((p->pending[b >> 5] >> (b & 31)) & 1u);
         p->seq_gen[b] = gen;
-        // generated tokens before this step's (a token an eviction already appended is not counted)
-        p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b] - (appended && (*appended)[b] ? 1 : 0);
+        p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b];  // generated tokens before this step's
         if (ctx->active[b]) {
             rows += (long long)ctx->KVH * (ctx->lp[b] + gen);
             ++na;
@@ -578,7 +572,6 @@ int ra_create_batched(ra_ctx** out, int layers, int q_heads, int kv_heads, int h
     ctx->c.assign((size_t)layers * batch, 0);
     ctx->nev.assign((size_t)layers * batch, 0);
     ctx->active.assign(batch, 1);
-    ctx->stack_done.assign(batch, 0);
     ctx->score_n.assign((size_t)layers * batch, 0);
     *out = ctx;
     return RA_OK;
@@ -1100,13 +1093,12 @@ int check_layer_call(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* 
 // The start of a decode step of the whole stack (ra_decode_step, or ra_decode_layer of layer 0):
 // wait for the evicted sets computed during the previous step, launch the next step's on the
 // side stream, and run every layer's round of the sequences that fire now and have those sets,
-// in one launch.  k_all / v_all: the step's rows of every layer, [L][B][KVH][d], when the caller
-// has them all (ra_decode_step); without them only the ordered layout is served, since the
-// order-free fill writes each layer's token itself.
-int step_prologue(ra_ctx* ctx, const uint16_t* k_all, const uint16_t* v_all, cudaStream_t s)
+// in one launch.  It needs none of the step's rows: in both layouts each layer's attention then
+// appends its token into the last slot, as after an eviction inside the layer's own call.
+int step_prologue(ra_ctx* ctx, cudaStream_t s)
 {
     cudaError_t e;
-    const bool serve = plan_usable(ctx) && (k_all != nullptr || ctx->compaction == RA_COMPACT_ORDERED);
+    const bool serve = plan_usable(ctx);
     if (ctx->plan_pending) {  // the evicted sets of this step, computed during the previous one
         if ((e = cudaStreamWaitEvent(s, ctx->plan_ev, 0)) != cudaSuccess) return cuda_fail(ctx, e, "plan wait");
         ctx->plan_pending = false;
@@ -1163,19 +1155,16 @@ int step_prologue(ra_ctx* ctx, const uint16_t* k_all, const uint16_t* v_all, cud
         }
     }
     // The sequences that fire at this step in every layer alike, with every layer's evicted set
-    // computed ahead: all their rounds in one launch, in place, before the first layer.  Ordered:
-    // the survivors move down and the layers then append the token as usual.  Order-free: the
-    // evicted slots are refilled from the newest rows, the step's token included, so the layers
-    // attend with the token already cached.
-    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
+    // computed ahead: all their rounds in one launch, in place, before the first layer: the
+    // survivors move down (ordered) or the evicted slots are refilled from the newest rows
+    // (order-free), and the layers then append the token as usual.
     if (serve) {
         const bool fill = ctx->compaction == RA_COMPACT_HOLEFILL;
         EvictParams sp{};
         sp.lay = ctx->lay;
         sp.ev_plan_parity = cur;
         sp.holefill = fill ? 1 : 0;
-        sp.k_new = k_all;
-        sp.v_new = v_all;
+        sp.pending = 1;
         int n = 0;
         double moved = 0;
         for (int b = 0; b < ctx->B; ++b) {
@@ -1204,19 +1193,12 @@ int step_prologue(ra_ctx* ctx, const uint16_t* k_all, const uint16_t* v_all, cud
                 ps.done();
             }
             if (e != cudaSuccess) return cuda_fail(ctx, e, "whole-stack compaction launch");
-            for (int i = 0; i < n; ++i) {
+            for (int i = 0; i < n; ++i)
                 for (int l = 0; l < ctx->L; ++l) {
                     const size_t k = (size_t)l * ctx->B + sp.trig[i];
-                    if (fill) {  // K + r rows, the token's among them
-                        ctx->c[k] = ctx->K + ctx->r;
-                        ctx->g[k] += 1;
-                    } else {
-                        ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written
-                    }
+                    ctx->c[k] = ctx->K + ctx->r - 1;  // rows left before the step's token is written (last)
                     ctx->nev[k] += 1;
                 }
-                if (fill) ctx->stack_done[sp.trig[i]] = 1;
-            }
             ctx->no_early_once = true;
         }
     }
@@ -1230,7 +1212,6 @@ int step_prologue(ra_ctx* ctx, const uint16_t* k_all, const uint16_t* v_all, cud
 // halves swap roles.
 int step_epilogue(ra_ctx* ctx, cudaStream_t s)
 {
-    std::fill(ctx->stack_done.begin(), ctx->stack_done.end(), 0);
     if (!ctx->step_open) return RA_OK;
     ctx->step_open = false;
     ctx->parity = 1 - ctx->step_cur;
@@ -1255,7 +1236,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
     cudaStream_t s = (cudaStream_t)stream;
     if (layer == 0) {
         if (ctx->step_open && (rc = step_epilogue(ctx, s)) != RA_OK) return rc;
-        if ((rc = step_prologue(ctx, nullptr, nullptr, s)) != RA_OK) return rc;
+        if ((rc = step_prologue(ctx, s)) != RA_OK) return rc;
     }
     rc = decode_layer_impl(ctx, layer, q, k_new, v_new, out, scale, stream, ctx->step_open ? ctx->step_cur : -1);
     if (layer == ctx->L - 1 && ctx->step_open) {
@@ -1276,7 +1257,6 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
     const size_t base = (size_t)layer * ctx->B;
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
-    std::vector<uint8_t> appended((size_t)ctx->B, 0);  // sequences whose token the eviction wrote
     std::vector<int32_t> old_rows((size_t)ctx->B, -1);  // sequences the attention launch compacts: rows before
     // The attention pass compacts (time order kept) when each tile's evicted rows fit its 64-bit mask.
     const bool fuse_compaction = ctx->compaction == RA_COMPACT_FUSED && ctx->r <= 64;  // tiles have <= 64 rows
@@ -1296,18 +1276,11 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
     // predecessor computes, and with one layer the predecessor is this layer's previous step.
     ep.early = (ctx->policy != RA_POLICY_SNAPKV && ctx->L >= 2) ? 1 : 0;
     const int score_early = ctx->L >= 2 ? 1 : 0;  // the scoring pass reads only older kernels' output
-    if (ep.holefill) {  // the token refills an evicted slot: the select kernel writes it
-        ep.k_new = k_new;
-        ep.v_new = v_new;
-    }
+    ep.pending = 1;  // the step's token is appended by the attention launch below
     int n = 0;
     double moved = 0;
     for (int b = 0; b < ctx->B; ++b) {
         if (!ctx->active[b]) continue;
-        if (!ctx->stack_done.empty() && ctx->stack_done[b]) {  // evicted and appended by this step's fill
-            appended[b] = 1;
-            continue;
-        }
         const int g1 = ctx->g[base + b] + 1, c1 = ctx->c[base + b] + 1;
         if (g1 % ctx->r == 0 && c1 - ctx->r > ctx->K) {
             ep.trig[n] = (int16_t)b;
@@ -1336,17 +1309,11 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
         for (int i = 0; i < n; ++i) {
             const int b = ep.trig[i];
             ctx->nev[base + b] += 1;
-            if (ep.holefill) {  // the token is in the cache already
-                ctx->c[base + b] = ctx->K + ctx->r;
-                ctx->g[base + b] += 1;
-                appended[b] = 1;
-            } else {
-                if (fuse_compaction) {
-                    old_rows[b] = ep.trig_c[i];
-                    compacted += (double)(ctx->K + ctx->r) * ctx->KVH;
-                }
-                ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written
+            if (fuse_compaction) {
+                old_rows[b] = ep.trig_c[i];
+                compacted += (double)(ctx->K + ctx->r) * ctx->KVH;
             }
+            ctx->c[base + b] = ctx->K + ctx->r - 1;  // rows left before the token is written (last)
         }
     }
     // 2. Fused append + attention (+ merge of the split pieces).
@@ -1364,7 +1331,7 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
     int n_active = 0, ctas = 0;
     double rows = 0;
     int shape = kAttnWide;
-    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &shape, &appended, &old_rows)) != RA_OK)
+    if ((rc = plan_attention(ctx, layer, 1, &p, &n_active, &ctas, &rows, &shape, &old_rows)) != RA_OK)
         return rc;
     if (n_active == 0) return RA_OK;
     set_scale(&p, scale);
@@ -1389,7 +1356,7 @@ int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t*
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "attention launch");
     for (int b = 0; b < ctx->B; ++b) {
-        if (!ctx->active[b] || appended[b]) continue;
+        if (!ctx->active[b]) continue;
         ctx->c[base + b] += 1;
         ctx->g[base + b] += 1;
     }
@@ -1412,7 +1379,7 @@ int ra_decode_step(ra_ctx* ctx, const uint16_t* q_all, const uint16_t* k_all, co
     const size_t qs = (size_t)ctx->B * ctx->H * kHeadDim, ks = (size_t)ctx->B * ctx->KVH * kHeadDim;
     cudaStream_t s = (cudaStream_t)stream;
     if (ctx->step_open && (rc = step_epilogue(ctx, s)) != RA_OK) return rc;  // a per-layer step left open
-    if ((rc = step_prologue(ctx, k_all, v_all, s)) != RA_OK) return rc;
+    if ((rc = step_prologue(ctx, s)) != RA_OK) return rc;
     for (int l = 0; l < ctx->L; ++l)
         if ((rc = decode_layer_impl(ctx, l, q_all + l * qs, k_all + l * ks, v_all + l * ks, out_all + l * qs, scale,
                                     stream, ctx->step_cur)) != RA_OK)

@@ -316,17 +316,20 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         }
     }
     if (!p.holefill) return;
-    // Order-free compaction, in place: evicted slot e_i takes the row of slot top - m + i, where
-    // top is the slot count including a pending token (the newest slot, taken from the caller's
-    // rows).  Those m <= r slots are all buffer slots, so sources and destinations never overlap.
+    // Order-free compaction, in place.  With top the slot count including a pending token: evicted
+    // slot e_i takes the row of slot top - m + i for i < m - 1, and the newest row ends in the new
+    // last slot top - m - 1, whose own row, unless e_{m-1} is that slot, fills e_{m-1}.  A pending
+    // token is the newest row: the attention kernel appends it into the new last slot afterwards.
+    // Slots top - m .. top - 1 are buffer slots, so no move reads a slot that another writes.
     if (s_total != (uint32_t)m) return;
-    const int top = p.k_new ? c + 1 : c;
+    const int top = p.pending ? c + 1 : c, last = top - m - 1;
     const long long row0 = L.gen_row0 + (long long)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
     int32_t* gpos = L.pos + (size_t)L.region[((size_t)p.layer * L.B + b) * L.KVH + h] * L.Cmax;
     const int part = lane & 15;
-    uint16_t* pool = lane < 16 ? L.kpool : L.vpool;
+    uint16_t* pool = lane < 16 ? L.kpool : L.vpool;  // lanes 0-15 move K, 16-31 V, 16 bytes each
+    auto row = [&](int slot) { return reinterpret_cast<uint4*>(pool + (row0 + slot) * kHeadDim) + part; };
     constexpr int kWarpsSel = kSelThreads / 32, kBatch = 8;  // rows a warp has in flight
-    for (int i0 = warp; i0 < m; i0 += kWarpsSel * kBatch) {
+    for (int i0 = warp; i0 < m - 1; i0 += kWarpsSel * kBatch) {
         uint4 v[kBatch];
         int32_t pv[kBatch];
         int to[kBatch];
@@ -334,24 +337,39 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         for (int u = 0; u < kBatch; ++u) {  // every load of the batch first ...
             const int i = i0 + u * kWarpsSel;
             to[u] = -1;
-            if (i < m) {
-                const int from = top - m + i;
+            if (i < m - 1) {
                 to[u] = s_ev[i];
-                if (from == c) {  // the step's pending token
-                    const uint16_t* src = (lane < 16 ? p.k_new : p.v_new) + ((size_t)b * L.KVH + h) * kHeadDim;
-                    v[u] = reinterpret_cast<const uint4*>(src)[part];
-                    pv[u] = L.seq_lp[b] + g - 1;
-                } else {
-                    v[u] = reinterpret_cast<const uint4*>(pool + (row0 + from) * kHeadDim)[part];
-                    pv[u] = gpos[from];
-                }
+                v[u] = *row(top - m + i);
+                pv[u] = gpos[top - m + i];
             }
         }
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {  // ... then the stores
             if (to[u] < 0) continue;
-            reinterpret_cast<uint4*>(pool + (row0 + to[u]) * kHeadDim)[part] = v[u];
+            *row(to[u]) = v[u];
             if (lane == 0) gpos[to[u]] = pv[u];
+        }
+    }
+    if (warp == kWarpsSel - 1) {  // the last evicted slot and the new last slot
+        const int e = s_ev[m - 1];
+        const bool fill_e = e != last, newest = !p.pending;
+        uint4 a = make_uint4(0u, 0u, 0u, 0u), n = a;
+        int32_t pa = 0, pn = 0;
+        if (fill_e) {
+            a = *row(last);
+            pa = gpos[last];
+        }
+        if (newest) {
+            n = *row(top - 1);
+            pn = gpos[top - 1];
+        }
+        if (fill_e) {
+            *row(e) = a;
+            if (lane == 0) gpos[e] = pa;
+        }
+        if (newest) {
+            *row(last) = n;
+            if (lane == 0) gpos[last] = pn;
         }
     }
 }
@@ -1202,10 +1220,11 @@ __global__ void __launch_bounds__(kStkThreads) compact_stack_kernel(const __grid
 // ----------------------------------------------------------------------------- fill_stack (order-free, in place)
 // The order-free counterpart of compact_stack_kernel: at the start of a whole-stack step, every
 // layer's round of the sequences that fire, in one launch, from evicted sets computed ahead.  One
-// CTA per (layer, sequence, KV head) refills evicted slot e_i with the row of slot top - m + i, as
-// select_kernel does within a layer: top counts the step's token, the newest of those rows, which
-// comes from the caller's rows of that layer ([layers][batch][kv_heads][d]) with its position.
-// Those m <= r slots are all buffer slots, so sources and destinations never overlap.
+// CTA per (layer, sequence, KV head) moves rows as select_kernel does with the step's token
+// pending: evicted slot e_i takes the row of slot c + 1 - m + i for i < m - 1, and the row of the
+// new last slot c - m, unless e_{m-1} is that slot, fills e_{m-1}; each layer's attention then
+// appends its token into the new last slot.  Slots c - m .. c - 1 are buffer slots, so no move
+// reads a slot that another writes.
 constexpr int kFillThreads = 256;
 
 __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_constant__ EvictParams p)
@@ -1216,11 +1235,11 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int item = blockIdx.x;  // layer-major (layer, sequence, KV head)
     const int h = item % L.KVH, t = (item / L.KVH) % p.n_trig, layer = item / (L.KVH * p.n_trig);
-    const int b = p.trig[t], c = p.trig_c[t], N = p.trig_n[t], g = p.trig_g[t];
+    const int b = p.trig[t], c = p.trig_c[t], N = p.trig_n[t];
     const int m = N - L.K;
-    // The plan (complete: the stream waited for it), the tables and the prompt length are read
-    // before waiting for the predecessor; the rows and positions it may have written, after.
-    // Every exit waits first, so that no successor starts before the predecessor completes.
+    // The plan (complete: the stream waited for it) and the tables are read before waiting for
+    // the predecessor; the rows and positions it may have written, after.  Every exit waits
+    // first, so that no successor starts before the predecessor completes.
     if (m < 1 || m > L.r || m > kEvCap || N > c || c + 1 > L.Cmax) {  // the host rules this out
         pdl_wait();
         pdl_launch_dependents();
@@ -1232,7 +1251,6 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
     if (tid == 0) bad = __ldcg(plan) != m;
     for (int i = tid; i < m; i += kFillThreads) ev[i] = __ldcg(plan + 1 + i);
     const int reg = L.region[((size_t)layer * L.B + b) * L.KVH + h];
-    const int32_t tok_pos = L.seq_lp[b] + g - 1;
     __syncthreads();
     bool wrong = false;  // the plan: m ordinals, ascending, below N
     for (int i = tid; i < m; i += kFillThreads) wrong = wrong || ev[i] < 0 || ev[i] >= N || (i + 1 < m && ev[i] >= ev[i + 1]);
@@ -1246,10 +1264,10 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
     }
     const long long row0 = L.gen_row0 + (long long)reg * L.Cmax;
     int32_t* gpos = L.pos + (size_t)reg * L.Cmax;
-    const size_t tok = (((size_t)layer * L.B + b) * L.KVH + h) * kHeadDim;
-    const int top = c + 1, part = lane & 15;
+    const int top = c + 1, last = c - m, part = lane & 15;
     uint16_t* pool = lane < 16 ? L.kpool : L.vpool;  // lanes 0-15 move K, 16-31 V, 16 bytes each
     constexpr int kWarps = kFillThreads / 32, kBatch = 8;  // rows a warp has in flight
+    // moves i < m - 1: slot top - m + i to e_i; move m - 1: the new last slot to e_{m-1}, if they differ
     for (int i0 = warp; i0 < m; i0 += kWarps * kBatch) {
         uint4 v[kBatch];
         int32_t pv[kBatch];
@@ -1258,16 +1276,11 @@ __global__ void __launch_bounds__(kFillThreads) fill_stack_kernel(const __grid_c
         for (int u = 0; u < kBatch; ++u) {  // every load of the batch first ...
             const int i = i0 + u * kWarps;
             to[u] = -1;
-            if (i < m) {
-                const int from = top - m + i;
+            if (i < m && (i < m - 1 || ev[i] != last)) {
+                const int from = i < m - 1 ? top - m + i : last;
                 to[u] = ev[i];
-                if (from == c) {  // the step's token
-                    v[u] = reinterpret_cast<const uint4*>((lane < 16 ? p.k_new : p.v_new) + tok)[part];
-                    pv[u] = tok_pos;
-                } else {
-                    v[u] = reinterpret_cast<const uint4*>(pool + (row0 + from) * kHeadDim)[part];
-                    pv[u] = gpos[from];
-                }
+                v[u] = reinterpret_cast<const uint4*>(pool + (row0 + from) * kHeadDim)[part];
+                pv[u] = gpos[from];
             }
         }
 #pragma unroll

@@ -72,10 +72,9 @@ struct EvictParams {
     int block;     // RA_POLICY_BLOCK: positions per block
     int holefill;  // RA_COMPACT_HOLEFILL: keys per position, evicted slots refilled in place by select
     int early;     // select may compute before its predecessor finishes (it writes only after the wait)
-    // Fused step under hole-filling: the step's new rows [B][KVH][128] (the token is the newest slot
-    // and always among those that refill the evicted ones); null when the token is already cached.
-    const uint16_t* k_new;
-    const uint16_t* v_new;
+    // Hole-filling with the step's token still pending (the fused step): the cache holds trig_c
+    // rows and the token is appended afterwards, into the new last slot; 0: the token is cached.
+    int pending;
     int n_trig;
     int16_t trig[RA_MAX_BATCH];    // triggered sequence ids
     int32_t trig_c[RA_MAX_BATCH];  // rows in the cache (a pending new token is not among them)

@@ -30,21 +30,27 @@ def test_no_round_without_trigger():
     assert ev.size == 0 and new.size == 56
 
 
-@pytest.mark.parametrize("K,r,c", [(96, 32, 160), (40, 16, 71), (0, 8, 16), (5, 64, 70)])
+@pytest.mark.parametrize("K,r,c", [(96, 32, 160), (40, 16, 71), (0, 8, 16), (5, 64, 70), (3, 2, 7), (5, 1, 7)])
 def test_round_invariants(K, r, c):
-    """Only the evicted slots change, each taking one of the newest slots' rows in order; the
-    cache shrinks by m; the kept set is exactly K candidates plus the whole buffer."""
+    """The evicted slots take the rows of slots c - m .. c - 2 in order, and the newest row ends
+    in the new last slot (whose own row, when kept, fills the last evicted slot); every other
+    slot keeps its row; the cache shrinks by m; the kept set is exactly K candidates plus the
+    whole buffer."""
     rng = np.random.default_rng(K + r)
     gen = np.sort(rng.choice(10_000, size=c, replace=False)).astype(np.int32)
     g = (c // r + 1) * r  # a firing step (g multiple of r)
     new, ev = _round(gen, g, K, r)
     n = c - r
     m = n - K
+    last = c - m - 1
     assert ev.size == m and new.size == c - m
     assert np.all(np.diff(ev) > 0) and (ev.size == 0 or ev[-1] < n)
-    for i, e in enumerate(ev):
+    for i, e in enumerate(ev[:-1]):
         assert new[e] == gen[c - m + i]
-    untouched = np.setdiff1d(np.arange(c - m), ev)
+    assert new[last] == gen[c - 1]  # the newest row is the last
+    if ev[-1] != last:
+        assert new[ev[-1]] == gen[last]
+    untouched = np.setdiff1d(np.arange(c - m), np.append(ev, last))
     np.testing.assert_array_equal(new[untouched], gen[untouched])
     kept_cand = set(gen[:n].tolist()) - set(gen[ev].tolist())
     assert len(kept_cand) == K
@@ -143,4 +149,4 @@ def test_repeated_rounds_keep_distinct_positions():
         if ev.size:
             assert gen.size == K + r and before == K + 2 * r
         assert len(set(gen.tolist())) == gen.size
-        assert gen.max() == lp + g - 1  # the newest token is always cached
+        assert gen[-1] == lp + g - 1  # the newest token is always cached, in the last slot
