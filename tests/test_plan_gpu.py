@@ -156,3 +156,30 @@ def test_evicted_sets_computed_ahead_with_fewer_candidates_than_a_warp(compactio
     _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
     assert n_stack > 0
     run.close()
+
+
+@pytest.mark.parametrize("compaction", [0, 1], ids=["ordered", "orderfree"])
+def test_stacked_and_per_layer_steps_interleaved(compaction):
+    """ra_decode_step and in-order ra_decode_layer steps, alternating in runs of different lengths:
+    the sets computed during one form's step serve the other's, bit-exact against the oracle."""
+    import paper_2609_03430_gb300 as ra
+
+    K, r = 96, 16
+    run = Runner(L=3, H=16, KVH=4, prompt_lens=[12, 0, 40, 7], K=K, r=r, eseed=95, dseed=96, fused=True,
+                 compaction=compaction)
+    _restore_phased(run, [0, 5, 15, 9], epoch=20)
+    ra.ra_profile_reset(run.ctx)
+    forms = ([0] * 3 + [1] * 2 + [0] + [1] * 5) * 6  # 0: the stacked call, 1: per-layer calls
+    for t, form in enumerate(forms[:3 * r + 2]):
+        if form == 0:
+            _step_all(run, t)
+        else:
+            run.step_idx = t
+            run.step()
+        if t % 5 == 0:
+            run.check_state()
+    run.check_state()
+    assert int(run.orc.n_evictions.min()) >= 2
+    _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
+    assert n_stack > 0
+    run.close()
