@@ -92,6 +92,57 @@ def test_workload_parity_sampled(cfg, compaction):
     wl.cache.close()
 
 
+def test_config2_every_head_index_replay():
+    """Config 2 (the Qwen3-4B shape) at full size, every one of its 4 608 (sequence, layer, KV head)
+    units: the oracle replays each head's rounds over r + 2 steps of the benchmark's launch
+    configuration, and every head's surviving positions must match bit-exactly."""
+    import torch
+
+    import bench
+    import oracle
+    import paper_2609_03430_gb300 as ra
+    import synth.gpu as sg
+
+    torch.cuda.set_device(0)
+    wl = bench.Workload(2, ring=1)
+    L, B, H, KVH, K, r, D = wl.L, wl.B, wl.H, wl.KVH, wl.K, wl.r, 128
+    orc = oracle.OracleCache(L, KVH, wl.lp, K, r, wl.eseed)
+    for b in range(B):
+        c, g = wl.c0[b], wl.g0[b]
+        for l in range(L):
+            for h in range(KVH):
+                orc.gen[(b, l, h)] = np.arange(wl.lp[b] + g - c, wl.lp[b] + g, dtype=np.int32)
+            orc.g[b, l] = g
+    dev = wl.dev
+    q = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((L, B, KVH, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    out = torch.empty((L, B, H, D), dtype=torch.int16, device=dev)
+    for t in range(r + 2):
+        qpos = torch.full((B, H, 1), t, dtype=torch.int32, device=dev)
+        npos = torch.tensor([[wl.lp[b] + wl.g0[b] + t] * KVH for b in range(B)], dtype=torch.int32,
+                            device=dev).reshape(B, KVH, 1)
+        for l in range(L):
+            sg.fill_rows(q[l].view(B, H, 1, D), qpos, wl.dseed, 2, l, 0)
+            sg.fill_rows(kn[l].view(B, KVH, 1, D), npos, wl.dseed, 0, l, 0, wl._scale(l))
+            sg.fill_rows(vn[l].view(B, KVH, 1, D), npos, wl.dseed, 1, l, 0)
+        ra.ra_decode_step(wl.ctx, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), out.data_ptr(), 0.0)
+        for b in range(B):
+            for l in range(L):
+                orc.append(b, l)
+                orc.evict(b, l)
+    torch.cuda.synchronize()
+    ra.ra_check_device(wl.ctx)
+    for b in range(B):
+        for l in range(L):
+            g, c, nev = ra.ra_get_counters(wl.ctx, b, l)
+            assert g == orc.g[b, l] and nev == 1  # every head evicted once in the window
+            for h in range(KVH):
+                got = ra.ra_get_positions(wl.ctx, l, b, h, K + 2 * r)
+                np.testing.assert_array_equal(got, orc.gen[(b, l, h)], err_msg=f"positions {(b, l, h)}")
+    wl.cache.close()
+
+
 def test_scored_comparator_parity_full_size():
     """The scored comparator at the ragged workload's full size (the configuration bench.py times it
     in): query window restored, r + 2 steps so that every sequence scores once; sampled heads' raw
