@@ -1248,7 +1248,7 @@ int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k
 
 namespace {
 // plan_parity >= 0: evicted sets computed ahead into that half of the plan buffer may be used
-// (ra_decode_step, which has ordered the stream after their computation)
+// (inside a step whose prologue has ordered the stream after their computation)
 int decode_layer_impl(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
                       uint16_t* out, float scale, void* stream, int plan_parity)
 {
