@@ -279,13 +279,13 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
     }
     if (acc >= (1LL << 31)) return fail(ctx, RA_ERR_UNSUPPORTED, "layer holds more than 2^31 tiles");
     p->total = (int)acc;
-    const int wpc = attn_warps_per_cta(*shape, ctx->G);
-    const long long nwarps_max = (long long)ctx->sms * wpc;
+    const int wpc = attn_warps_per_cta(*shape, ctx->G), cps = attn_ctas_per_sm(*shape);
+    const long long nwarps_max = (long long)ctx->sms * cps * wpc;
     const long long W = std::max<long long>(1, (acc + nwarps_max - 1) / nwarps_max);
     const long long nchunks = (acc + W - 1) / W;
     p->W = (int)W;
     p->nchunks = (int)nchunks;
-    *ctas = (int)std::min<long long>(ctx->sms, (nchunks + wpc - 1) / wpc);
+    *ctas = (int)std::min<long long>((long long)ctx->sms * cps, (nchunks + wpc - 1) / wpc);
     p->nwarps = *ctas * wpc;
     *n_active = na;
     *slots = (double)rows;
@@ -327,7 +327,8 @@ int layout_base(ra_ctx* ctx)
     ctx->off_plan = take((size_t)batch * kv_heads * (kPlanHeader + r) * 4);
     // chunks of the attention split: one per warp
     const size_t max_chunks =
-        (size_t)kMaxSMs * std::max(attn_warps_per_cta(kAttnWide, ctx->G), attn_warps_per_cta(kAttnNarrow, ctx->G)) + 1;
+        (size_t)kMaxSMs * std::max(attn_warps_per_cta(kAttnWide, ctx->G) * attn_ctas_per_sm(kAttnWide),
+                                   attn_warps_per_cta(kAttnNarrow, ctx->G) * attn_ctas_per_sm(kAttnNarrow)) + 1;
     ctx->partial_records = max_chunks + (size_t)batch * kv_heads;
     ctx->off_partial = take(ctx->partial_records * partial_stride(ctx->G) * 4);
     ctx->off_arrive = take((size_t)batch * kv_heads * 4);

@@ -224,6 +224,12 @@ inline int attn_warps_per_cta(int shape, int G)
 {
     return shape == kAttnNarrow ? attn_narrow::attn_warps_per_cta(G) : attn_wide::attn_warps_per_cta(G);
 }
+// CTAs of a shape that one SM holds at once (the narrow build may be split into several smaller
+// CTAs, so that an SM frees part of its shared memory for the next layer as each CTA finishes).
+#ifndef RA_ATTN_NARROW_CTAS
+#define RA_ATTN_NARROW_CTAS 1
+#endif
+inline int attn_ctas_per_sm(int shape) { return shape == kAttnNarrow ? RA_ATTN_NARROW_CTAS : 1; }
 inline int attn_tile_rows(int shape, int G)
 {
     return shape == kAttnNarrow ? attn_narrow::attn_tile_rows(G) : attn_wide::attn_tile_rows(G);
