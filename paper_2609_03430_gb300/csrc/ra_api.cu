@@ -261,6 +261,13 @@ int plan_attention(ra_ctx* ctx, int layer, int fused, AttnParams* p, int* n_acti
         const int gen = cached + (int)((p->pending[b >> 5] >> (b & 31)) & 1u);
         p->seq_gen[b] = gen;
         p->seq_g[b] = ctx->g[(size_t)layer * ctx->B + b];  // generated tokens before this step's
+        p->seq_lp[b] = ctx->lp[b];
+        p->seq_region[b] = ctx->rbase[(size_t)layer * ctx->B + b];
+        const int32_t* pg = ctx->pages.data() + (size_t)b * ctx->max_pages;
+        const int np = (ctx->lp[b] + kPromptPage - 1) / kPromptPage;
+        bool consecutive = true;
+        for (int j = 1; j < np && consecutive; ++j) consecutive = pg[j] == pg[0] + j;
+        p->seq_page0[b] = np == 0 ? 0 : (consecutive ? pg[0] : -1);
         if (ctx->active[b]) {
             rows += (long long)ctx->KVH * (ctx->lp[b] + gen);
             ++na;

@@ -129,7 +129,8 @@ struct TileIter {
     int lp, gen;                     // prompt rows, generated rows (incl. a fused new token)
     bool comp;                       // the head compacts in this launch: its generated rows are the old region's
     long long pbase, grow;           // the head's prompt rows: pbase + page * KVH * kPromptPage + offset; first generated row
-    const int32_t* ptab;             // the sequence's page table
+    const int32_t* ptab;             // the sequence's page table (null: its pages are page0, page0 + 1, ...)
+    int page0;
     int pg_i, pg_cur, pg_next;       // page-table entry i of the current prompt tile, and entry i + 1 (read ahead)
     bool piece_start;
 };
@@ -148,19 +149,20 @@ template <bool COMPACT>
 __device__ __forceinline__ void enter_head(TileIter& it, const AttnParams& p)
 {
     const DevLayout& L = p.lay;
-    it.lp = L.seq_lp[it.b];
+    it.lp = p.seq_lp[it.b];
     it.gen = p.seq_gen[it.b];
     it.tp = (it.lp + p.tile - 1) / p.tile;
     it.pbase = prompt_row(L, p.layer, 0, it.h, 0);
-    it.ptab = L.pages + (size_t)it.b * L.max_pages;
+    it.page0 = p.seq_page0[it.b];
+    it.ptab = it.page0 >= 0 ? nullptr : L.pages + (size_t)it.b * L.max_pages;
     it.pg_i = 0;
     if (it.lp > 0) {
-        it.pg_cur = __ldg(it.ptab);
-        it.pg_next = it.lp > kPromptPage ? __ldg(it.ptab + 1) : 0;
+        it.pg_cur = it.ptab ? __ldg(it.ptab) : it.page0;
+        it.pg_next = it.lp > kPromptPage ? (it.ptab ? __ldg(it.ptab + 1) : it.page0 + 1) : 0;
     }
     it.comp = COMPACT && ((p.compacting[it.b >> 5] >> (it.b & 31)) & 1u);
     const int reg = it.comp ? L.plan[(size_t)(it.b * L.KVH + it.h) * (kPlanHeader + L.r)]  // the old region
-                            : L.region[((size_t)p.layer * L.B + it.b) * L.KVH + it.h];
+                            : p.seq_region[it.b] * L.KVH + it.h;
     it.grow = L.gen_row0 + (long long)reg * L.Cmax;
     it.piece_start = true;
 }
@@ -205,9 +207,9 @@ __device__ bool iter_next(TileIter& it, const AttnParams& p, TileDesc& d, int wa
     if (it.k < it.tp) {  // a prompt tile lies inside one page (kPromptPage is a multiple of T)
         const int p0 = it.k * T, pi = p0 / kPromptPage;
         if (pi != it.pg_i) {  // another page: the next one's entry was read ahead (a chunk may start mid-prompt)
-            it.pg_cur = pi == it.pg_i + 1 ? it.pg_next : __ldg(it.ptab + pi);
+            it.pg_cur = pi == it.pg_i + 1 ? it.pg_next : (it.ptab ? __ldg(it.ptab + pi) : it.page0 + pi);
             it.pg_i = pi;
-            it.pg_next = (pi + 1) * kPromptPage < it.lp ? __ldg(it.ptab + pi + 1) : 0;
+            it.pg_next = (pi + 1) * kPromptPage < it.lp ? (it.ptab ? __ldg(it.ptab + pi + 1) : it.page0 + pi + 1) : 0;
         }
         d.row = it.pbase + (long long)it.pg_cur * p.lay.KVH * kPromptPage + p0 % kPromptPage;
         d.n = min(T, it.lp - p0);
@@ -550,7 +552,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
             if (!(COMPACT && (hd.y & kCompact))) {  // (a compacting head writes it with its survivors)
                 const long long row = (long long)hd.w + n - 1;
                 reinterpret_cast<uint4*>((lane < 16 ? p.lay.kpool : p.lay.vpool) + row * kHeadDim)[c] = v;
-                if (lane == 0) p.lay.pos[row - p.lay.gen_row0] = p.lay.seq_lp[b] + p.seq_g[b];
+                if (lane == 0) p.lay.pos[row - p.lay.gen_row0] = p.seq_lp[b] + p.seq_g[b];
             }
             __syncwarp();
         }
@@ -819,7 +821,7 @@ __global__ void __launch_bounds__(Cfg<G>::WARPS * 32, 1)
                 if (evicted(jj)) continue;
                 const int b = hd.z / p.lay.KVH;
                 const bool newtok = (hd.y & kNewTok) && jj == n - 1;
-                dpos[dest(jj)] = newtok ? p.lay.seq_lp[b] + p.seq_g[b] : __ldg(spos + j0 + jj);
+                dpos[dest(jj)] = newtok ? p.seq_lp[b] + p.seq_g[b] : __ldg(spos + j0 + jj);
             }
         }
 

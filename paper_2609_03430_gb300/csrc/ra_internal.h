@@ -127,6 +127,12 @@ struct AttnParams {
     int32_t seq_base[RA_MAX_BATCH + 1];  // KVH * prefix of tiles per head over active sequences
     int32_t seq_gen[RA_MAX_BATCH];       // generated rows attended per head (incl. a fused new token)
     int32_t seq_g[RA_MAX_BATCH];         // tokens generated before this step's (fused) / up to it (separate)
+    // From the host mirror, so that entering a head needs no load from memory: the prompt length,
+    // the first prompt page when the sequence's pages are consecutive (-1: walk the page table), and
+    // this layer's region base (the region of KV head h is base * KVH + h)
+    int32_t seq_lp[RA_MAX_BATCH];
+    int32_t seq_page0[RA_MAX_BATCH];
+    int32_t seq_region[RA_MAX_BATCH];
     uint32_t pending[RA_MAX_BATCH / 32]; // fused step: sequences whose new token this kernel appends
     // fused step: sequences that evicted this step and whose compaction this kernel does -- it reads
     // their old regions (plan header), masks the evicted rows and writes every survivor (and the new
