@@ -326,10 +326,11 @@ int ra_decode_attn(ra_ctx* ctx, int layer, const uint16_t* q, uint16_t* out, flo
  * new token, and merges its own split pieces.  k_new, v_new: device
  * [batch][kv_heads][head_dim]; q, out: device [batch][q_heads][head_dim].
  * RA_ERR_CAPACITY as for ra_append_kv.  Layers called in order 0 .. layers-1
- * form a step, as in ra_decode_step: with ordered compaction, layer 0's call
- * also runs every layer's round of the sequences that fire, from evicted sets
- * computed during the previous step (same result as each layer evicting in
- * its own call), and layer layers-1's call joins the library's stream back.
+ * form a step, as in ra_decode_step: with ordered or order-free compaction and
+ * a policy other than the scored one, layer 0's call also runs every layer's
+ * round of the sequences that fire, from evicted sets computed during the
+ * previous step (same result as each layer evicting in its own call), and
+ * layer layers-1's call joins the library's stream back.
  */
 int ra_decode_layer(ra_ctx* ctx, int layer, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
                     uint16_t* out, float scale, void* stream);
