@@ -686,6 +686,21 @@ def run_holefill_variant(args, rank, world, barrier, peaks, ordered_ms, ordered_
             "rounds_in_evented_pass": rounds, "kernels": kern}
 
 
+def run_per_layer_variant(args, rank, world, barrier, stacked_ms):
+    """The same step through the per-layer call a real model makes (ra_decode_layer for layers
+    0 .. L-1 in order: layer 0's call opens the step), on the same caches rebuilt from the same
+    seeds, timed like the main run."""
+    wl = Workload(args.config, rank=rank, compaction=COMPACTIONS[args.compaction], calls="layer")
+    for t in range(args.warmup):
+        wl.step(t)
+    wl.ra.ra_check_device(wl.ctx)
+    ms, _, _, _ = timed_steps(wl, args.steps, args.warmup, barrier)
+    ms_step, units = reduce_over_ranks(ms, float(wl.B), world)
+    wl.cache.close()
+    return {"calls": "ra_decode_layer per layer, in layer order", "value": units / (ms_step * 1e-3), "unit": UNIT,
+            "ms_per_step": ms_step, "step_time_vs_stacked": ms_step / stacked_ms}
+
+
 def run_ours(args, w):
     import torch
 
@@ -805,6 +820,9 @@ def run_ours(args, w):
     holefill = None
     if main_policy == 0 and args.compaction == "ordered" and args.variants == "on":
         holefill = run_holefill_variant(args, rank, world, barrier, peaks, ms_step, kern, rounds)
+    per_layer = None
+    if main_policy == 0 and args.calls == "step" and args.variants == "on":
+        per_layer = run_per_layer_variant(args, rank, world, barrier, ms_step)
     roof_evict = eviction_roofline(kern, rounds, peaks, peak_src, args.traffic_evict,
                                    (holefill["kernels"], holefill["rounds_in_evented_pass"]) if holefill else None,
                                    win_evict, args.compaction)
@@ -826,6 +844,8 @@ def run_ours(args, w):
             line["comparator"] = comparator
         if holefill is not None:
             line["holefill_variant"] = holefill
+        if per_layer is not None:
+            line["per_layer_variant"] = per_layer
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
