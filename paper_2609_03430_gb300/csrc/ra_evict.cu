@@ -962,7 +962,8 @@ __global__ void __launch_bounds__(32) plan_kernel(const __grid_constant__ EvictP
             const uint64_t E = 2ull * (uint64_t)m + 32ull;
             const uint32_t tau = E >= (uint64_t)N ? 0u : (uint32_t)(((uint64_t)(N - E) << 32) / (uint64_t)N);
             uint32_t cnt = 0;  // warp-uniform
-            constexpr int kChains = 8;  // independent Philox chains (and position loads) in flight per lane
+            // independent Philox chains (and position loads) in flight per lane: 4 measured faster than 8
+            constexpr int kChains = 4;
             // (warp-uniform trip count: every lane reaches each ballot, also when N < 32)
             for (int c0 = 0; c0 < N; c0 += kChains * 32) {
                 uint32_t kq[kChains];
