@@ -183,3 +183,22 @@ def test_stacked_and_per_layer_steps_interleaved(compaction):
     _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
     assert n_stack > 0
     run.close()
+
+
+@pytest.mark.parametrize("compaction", [0, 1], ids=["ordered", "orderfree"])
+def test_evicted_sets_computed_ahead_with_the_largest_buffer(compaction):
+    """r = 512, the largest buffer the sets computed ahead serve: each round evicts 512 per head, more
+    than the sampled cut's list holds, so the plan kernel takes its exact radix passes."""
+    import paper_2609_03430_gb300 as ra
+
+    K, r = 1024, 512
+    run = Runner(L=2, H=8, KVH=2, prompt_lens=[5, 0, 30], K=K, r=r, eseed=97, dseed=98, compaction=compaction)
+    _restore_phased(run, [r - 4, r - 11, r - 21], epoch=6)  # each fires within 21 steps, planned a step ahead
+    ra.ra_profile_reset(run.ctx)
+    for t in range(24):
+        _step_all(run, t)
+    run.check_state()
+    assert int(run.orc.n_evictions.min()) >= 1
+    _, n_stack, _ = ra.ra_profile_read(run.ctx, ra.RA_KERNEL_STACK)
+    assert n_stack == 3
+    run.close()
